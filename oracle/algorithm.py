@@ -1,0 +1,67 @@
+"""Algorithm 1 (Hier-AVG, Sec. 3.1) driven over P simulated learners.
+
+State: a list of learner-indexed arrays (each with leading axis P).  One global
+round is
+
+    for b in 0 .. beta-1:            (beta = K2 here: local averages per round)
+        for k in 1 .. K1:  every learner j takes one local SGD step
+        local average within every cluster of S learners
+    global average over all P learners (every learner is then synchronised)
+
+The global step counter t counts local SGD steps from 0 and continues across
+rounds.  Reading of "randomly sample a mini-batch": the per-learner data are i.i.d.
+draws, so learner j at step t takes rows (t*B + s) mod N, s = 0..B-1, of its own
+data set.
+"""
+from __future__ import annotations
+
+from typing import List
+
+import numpy as np
+
+from .averaging import global_average, local_average
+from .learner import sgd_update
+
+
+def batch_rows(t: int, B: int, N: int) -> np.ndarray:
+    """Row indices of the mini-batch at local step t."""
+    return (t * B + np.arange(B)) % N
+
+
+class HierAvgOracle:
+    def __init__(self, P: int, S: int, K1: int, K2: int, lr: float, problem,
+                 params: List[np.ndarray], mode: str = "fp32"):
+        if min(P, S, K1, K2) < 1 or P % S != 0:
+            raise ValueError("need P, S, K1, K2 >= 1 and S | P")
+        for p in params:
+            if p.shape[0] != P:
+                raise ValueError("every parameter array must have leading axis P")
+        self.P, self.S, self.K1, self.K2, self.lr = P, S, K1, K2, lr
+        self.problem, self.mode = problem, mode
+        dt = np.float64 if mode == "f64" else np.float32
+        self.params = [np.array(p, dtype=dt, copy=True) for p in params]
+        self.t = 0
+
+    def step(self) -> None:
+        """One local SGD step on every learner (Algorithm 1, innermost loop)."""
+        for j in range(self.P):
+            pj = [p[j] for p in self.params]
+            grads = self.problem.gradients(j, self.t, pj)
+            for p, g in zip(self.params, grads):
+                p[j] = sgd_update(p[j], g, self.lr, self.mode)
+        self.t += 1
+
+    def local_average(self) -> None:
+        for p in self.params:
+            local_average(p, self.S)
+
+    def global_average(self) -> None:
+        for p in self.params:
+            global_average(p)
+
+    def round(self) -> None:
+        for _b in range(self.K2):
+            for _k in range(self.K1):
+                self.step()
+            self.local_average()
+        self.global_average()
