@@ -1,0 +1,286 @@
+// Local and global averages of Algorithm 1 (Sec. 3.1) over a learner-indexed
+// fp32 matrix w[P, ld]: in-memory segmented / full means over the learner axis.
+//
+// Each thread owns one 16-byte column slice (4 consecutive parameters) and walks
+// the n rows of its cluster (or of all P learners): loads are 128-bit and a warp
+// reads 512 contiguous bytes per row, so every row access is fully coalesced.
+// The sum over rows follows the canonical adjacent-pair tree (v[i] += v[i+h] for
+// h = 1, 2, 4, ..., unpaired elements carried up), evaluated as a streaming binary
+// counter: pushing value i combines it with the pending partials of the same
+// size, exactly like incrementing a binary number, so only log2(n)+1 partials
+// live in registers.  Then one IEEE division by n and a broadcast write-back.
+// The arithmetic is __fadd_rn / __fdiv_rn only (no FMA, no flush to zero), so the
+// result is bit-identical to the CPU definition of the same tree.
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "internal.h"
+
+namespace ha {
+namespace {
+
+__device__ __forceinline__ float vadd(float a, float b) { return __fadd_rn(a, b); }
+__device__ __forceinline__ float4 vadd(float4 a, float4 b) {
+  return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z),
+                     __fadd_rn(a.w, b.w));
+}
+__device__ __forceinline__ float vdiv(float a, float n) { return __fdiv_rn(a, n); }
+__device__ __forceinline__ float4 vdiv(float4 a, float n) {
+  return make_float4(__fdiv_rn(a.x, n), __fdiv_rn(a.y, n), __fdiv_rn(a.z, n),
+                     __fdiv_rn(a.w, n));
+}
+
+// Sum of the 2^LOG consecutive rows starting at p (row stride ld_v in vectors).
+template <int LOG, class V>
+__device__ __forceinline__ V tree_pow2(const V* __restrict__ p, int64_t ld_v) {
+  constexpr int N = 1 << LOG;
+  V stack[LOG + 1];
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
+    V x = p[static_cast<int64_t>(i) * ld_v];
+    int l = 0;
+#pragma unroll
+    for (; l < LOG; ++l) {
+      if (((i >> l) & 1) == 0) break;
+      x = vadd(stack[l], x);
+    }
+    stack[l] = x;
+  }
+  return stack[LOG];
+}
+
+template <class V>
+__device__ __forceinline__ void store_rows(V* p, int64_t ld_v, int n, V m) {
+#pragma unroll 8
+  for (int i = 0; i < n; ++i) p[static_cast<int64_t>(i) * ld_v] = m;
+}
+
+// Group means, n = 2^LOG rows per group; grid.y = group index.
+template <int LOG>
+__global__ void __launch_bounds__(256) k_mean_pow2(float4* __restrict__ w, int64_t ld_v,
+                                                   int64_t cols_v) {
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (c >= cols_v) return;
+  float4* p = w + static_cast<int64_t>(blockIdx.y) * (int64_t(1) << LOG) * ld_v + c;
+  const float4 m = vdiv(tree_pow2<LOG>(p, ld_v), static_cast<float>(1 << LOG));
+  store_rows(p, ld_v, 1 << LOG, m);
+}
+
+// Fused last local average + global average: G = 2^LOGG clusters of S = 2^LOGS.
+// The global tree runs over the P values the local average would have written
+// (S copies of each cluster mean, in learner order), so the result is the literal
+// two-pass result: the S equal copies of a cluster form one complete sub-tree of
+// the global tree, whose value is the cluster mean added to itself LOGS times.
+template <int LOGS, int LOGG>
+__global__ void __launch_bounds__(256) k_local_global_pow2(float4* __restrict__ w,
+                                                           int64_t ld_v, int64_t cols_v) {
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (c >= cols_v) return;
+  constexpr int S = 1 << LOGS, G = 1 << LOGG;
+  float4* p = w + c;
+  float4 stack[LOGG + 1];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    float4 x = vdiv(tree_pow2<LOGS>(p + static_cast<int64_t>(g) * S * ld_v, ld_v),
+                    static_cast<float>(S));
+#pragma unroll
+    for (int l = 0; l < LOGS; ++l) x = vadd(x, x);
+    int l = 0;
+#pragma unroll
+    for (; l < LOGG; ++l) {
+      if (((g >> l) & 1) == 0) break;
+      x = vadd(stack[l], x);
+    }
+    stack[l] = x;
+  }
+  const float4 m = vdiv(stack[LOGG], static_cast<float>(S * G));
+  store_rows(p, ld_v, S * G, m);
+}
+
+// Generic path: any n (also non-powers of two) and scalar columns.  The binary
+// counter lives in a small local array; after n pushes its pending partials are
+// the set bits of n, folded from the smallest upward.
+template <class V>
+__device__ V tree_any(const V* __restrict__ p, int64_t ld_v, int n) {
+  V stack[32];
+  for (int i = 0; i < n; ++i) {
+    V x = p[static_cast<int64_t>(i) * ld_v];
+    int l = 0;
+    while ((i >> l) & 1) {
+      x = vadd(stack[l], x);
+      ++l;
+    }
+    stack[l] = x;
+  }
+  V acc{};
+  bool have = false;
+  for (int l = 0; l < 32; ++l) {
+    if ((n >> l) & 1) {
+      acc = have ? vadd(stack[l], acc) : stack[l];
+      have = true;
+    }
+  }
+  return acc;
+}
+
+template <class V>
+__global__ void __launch_bounds__(256) k_mean_any(V* __restrict__ w, int64_t ld_v,
+                                                  int64_t cols_v, int n) {
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (c >= cols_v) return;
+  V* p = w + static_cast<int64_t>(blockIdx.y) * n * ld_v + c;
+  const V m = vdiv(tree_any(p, ld_v, n), static_cast<float>(n));
+  store_rows(p, ld_v, n, m);
+}
+
+template <class V>
+__global__ void __launch_bounds__(256) k_local_global_any(V* __restrict__ w, int64_t ld_v,
+                                                          int64_t cols_v, int S, int G) {
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (c >= cols_v) return;
+  V* p = w + c;
+  V stack[32];
+  int64_t i = 0;   // index of the next pushed value of the global sequence
+  for (int g = 0; g < G; ++g) {
+    const V m = vdiv(tree_any(p + static_cast<int64_t>(g) * S * ld_v, ld_v, S),
+                     static_cast<float>(S));
+    for (int r = 0; r < S; ++r, ++i) {
+      V x = m;
+      int l = 0;
+      while ((i >> l) & 1) {
+        x = vadd(stack[l], x);
+        ++l;
+      }
+      stack[l] = x;
+    }
+  }
+  const int n = S * G;
+  V acc{};
+  bool have = false;
+  for (int l = 0; l < 32; ++l) {
+    if ((n >> l) & 1) {
+      acc = have ? vadd(stack[l], acc) : stack[l];
+      have = true;
+    }
+  }
+  store_rows(p, ld_v, n, vdiv(acc, static_cast<float>(n)));
+}
+
+constexpr int kThreads = 256;
+
+int ilog2_exact(int64_t n) {
+  if (n < 1 || (n & (n - 1)) != 0) return -1;
+  int l = 0;
+  while ((int64_t(1) << l) < n) ++l;
+  return l;
+}
+
+template <int LOG>
+void launch_mean_pow2(float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
+                      cudaStream_t s) {
+  dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
+            static_cast<unsigned>(groups));
+  k_mean_pow2<LOG><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v);
+}
+
+bool mean_pow2_dispatch(int log, float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
+                        cudaStream_t s) {
+  switch (log) {
+    case 1: launch_mean_pow2<1>(w, ld_v, cols_v, groups, s); return true;
+    case 2: launch_mean_pow2<2>(w, ld_v, cols_v, groups, s); return true;
+    case 3: launch_mean_pow2<3>(w, ld_v, cols_v, groups, s); return true;
+    case 4: launch_mean_pow2<4>(w, ld_v, cols_v, groups, s); return true;
+    case 5: launch_mean_pow2<5>(w, ld_v, cols_v, groups, s); return true;
+    case 6: launch_mean_pow2<6>(w, ld_v, cols_v, groups, s); return true;
+    case 7: launch_mean_pow2<7>(w, ld_v, cols_v, groups, s); return true;
+    default: return false;
+  }
+}
+
+template <int LOGS, int LOGG>
+void launch_lg(float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
+  dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
+  k_local_global_pow2<LOGS, LOGG><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v);
+}
+
+template <int LOGS>
+bool lg_dispatch_g(int logg, float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
+  if (logg == 0) { launch_lg<LOGS, 0>(w, ld_v, cols_v, s); return true; }
+  if constexpr (LOGS + 1 <= 7) if (logg == 1) { launch_lg<LOGS, 1>(w, ld_v, cols_v, s); return true; }
+  if constexpr (LOGS + 2 <= 7) if (logg == 2) { launch_lg<LOGS, 2>(w, ld_v, cols_v, s); return true; }
+  if constexpr (LOGS + 3 <= 7) if (logg == 3) { launch_lg<LOGS, 3>(w, ld_v, cols_v, s); return true; }
+  if constexpr (LOGS + 4 <= 7) if (logg == 4) { launch_lg<LOGS, 4>(w, ld_v, cols_v, s); return true; }
+  if constexpr (LOGS + 5 <= 7) if (logg == 5) { launch_lg<LOGS, 5>(w, ld_v, cols_v, s); return true; }
+  if constexpr (LOGS + 6 <= 7) if (logg == 6) { launch_lg<LOGS, 6>(w, ld_v, cols_v, s); return true; }
+  return false;
+}
+
+bool lg_dispatch(int logs, int logg, float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
+  switch (logs) {
+    case 1: return lg_dispatch_g<1>(logg, w, ld_v, cols_v, s);
+    case 2: return lg_dispatch_g<2>(logg, w, ld_v, cols_v, s);
+    case 3: return lg_dispatch_g<3>(logg, w, ld_v, cols_v, s);
+    case 4: return lg_dispatch_g<4>(logg, w, ld_v, cols_v, s);
+    case 5: return lg_dispatch_g<5>(logg, w, ld_v, cols_v, s);
+    default: return false;
+  }
+}
+
+template <class V>
+void launch_mean_any(V* w, int64_t ld_v, int64_t cols_v, int n, int64_t groups,
+                     cudaStream_t s) {
+  dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
+            static_cast<unsigned>(groups));
+  k_mean_any<V><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v, n);
+}
+
+template <class V>
+void launch_lg_any(V* w, int64_t ld_v, int64_t cols_v, int S, int G, cudaStream_t s) {
+  dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
+  k_local_global_any<V><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v, S, G);
+}
+
+}  // namespace
+
+// Vector path for the 16-byte aligned bulk, scalar generic path for the tail.
+static bool vec_ok(const float* w, int64_t ld) {
+  return (reinterpret_cast<uintptr_t>(w) % 16 == 0) && (ld % 4 == 0);
+}
+
+cudaError_t launch_group_mean(float* w, int64_t P, int64_t n, int64_t D, int64_t ld,
+                              cudaStream_t s) {
+  if (D == 0 || n == 1) return cudaSuccess;   // a mean of one row is that row
+  const int64_t groups = P / n;
+  int64_t head = 0;
+  if (vec_ok(w, ld) && D >= 4) {
+    head = D & ~int64_t(3);
+    float4* w4 = reinterpret_cast<float4*>(w);
+    const int log = ilog2_exact(n);
+    if (!(log >= 1 && mean_pow2_dispatch(log, w4, ld / 4, head / 4, groups, s)))
+      launch_mean_any<float4>(w4, ld / 4, head / 4, static_cast<int>(n), groups, s);
+  }
+  if (head < D) launch_mean_any<float>(w + head, ld, D - head, static_cast<int>(n), groups, s);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, int64_t ld,
+                                     cudaStream_t s) {
+  if (D == 0) return cudaSuccess;
+  // S = 1: the local average is the identity, so the pair is one global mean.
+  // (S = P is NOT shortcut: the literal second pass re-averages P equal copies.)
+  if (S == 1) return launch_group_mean(w, P, P, D, ld, s);
+  const int64_t G = P / S;
+  int64_t head = 0;
+  if (vec_ok(w, ld) && D >= 4) {
+    head = D & ~int64_t(3);
+    float4* w4 = reinterpret_cast<float4*>(w);
+    const int logs = ilog2_exact(S), logg = ilog2_exact(G);
+    if (!(logs >= 1 && logg >= 0 && lg_dispatch(logs, logg, w4, ld / 4, head / 4, s)))
+      launch_lg_any<float4>(w4, ld / 4, head / 4, static_cast<int>(S), static_cast<int>(G), s);
+  }
+  if (head < D)
+    launch_lg_any<float>(w + head, ld, D - head, static_cast<int>(S), static_cast<int>(G), s);
+  return cudaGetLastError();
+}
+
+}  // namespace ha

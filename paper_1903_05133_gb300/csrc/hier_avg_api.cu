@@ -1,0 +1,648 @@
+// C ABI of the Hier-AVG hot path (declared in include/hier_avg.h): argument
+// validation, the parameter and workspace layout, TMA descriptor construction,
+// and the order of kernel launches that makes one local step, one local / global
+// average and one round of Algorithm 1 (Sec. 3.1).
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "internal.h"
+
+namespace {
+
+using ha::TcBwdArgs;
+using ha::TcFwdArgs;
+
+constexpr int64_t kAlign = 1024;
+int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+struct ProfRec {
+  int kind;
+  cudaEvent_t a, b;
+  double bytes;
+};
+
+}  // namespace
+
+struct hier_avg {
+  // configuration (Sec. 2 notation)
+  int P = 0, S = 0, K1 = 0, K2 = 0, B = 0, L = 0, prec = 0;
+  float lr = 0.f;
+  std::vector<int> dims;
+  // parameter row layout
+  int64_t D = 0, ld = 0;
+  std::vector<int64_t> woff, boff;
+  // workspace layout
+  int Bn = 0, Kp = 0;
+  std::vector<int> pitch;                       // per width index l = 0..L
+  std::vector<int64_t> off_H, off_HT, off_dZ, off_dZT;
+  int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
+  // binding
+  bool bound = false;
+  int device = 0;
+  float* params = nullptr;
+  uint8_t* ws = nullptr;
+  const void* X = nullptr;
+  const int32_t* y = nullptr;
+  int64_t N = 0;
+  cudaStream_t stream = nullptr;
+  std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_ht, tm_dz, tm_dzt;
+  int64_t t = 0;
+  // profiling
+  bool prof = false;
+  std::vector<ProfRec> recs;
+  std::vector<cudaEvent_t> pool;
+  size_t pool_used = 0;
+  std::string err;
+
+  int fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    err = buf;
+    return code;
+  }
+  int cuda(cudaError_t e, const char* what) {
+    if (e == cudaSuccess) return HA_OK;
+    return fail(HA_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+  }
+  template <class T>
+  T* wsp(int64_t off) { return reinterpret_cast<T*>(ws + off); }
+  int* err_word() { return wsp<int>(off_err); }
+  float* loss() { return wsp<float>(off_loss); }
+
+  cudaEvent_t ev() {
+    if (pool_used == pool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[pool_used++];
+  }
+  // Bracket one launch with events when profiling is on.
+  template <class F>
+  int timed(int kind, double bytes, F&& launch, const char* what) {
+    cudaEvent_t a = nullptr, b = nullptr;
+    if (prof) {
+      a = ev();
+      b = ev();
+      if (a && b) cudaEventRecord(a, stream);
+    }
+    const cudaError_t e = launch();
+    if (e != cudaSuccess) return cuda(e, what);
+    if (prof && a && b) {
+      cudaEventRecord(b, stream);
+      recs.push_back({kind, a, b, bytes});
+    }
+    return HA_OK;
+  }
+};
+
+namespace {
+
+bool valid_handle(const hier_avg* h) { return h != nullptr; }
+
+int plan_layout(hier_avg* h) {
+  const int L = h->L;
+  int64_t pos = 0;
+  h->woff.assign(L, 0);
+  h->boff.assign(L, 0);
+  h->D = 0;
+  for (int l = 0; l < L; ++l) {
+    const int64_t in = h->dims[l], out = h->dims[l + 1];
+    h->woff[l] = pos;
+    pos = round_up(pos + in * out, 64);
+    h->boff[l] = pos;
+    pos = round_up(pos + out, 64);
+    h->D += in * out + out;
+  }
+  h->ld = round_up(pos, 64);
+
+  const int64_t P = h->P, B = h->B;
+  int64_t off = 0;
+  auto take = [&](int64_t bytes) {
+    const int64_t o = off;
+    off = round_up(off + bytes, kAlign);
+    return o;
+  };
+  h->off_H.assign(L + 1, 0);
+  h->off_HT.assign(L + 1, 0);
+  h->off_dZ.assign(L + 1, 0);
+  h->off_dZT.assign(L + 1, 0);
+  h->pitch.assign(L + 1, 0);
+  if (h->prec == HA_PREC_BF16) {
+    h->Bn = static_cast<int>(round_up(B, 16));
+    h->Kp = 64;
+    for (int l = 0; l <= L; ++l) h->pitch[l] = static_cast<int>(round_up(h->dims[l], 64));
+    for (int l = 0; l < L; ++l) {
+      h->off_H[l] = take(P * h->Bn * h->pitch[l] * 2);
+      h->off_HT[l] = take(P * h->dims[l] * h->Kp * 2);
+    }
+    for (int l = 1; l <= L; ++l) {
+      h->off_dZ[l] = take(P * h->Bn * h->pitch[l] * 2);
+      h->off_dZT[l] = take(P * h->dims[l] * h->Kp * 2);
+    }
+  } else {
+    for (int l = 0; l <= L; ++l) h->pitch[l] = h->dims[l];
+    for (int l = 0; l < L; ++l) h->off_H[l] = take(P * B * h->dims[l] * 4);
+    for (int l = 1; l <= L; ++l) h->off_dZ[l] = take(P * B * h->dims[l] * 4);
+  }
+  h->off_Z = take(P * B * h->dims[L] * 4);
+  h->off_loss = take(P * 4);
+  h->off_err = take(16);
+  h->ws_bytes = off;
+  return HA_OK;
+}
+
+int make_map(hier_avg* h, CUtensorMap* m, CUtensorMapDataType dt, void* base, uint64_t d0,
+             uint64_t d1, uint64_t d2, uint64_t s1_bytes, uint64_t s2_bytes, uint32_t b0,
+             uint32_t b1, CUtensorMapSwizzle sw) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return h->fail(HA_ECUDA, "cuTensorMapEncodeTiled is unavailable");
+  const cuuint64_t dims[3] = {d0, d1, d2};
+  const cuuint64_t strides[2] = {s1_bytes, s2_bytes};
+  const cuuint32_t box[3] = {b0, b1, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = enc(m, dt, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return h->fail(HA_ECUDA, "cuTensorMapEncodeTiled failed (%d) for dims %llu x %llu x %llu",
+                   static_cast<int>(r), (unsigned long long)d0, (unsigned long long)d1,
+                   (unsigned long long)d2);
+  return HA_OK;
+}
+
+int build_maps(hier_avg* h) {
+  const int L = h->L;
+  h->tm_wf.resize(L);
+  h->tm_wb.resize(L);
+  h->tm_h.resize(L);
+  h->tm_ht.resize(L);
+  h->tm_dz.resize(L + 1);
+  h->tm_dzt.resize(L + 1);
+  const uint64_t P = h->P, Bn = h->Bn, Kp = h->Kp;
+  int rc;
+  for (int l = 0; l < L; ++l) {
+    const uint64_t in = h->dims[l], out = h->dims[l + 1];
+    float* W = h->params + h->woff[l];
+    if ((rc = make_map(h, &h->tm_wf[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
+                       h->ld * 4, 64, 128, CU_TENSOR_MAP_SWIZZLE_NONE)))
+      return rc;
+    if ((rc = make_map(h, &h->tm_wb[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
+                       h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
+      return rc;
+    const uint64_t pin = h->pitch[l];
+    if ((rc = make_map(h, &h->tm_h[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_H[l], pin,
+                       Bn, P, pin * 2, Bn * pin * 2, 64, static_cast<uint32_t>(Bn),
+                       CU_TENSOR_MAP_SWIZZLE_128B)))
+      return rc;
+    if ((rc = make_map(h, &h->tm_ht[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_HT[l], Kp,
+                       in, P, Kp * 2, in * Kp * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B)))
+      return rc;
+  }
+  for (int l = 1; l <= L; ++l) {
+    const uint64_t d = h->dims[l], pd = h->pitch[l];
+    if ((rc = make_map(h, &h->tm_dz[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_dZ[l], pd,
+                       Bn, P, pd * 2, Bn * pd * 2, 64, static_cast<uint32_t>(Bn),
+                       CU_TENSOR_MAP_SWIZZLE_128B)))
+      return rc;
+    if ((rc = make_map(h, &h->tm_dzt[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_dZT[l],
+                       Kp, d, P, Kp * 2, d * Kp * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)))
+      return rc;
+  }
+  return HA_OK;
+}
+
+int check_bound(hier_avg* h) {
+  if (!h) return HA_EINVAL;
+  if (!h->bound) return h->fail(HA_ESTATE, "hier_avg_bind has not been called");
+  cudaSetDevice(h->device);
+  return HA_OK;
+}
+
+// Algorithmic bytes of the big kernels (fp32 master read + write, activations).
+double bytes_forward(const hier_avg* h, int l) {
+  const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
+  const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
+  return P * (in * out * 4.0 + out * 4.0 + B * in * act + B * out * (l + 1 == h->L ? 4.0 : 2 * act));
+}
+double bytes_backward(const hier_avg* h, int l) {
+  const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
+  const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
+  const double dx = l > 0 ? (B * in * act * 2 + in * 8.0) : 0.0;
+  return P * (in * out * 8.0 + B * in * act + 2 * B * out * act + dx);
+}
+
+int do_step(hier_avg* h) {
+  const int L = h->L, P = h->P, B = h->B;
+  cudaStream_t s = h->stream;
+  int rc;
+  if (h->prec == HA_PREC_BF16) {
+    const int d0 = h->dims[0];
+    rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, [&] {
+      return ha::launch_gather_bf16(static_cast<const __nv_bfloat16*>(h->X), h->N, d0, B, h->Bn,
+                                    h->Kp, h->pitch[0], h->t, P, h->wsp<__nv_bfloat16>(h->off_H[0]),
+                                    h->wsp<__nv_bfloat16>(h->off_HT[0]), s);
+    }, "gather");
+    if (rc) return rc;
+    for (int l = 0; l < L; ++l) {
+      TcFwdArgs a{};
+      a.in = h->dims[l];
+      a.out = h->dims[l + 1];
+      a.B = B;
+      a.Bn = h->Bn;
+      a.Kp = h->Kp;
+      a.ld = h->ld;
+      a.bias = h->params + h->boff[l];
+      a.relu = l + 1 < L;
+      if (a.relu) {
+        a.h_out = h->wsp<__nv_bfloat16>(h->off_H[l + 1]);
+        a.pitch_out = h->pitch[l + 1];
+        a.ht_out = h->wsp<__nv_bfloat16>(h->off_HT[l + 1]);
+      } else {
+        a.z_out = h->wsp<float>(h->off_Z);
+      }
+      a.err = h->err_word();
+      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), [&] {
+        return ha::launch_tc_forward(h->tm_wf[l], h->tm_h[l], a, P, s);
+      }, "forward");
+      if (rc) return rc;
+    }
+    const int C = h->dims[L];
+    rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
+      return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, h->Kp, C,
+                                  h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
+                                  h->wsp<__nv_bfloat16>(h->off_dZ[L]),
+                                  h->wsp<__nv_bfloat16>(h->off_dZT[L]), h->loss(), P, s);
+    }, "xent");
+    if (rc) return rc;
+    for (int l = L - 1; l >= 0; --l) {
+      TcBwdArgs a{};
+      a.in = h->dims[l];
+      a.out = h->dims[l + 1];
+      a.B = B;
+      a.Bn = h->Bn;
+      a.Kp = h->Kp;
+      a.ld = h->ld;
+      a.lr = h->lr;
+      a.has_dx = l > 0;
+      if (a.has_dx) {
+        a.bias_prev = h->params + h->boff[l - 1];
+        a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[l]);
+        a.pitch_in = h->pitch[l];
+        a.dzt_prev = h->wsp<__nv_bfloat16>(h->off_dZT[l]);
+      }
+      a.err = h->err_word();
+      rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+        return ha::launch_tc_backward(h->tm_wb[l], h->tm_ht[l], h->tm_dz[l + 1], h->tm_dzt[l + 1],
+                                      a, P, s);
+      }, "backward");
+      if (rc) return rc;
+    }
+  } else {
+    const int d0 = h->dims[0];
+    rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 4 * 2, [&] {
+      return ha::launch_gather_f32(static_cast<const float*>(h->X), h->N, d0, B, h->t, P,
+                                   h->wsp<float>(h->off_H[0]), s);
+    }, "gather");
+    if (rc) return rc;
+    for (int l = 0; l < L; ++l) {
+      const bool last = l + 1 == L;
+      float* outp = last ? h->wsp<float>(h->off_Z) : h->wsp<float>(h->off_H[l + 1]);
+      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), [&] {
+        return ha::launch_fwd_f32(h->wsp<float>(h->off_H[l]), h->params + h->woff[l],
+                                  h->params + h->boff[l], h->ld, h->dims[l], h->dims[l + 1], B,
+                                  last ? 0 : 1, outp, P, s);
+      }, "forward");
+      if (rc) return rc;
+    }
+    rc = h->timed(HA_KERNEL_XENT, double(P) * B * h->dims[L] * 4 * 2, [&] {
+      return ha::launch_xent_f32(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->dims[L],
+                                 h->wsp<float>(h->off_dZ[L]), h->loss(), P, s);
+    }, "xent");
+    if (rc) return rc;
+    for (int l = L - 1; l >= 0; --l) {
+      rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+        cudaError_t e = cudaSuccess;
+        if (l > 0)
+          e = ha::launch_dx_f32(h->wsp<float>(h->off_dZ[l + 1]), h->params + h->woff[l], h->ld,
+                                h->wsp<float>(h->off_H[l]), h->dims[l], h->dims[l + 1], B,
+                                h->wsp<float>(h->off_dZ[l]), P, s);
+        if (e != cudaSuccess) return e;
+        return ha::launch_dw_update_f32(h->wsp<float>(h->off_dZ[l + 1]), h->wsp<float>(h->off_H[l]),
+                                        h->params + h->woff[l], h->params + h->boff[l], h->ld,
+                                        h->dims[l], h->dims[l + 1], B, h->lr, P, s);
+      }, "backward");
+      if (rc) return rc;
+    }
+  }
+  ++h->t;
+  return HA_OK;
+}
+
+int do_local(hier_avg* h) {
+  return h->timed(HA_KERNEL_LOCAL_AVG, 8.0 * h->P * h->ld, [&] {
+    return ha::launch_group_mean(h->params, h->P, h->S, h->ld, h->ld, h->stream);
+  }, "local average");
+}
+
+int do_local_global(hier_avg* h) {
+  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, [&] {
+    return ha::launch_local_global_mean(h->params, h->P, h->S, h->ld, h->ld, h->stream);
+  }, "local+global average");
+}
+
+int do_round(hier_avg* h) {
+  int rc;
+  for (int b = 0; b < h->K2; ++b) {
+    for (int k = 0; k < h->K1; ++k)
+      if ((rc = do_step(h))) return rc;
+    if (b + 1 < h->K2 && (rc = do_local(h))) return rc;
+  }
+  return do_local_global(h);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* hier_avg_strerror(int status) {
+  switch (status) {
+    case HA_OK: return "ok";
+    case HA_EINVAL: return "invalid argument";
+    case HA_ENOMEM: return "buffer too small";
+    case HA_ECUDA: return "CUDA error";
+    case HA_ESTATE: return "call out of order";
+    case HA_ETIMEOUT: return "device-side wait timed out";
+    case HA_EUNSUPPORTED: return "unsupported configuration";
+    default: return "unknown status";
+  }
+}
+
+const char* hier_avg_last_error(const hier_avg* h) { return h ? h->err.c_str() : "null handle"; }
+
+static int check_avg_args(const float* w, int64_t P, int64_t S, int64_t D, int64_t ld) {
+  if (P < 1 || S < 1 || P % S != 0 || D < 0 || ld < D) return HA_EINVAL;
+  if (D > 0 && !w) return HA_EINVAL;
+  if (P > (int64_t(1) << 30) || D > (int64_t(1) << 40)) return HA_EINVAL;
+  return HA_OK;
+}
+
+int hier_avg_local_average_buffer(float* w_dev, int64_t P, int64_t S, int64_t D, int64_t ld,
+                                  void* stream) {
+  if (int rc = check_avg_args(w_dev, P, S, D, ld)) return rc;
+  return ha::launch_group_mean(w_dev, P, S, D, ld, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? HA_OK
+             : HA_ECUDA;
+}
+
+int hier_avg_global_average_buffer(float* w_dev, int64_t P, int64_t D, int64_t ld, void* stream) {
+  if (int rc = check_avg_args(w_dev, P, 1, D, ld)) return rc;
+  return ha::launch_group_mean(w_dev, P, P, D, ld, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? HA_OK
+             : HA_ECUDA;
+}
+
+int hier_avg_local_global_average_buffer(float* w_dev, int64_t P, int64_t S, int64_t D,
+                                         int64_t ld, void* stream) {
+  if (int rc = check_avg_args(w_dev, P, S, D, ld)) return rc;
+  return ha::launch_local_global_mean(w_dev, P, S, D, ld, static_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? HA_OK
+             : HA_ECUDA;
+}
+
+int hier_avg_create(int P, int S, int K1, int K2, float lr, int B, const int* dims, int n_dims,
+                    int precision, hier_avg** out) {
+  if (!out) return HA_EINVAL;
+  *out = nullptr;
+  if (P < 1 || S < 1 || K1 < 1 || K2 < 1 || B < 1 || P % S != 0) return HA_EINVAL;
+  if (!std::isfinite(lr) || !dims || n_dims < 2 || n_dims > 64) return HA_EINVAL;
+  if (precision != HA_PREC_FP32 && precision != HA_PREC_BF16) return HA_EINVAL;
+  for (int l = 0; l < n_dims; ++l)
+    if (dims[l] < 1 || dims[l] > (1 << 20)) return HA_EINVAL;
+  if (P > 65535) return HA_EUNSUPPORTED;   // learner index is a grid dimension
+  if (precision == HA_PREC_BF16) {
+    if (B > 64) return HA_EUNSUPPORTED;
+    for (int l = 0; l + 1 < n_dims; ++l)
+      if (dims[l] % 8 != 0) return HA_EUNSUPPORTED;
+  }
+  hier_avg* h = new (std::nothrow) hier_avg();
+  if (!h) return HA_ENOMEM;
+  h->P = P;
+  h->S = S;
+  h->K1 = K1;
+  h->K2 = K2;
+  h->B = B;
+  h->lr = lr;
+  h->prec = precision;
+  h->dims.assign(dims, dims + n_dims);
+  h->L = n_dims - 1;
+  plan_layout(h);
+  *out = h;
+  return HA_OK;
+}
+
+void hier_avg_destroy(hier_avg* h) {
+  if (!h) return;
+  for (cudaEvent_t e : h->pool) cudaEventDestroy(e);
+  delete h;
+}
+
+int hier_avg_param_layout(const hier_avg* h, int64_t* D, int64_t* ld, int64_t* offsets) {
+  if (!valid_handle(h)) return HA_EINVAL;
+  if (D) *D = h->D;
+  if (ld) *ld = h->ld;
+  if (offsets)
+    for (int l = 0; l < h->L; ++l) {
+      offsets[2 * l] = h->woff[l];
+      offsets[2 * l + 1] = h->boff[l];
+    }
+  return HA_OK;
+}
+
+int hier_avg_workspace_bytes(const hier_avg* h, int64_t* bytes) {
+  if (!valid_handle(h) || !bytes) return HA_EINVAL;
+  *bytes = h->ws_bytes;
+  return HA_OK;
+}
+
+int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t workspace_bytes,
+                  const void* X_dev, const int32_t* y_dev, int64_t N, void* stream) {
+  if (!h) return HA_EINVAL;
+  h->bound = false;
+  if (!params_dev || !workspace_dev || !X_dev || !y_dev || N < 1)
+    return h->fail(HA_EINVAL, "bind: NULL buffer or N < 1");
+  if (reinterpret_cast<uintptr_t>(params_dev) % 256 || reinterpret_cast<uintptr_t>(workspace_dev) % 256)
+    return h->fail(HA_EINVAL, "bind: params and workspace must be 256-byte aligned");
+  if (h->prec == HA_PREC_BF16 && reinterpret_cast<uintptr_t>(X_dev) % 16)
+    return h->fail(HA_EINVAL, "bind: X must be 16-byte aligned");
+  if (workspace_bytes < h->ws_bytes)
+    return h->fail(HA_ENOMEM, "bind: workspace needs %lld bytes, got %lld",
+                   (long long)h->ws_bytes, (long long)workspace_bytes);
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, params_dev) != cudaSuccess || attr.type != cudaMemoryTypeDevice)
+    return h->fail(HA_EINVAL, "bind: params is not device memory");
+  h->device = attr.device;
+  cudaSetDevice(h->device);
+  h->params = params_dev;
+  h->ws = static_cast<uint8_t*>(workspace_dev);
+  h->X = X_dev;
+  h->y = y_dev;
+  h->N = N;
+  h->stream = static_cast<cudaStream_t>(stream);
+  h->t = 0;
+  int rc;
+  if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_bytes, h->stream), "bind: memset"))) return rc;
+  if (h->prec == HA_PREC_BF16) {
+    if ((rc = h->cuda(ha::tc_configure(), "bind: kernel attributes"))) return rc;
+    if ((rc = build_maps(h))) return rc;
+  }
+  h->bound = true;
+  return HA_OK;
+}
+
+int hier_avg_step(hier_avg* h) {
+  if (int rc = check_bound(h)) return rc;
+  return do_step(h);
+}
+
+int hier_avg_local_average(hier_avg* h) {
+  if (int rc = check_bound(h)) return rc;
+  return do_local(h);
+}
+
+int hier_avg_global_average(hier_avg* h) {
+  if (int rc = check_bound(h)) return rc;
+  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, [&] {
+    return ha::launch_group_mean(h->params, h->P, h->P, h->ld, h->ld, h->stream);
+  }, "global average");
+}
+
+int hier_avg_round(hier_avg* h) {
+  if (int rc = check_bound(h)) return rc;
+  return do_round(h);
+}
+
+int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, float* loss_host) {
+  if (int rc = check_bound(h)) return rc;
+  if (!X_host || !y_host || !loss_host) return h->fail(HA_EINVAL, "round_host: NULL host buffer");
+  const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
+  const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
+  const int64_t rows = static_cast<int64_t>(h->B) * h->K1 * h->K2;
+  int64_t r0 = (h->t * h->B) % h->N, left = rows < h->N ? rows : h->N;
+  if (rows >= h->N) r0 = 0;
+  while (left > 0) {   // at most two contiguous row ranges per learner (wrap-around)
+    const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
+    int rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
+                                       h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
+                                       h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice,
+                                       h->stream),
+                     "round_host: X copy");
+    if (rc) return rc;
+    rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
+                                   n * 4, h->P, cudaMemcpyHostToDevice, h->stream),
+                 "round_host: y copy");
+    if (rc) return rc;
+    left -= n;
+    r0 = 0;
+  }
+  if (int rc = do_round(h)) return rc;
+  if (int rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost,
+                                       h->stream), "round_host: loss copy"))
+    return rc;
+  return hier_avg_check(h);
+}
+
+int hier_avg_get_step(const hier_avg* h, int64_t* t) {
+  if (!h || !t) return HA_EINVAL;
+  *t = h->t;
+  return HA_OK;
+}
+
+int hier_avg_set_step(hier_avg* h, int64_t t) {
+  if (!h || t < 0) return HA_EINVAL;
+  h->t = t;
+  return HA_OK;
+}
+
+int hier_avg_losses(hier_avg* h, float* loss_host) {
+  if (int rc = check_bound(h)) return rc;
+  if (!loss_host) return HA_EINVAL;
+  if (int rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost,
+                                       h->stream), "losses: copy"))
+    return rc;
+  return h->cuda(cudaStreamSynchronize(h->stream), "losses: sync");
+}
+
+int hier_avg_check(hier_avg* h) {
+  if (int rc = check_bound(h)) return rc;
+  int word = 0;
+  if (int rc = h->cuda(cudaMemcpyAsync(&word, h->err_word(), 4, cudaMemcpyDeviceToHost, h->stream),
+                       "check: copy"))
+    return rc;
+  if (int rc = h->cuda(cudaStreamSynchronize(h->stream), "check: sync")) return rc;
+  if (word) {
+    cudaMemsetAsync(h->err_word(), 0, 4, h->stream);
+    return h->fail(HA_ETIMEOUT, "a bounded device wait expired (error word %d)", word);
+  }
+  return HA_OK;
+}
+
+int hier_avg_profile(hier_avg* h, int enable) {
+  if (!h) return HA_EINVAL;
+  if (h->bound) cudaStreamSynchronize(h->stream);
+  h->recs.clear();
+  h->pool_used = 0;
+  h->prof = enable != 0;
+  return HA_OK;
+}
+
+int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* launches,
+                          double* bytes) {
+  if (!h || kind < 0 || kind >= HA_KERNEL_KINDS) return HA_EINVAL;
+  if (h->bound) {
+    if (int rc = h->cuda(cudaStreamSynchronize(h->stream), "profile: sync")) return rc;
+  }
+  double ms = 0, by = 0;
+  int64_t n = 0;
+  for (const ProfRec& r : h->recs) {
+    if (r.kind != kind) continue;
+    float e = 0.f;
+    if (cudaEventElapsedTime(&e, r.a, r.b) == cudaSuccess) ms += e;
+    by += r.bytes;
+    ++n;
+  }
+  if (total_ms) *total_ms = ms;
+  if (launches) *launches = n;
+  if (bytes) *bytes = by;
+  return HA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,87 @@
+// Internal declarations shared by the C-ABI layer and the kernel translation units.
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "hier_avg.h"
+
+namespace ha {
+
+// ----------------------------------------------------------------- averaging
+// Means over groups of n consecutive rows of w[P, ld] (n | P), written back to
+// every row of the group.  n = 1 is a no-op.
+cudaError_t launch_group_mean(float* w, int64_t P, int64_t n, int64_t D, int64_t ld,
+                              cudaStream_t s);
+// The local average (clusters of S) followed by the global average, in one pass.
+cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, int64_t ld,
+                                     cudaStream_t s);
+
+// ----------------------------------------------------------------- bf16 tensor-core step
+// Activation buffers of the bf16 path (all zero-initialised once; kernels only
+// ever write the valid region, so the padding stays zero):
+//   H_l   [P][Bn][pitch(d_l)]  bf16  layer-l input rows (batch-major)
+//   HT_l  [P][d_l][Kp]         bf16  the same, transposed (feature-major)
+//   dZ_l  [P][Bn][pitch(d_l)]  bf16  gradient w.r.t. the pre-activation of layer l
+//   dZT_l [P][d_l][Kp]         bf16  transposed
+//   Z_L   [P][B][d_L]          fp32  logits of the last layer
+// Bn = B rounded up to 16 (the MMA N extent), Kp = 64 (B <= 64), pitch(d) = d
+// rounded up to 64.
+struct TcFwdArgs {
+  int in, out, B, Bn, Kp;
+  int64_t ld;                 // parameter row length (floats)
+  const float* bias;          // learner 0's b_l; learner j at + j * ld
+  int relu;                   // 1: hidden layer (ReLU, write H and HT), 0: logits
+  __nv_bfloat16* h_out;       // H_{l+1} [P][Bn][pitch_out]
+  int pitch_out;
+  __nv_bfloat16* ht_out;      // HT_{l+1} [P][out][Kp]
+  float* z_out;               // Z_L [P][B][out]
+  int* err;
+};
+struct TcBwdArgs {
+  int in, out, B, Bn, Kp;
+  int64_t ld;
+  float lr;
+  int has_dx;                 // compute dZ_{l-1} (every layer but the first)
+  float* bias_prev;           // learner 0's b_{l-1}
+  __nv_bfloat16* dz_prev;     // dZ_{l-1} [P][Bn][pitch_in]
+  int pitch_in;
+  __nv_bfloat16* dzt_prev;    // dZT_{l-1} [P][in][Kp]
+  int* err;
+};
+int tc_fwd_smem_bytes();
+int tc_bwd_smem_bytes();
+cudaError_t tc_configure();   // raises the dynamic shared-memory limits once
+cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
+                              const TcFwdArgs& a, int P, cudaStream_t s);
+cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& ht_in,
+                               const CUtensorMap& dz, const CUtensorMap& dzt,
+                               const TcBwdArgs& a, int P, cudaStream_t s);
+// Mini-batch fetch for the bf16 path: rows (t*B + b) mod N of X -> H_0 and HT_0.
+cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
+                               int Kp, int pitch0, int64_t t, int P, __nv_bfloat16* H0,
+                               __nv_bfloat16* HT0, cudaStream_t s);
+// Softmax cross-entropy gradient of the last layer (bf16 operands out), loss, and
+// the SGD update of the last bias.
+cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+                             int Bn, int Kp, int C, int pitch_c, float lr, float* bias_L,
+                             int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
+                             int P, cudaStream_t s);
+
+// ----------------------------------------------------------------- fp32 CUDA-core step
+// Buffers: H_l [P][B][d_l] fp32, Z_L [P][B][d_L], dZ_l [P][B][d_l] fp32.
+cudaError_t launch_gather_f32(const float* X, int64_t N, int d0, int B, int64_t t, int P,
+                              float* H0, cudaStream_t s);
+cudaError_t launch_fwd_f32(const float* H, const float* W, const float* bias, int64_t ld,
+                           int in, int out, int B, int relu, float* out_act, int P,
+                           cudaStream_t s);
+cudaError_t launch_xent_f32(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+                            int C, float* dZ, float* loss, int P, cudaStream_t s);
+cudaError_t launch_dx_f32(const float* dZ, const float* W, int64_t ld, const float* Hprev,
+                          int in, int out, int B, float* dZprev, int P, cudaStream_t s);
+cudaError_t launch_dw_update_f32(const float* dZ, const float* H, float* W, float* bias,
+                                 int64_t ld, int in, int out, int B, float lr, int P,
+                                 cudaStream_t s);
+
+}  // namespace ha

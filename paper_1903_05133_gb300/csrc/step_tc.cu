@@ -1,0 +1,555 @@
+// bf16 learner step on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+//
+// One local SGD step of Algorithm 1 (Sec. 3.1) for every learner of a ReLU MLP:
+// forward Z_l = H_{l-1} W_l^T + b_l, softmax cross-entropy gradient, backward
+// dH_{l-1} = dZ_l W_l (with W_l before its update) and W_l -= lr * dZ_l^T H_{l-1}.
+// The fp32 master weights W_l [P][out][in] are streamed from HBM by TMA and
+// rounded to bf16 in shared memory by the CTA itself; MMAs accumulate in fp32 in
+// tensor memory.  All operands use the K-major 128-byte-swizzle layout.
+//
+// Because the per-learner batch B (<= 64) is far below the MMA's M, every GEMM
+// is issued "swap-AB": the weight tile supplies M = 128 rows and the batch is
+// the N extent.
+//
+// Forward kernel  (grid: out tiles of 128 x P learners)
+//   warp 4: TMA producer - fp32 W tile [128 x 64] + bf16 H tile [Bn x 64] per stage
+//   warps 0-3: round W to bf16 into the swizzled A tile; then the epilogue
+//              (bias, ReLU, bf16 H and H^T of the next layer, or fp32 logits)
+//   warp 5: TMEM allocation + single-thread MMA issue, Z^T[128 x Bn] += W H^T
+// Backward kernel (grid: in tiles of 128 x P learners), one pass over W_l:
+//   per out-chunk of 64 rows: TMA loads fp32 W [64 x 128], dZ [Bn x 64],
+//   dZ^T [64 x 64]; warps 0-3 write W^T (bf16) for the dX MMA; MMA warp issues
+//     dH^T[128 x Bn] += W^T(chunk) dZ^T(chunk)          (accumulated over chunks)
+//     dW^T[128 x 64]  = H^T[128 x B] dZ(chunk)           (double-buffered in TMEM)
+//   warps 0-3 then update the fp32 chunk in shared memory (w - lr * dw, separate
+//   rounded multiply and subtract) and TMA-store it back: W is read once and
+//   written once per step.  Finally dZ_{l-1} = dH * [H_{l-1} > 0] and the bias
+//   b_{l-1} -= lr * sum_b dZ_{l-1}.
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ha {
+namespace {
+
+constexpr int kStages = 3;
+constexpr int kThreads = 192;          // warps 0-3 convert/epilogue, 4 TMA, 5 MMA
+constexpr int kConv = 128;
+
+// ------------------------------------------------------------------ forward
+constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile
+constexpr int kFwdWbf = 128 * 64 * 2;                  // 16 KB bf16 A tile
+constexpr int kFwdH = 64 * 128;                        //  8 KB bf16 B tile (Bn <= 64)
+constexpr int kFwdStage = kFwdWf32 + kFwdWbf + kFwdH;  // 56 KB
+constexpr int kFwdBarOff = kStages * kFwdStage;
+constexpr int kFwdSmem = kFwdBarOff + 256 + 1024;      // + barriers + alignment slack
+constexpr uint32_t kFwdTmemCols = 64;
+
+// Bounded wait whose outcome is made uniform across the warp, so that a warp never
+// reaches a .sync.aligned tcgen05 instruction with only some of its lanes.
+__device__ __forceinline__ bool wait_warp(uint64_t* bar, uint32_t parity, int* err) {
+  const bool r = mbar_wait(bar, parity, err);
+  return __all_sync(0xffffffffu, r);
+}
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  return reinterpret_cast<uint8_t*>((a + 1023) & ~uintptr_t(1023));
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
+                 const TcFwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = blockIdx.y, o0 = blockIdx.x * 128;
+  const int nk = (a.in + 63) / 64;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kFwdBarOff);
+  uint64_t* conv = full + kStages;
+  uint64_t* empty = conv + kStages;
+  uint64_t* done = empty + kStages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  auto wf = [&](int s) { return smem + s * kFwdStage; };
+  auto wb = [&](int s) { return smem + s * kFwdStage + kFwdWf32; };
+  auto hb = [&](int s) { return smem + s * kFwdStage + kFwdWf32 + kFwdWbf; };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&conv[s], kConv);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(done, 1);
+    fence_barrier_init();
+  }
+  if (warp == 5) {
+    tmem_alloc(tmem_slot, kFwdTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 4) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_h);
+      int issued = 0;
+      for (int c = 0; c < nk; ++c) {
+        const int s = c % kStages;
+        if (c >= kStages && !mbar_wait(&empty[s], ((c / kStages) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&full[s], kFwdWf32 + a.Bn * 128);
+        tma_load_3d(wf(s), &tm_w, &full[s], c * 64, o0, j);
+        tma_load_3d(hb(s), &tm_h, &full[s], c * 64, 0, j);
+        issued = c + 1;
+      }
+      // Every load issued must have landed before the CTA may exit.
+      for (int c = issued - kStages > 0 ? issued - kStages : 0; c < issued; ++c)
+        mbar_wait(&full[c % kStages], (c / kStages) & 1, a.err);
+    }
+  } else if (warp == 5) {
+    if (lane == 0) {
+      const uint32_t idesc = umma_idesc_bf16(128, a.Bn);
+      for (int c = 0; c < nk; ++c) {
+        const int s = c % kStages;
+        if (!mbar_wait(&conv[s], (c / kStages) & 1, a.err)) break;
+        tc_fence_after();
+        const uint64_t ad = umma_desc_sw128(smem_u32(wb(s)));
+        const uint64_t bd = umma_desc_sw128(smem_u32(hb(s)));
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (c > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&empty[s]);
+      }
+      tc_commit(done);
+      mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
+    }
+  } else {
+    // ---- warps 0-3: fp32 -> bf16 A tile, then the epilogue
+    const int t = threadIdx.x;
+    bool ok = true;
+    for (int c = 0; c < nk; ++c) {
+      const int s = c % kStages;
+      if (!wait_warp(&full[s], (c / kStages) & 1, a.err)) { ok = false; break; }
+      const float4* src = reinterpret_cast<const float4*>(wf(s));
+      uint8_t* dst = wb(s);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int f = t + kConv * i;        // float4 index in the [128][64] fp32 tile
+        const int r = f >> 4, k = (f & 15) * 4;
+        const float4 v = src[f];
+        uint2 pk;
+        pk.x = pack_bf16x2(v.x, v.y);
+        pk.y = pack_bf16x2(v.z, v.w);
+        *reinterpret_cast<uint2*>(dst + sw128_offset(r, k)) = pk;
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(&conv[s]);
+    }
+    if (ok) ok = wait_warp(done, 0, a.err);
+    tc_fence_after();
+    const int o = o0 + t;
+    const bool valid = o < a.out;
+    const float bias = valid ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    for (int cb = 0; cb < a.Bn; cb += 16) {
+      float v[16];
+      tmem_ld16(tbase + cb, v);
+      tmem_ld_wait();
+      if (!ok || !valid) continue;
+      if (a.relu) {
+        uint32_t pk[8];
+#pragma unroll
+        for (int q = 0; q < 16; q += 2) {
+          const float h0 = fmaxf(__fadd_rn(v[q], bias), 0.f);
+          const float h1 = fmaxf(__fadd_rn(v[q + 1], bias), 0.f);
+          const bool in0 = cb + q < a.B, in1 = cb + q + 1 < a.B;
+          pk[q / 2] = pack_bf16x2(in0 ? h0 : 0.f, in1 ? h1 : 0.f);
+          const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
+          if (in0) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] = hh.x;
+          if (in1) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_out + o] = hh.y;
+        }
+        uint4* dst = reinterpret_cast<uint4*>(a.ht_out + (static_cast<int64_t>(j) * a.out + o) * a.Kp + cb);
+        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 16; ++q)
+          if (cb + q < a.B)
+            a.z_out[(static_cast<int64_t>(j) * a.B + cb + q) * a.out + o] = __fadd_rn(v[q], bias);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kFwdTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ backward
+constexpr int kBwdWf32 = 64 * 128 * 4;                 // 32 KB fp32 W chunk [64 o][128 i]
+constexpr int kBwdWT = 128 * 64 * 2;                   // 16 KB bf16 W^T [128 i][64 o]
+constexpr int kBwdDZ = 64 * 128;                       //  8 KB bf16 dZ [Bn][64 o]
+constexpr int kBwdDZT = 64 * 128;                      //  8 KB bf16 dZ^T [64 o][64 b]
+constexpr int kBwdStage = kBwdWf32 + kBwdWT + kBwdDZ + kBwdDZT;   // 64 KB
+constexpr int kBwdHT = 128 * 128;                      // 16 KB bf16 H^T [128 i][64 b]
+constexpr int kBwdBarOff = kStages * kBwdStage + kBwdHT;
+constexpr int kBwdSmem = kBwdBarOff + 256 + 1024;
+constexpr uint32_t kBwdTmemCols = 256;                 // dX at 0, dW buffers at 64, 128
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tc_backward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_ht,
+                  const __grid_constant__ CUtensorMap tm_dz, const __grid_constant__ CUtensorMap tm_dzt,
+                  const TcBwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j = blockIdx.y, i0 = blockIdx.x * 128;
+  const int nc = (a.out + 63) / 64;
+  uint8_t* ht = smem + kStages * kBwdStage;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBwdBarOff);
+  uint64_t* conv = full + kStages;
+  uint64_t* mdone = conv + kStages;
+  uint64_t* empty = mdone + kStages;
+  uint64_t* tfree = empty + kStages;   // [2]
+  uint64_t* htfull = tfree + 2;
+  uint64_t* upd = htfull + 1;         // [kStages] updated chunk ready for the TMA store
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(upd + kStages);
+  auto wf = [&](int s) { return smem + s * kBwdStage; };
+  auto wt = [&](int s) { return smem + s * kBwdStage + kBwdWf32; };
+  auto dzb = [&](int s) { return smem + s * kBwdStage + kBwdWf32 + kBwdWT; };
+  auto dztb = [&](int s) { return smem + s * kBwdStage + kBwdWf32 + kBwdWT + kBwdDZ; };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&conv[s], kConv);
+      mbar_init(&mdone[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&tfree[0], kConv);
+    mbar_init(&tfree[1], kConv);
+    mbar_init(htfull, 1);
+    for (int s = 0; s < kStages; ++s) mbar_init(&upd[s], kConv);
+    fence_barrier_init();
+  }
+  if (warp == 5) {
+    tmem_alloc(tmem_slot, kBwdTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 4) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_ht);
+      tma_prefetch_desc(&tm_dz);
+      tma_prefetch_desc(&tm_dzt);
+      mbar_arrive_expect_tx(htfull, kBwdHT);
+      tma_load_3d(ht, &tm_ht, htfull, 0, i0, j);
+      const uint32_t bytes = kBwdWf32 + kBwdDZT + (a.has_dx ? a.Bn * 128 : 0);
+      int issued = 0;
+      for (int c = 0; c < nc; ++c) {
+        const int s = c % kStages;
+        if (c >= kStages && !mbar_wait(&empty[s], ((c / kStages) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&full[s], bytes);
+        tma_load_3d(wf(s), &tm_w, &full[s], i0, c * 64, j);
+        if (a.has_dx) tma_load_3d(dzb(s), &tm_dz, &full[s], c * 64, 0, j);
+        tma_load_3d(dztb(s), &tm_dzt, &full[s], 0, c * 64, j);
+        issued = c + 1;
+      }
+      mbar_wait(htfull, 0, a.err);
+      for (int c = issued - kStages > 0 ? issued - kStages : 0; c < issued; ++c)
+        mbar_wait(&full[c % kStages], (c / kStages) & 1, a.err);
+    }
+  } else if (warp == 5) {
+    if (lane == 0) {
+      const uint32_t idesc_dx = umma_idesc_bf16(128, a.Bn);
+      const uint32_t idesc_dw = umma_idesc_bf16(128, 64);
+      const int kb = (a.B + 15) / 16;   // K = B for dW
+      bool ok = mbar_wait(htfull, 0, a.err);
+      const uint64_t hd = umma_desc_sw128(smem_u32(ht));
+      int c = 0;
+      for (; ok && c < nc; ++c) {
+        const int s = c % kStages, buf = c & 1;
+        if (!mbar_wait(&conv[s], (c / kStages) & 1, a.err)) break;
+        if (c >= 2 && !mbar_wait(&tfree[buf], ((c / 2) - 1) & 1, a.err)) break;
+        tc_fence_after();
+        if (a.has_dx) {
+          const uint64_t ad = umma_desc_sw128(smem_u32(wt(s)));
+          const uint64_t bd = umma_desc_sw128(smem_u32(dzb(s)));
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc_dx, (c > 0 || kk > 0) ? 1u : 0u);
+        }
+        const uint64_t bd = umma_desc_sw128(smem_u32(dztb(s)));
+        for (int kk = 0; kk < kb; ++kk)
+          tc_mma_bf16(tmem + 64 + 64 * buf, hd + 2 * kk, bd + 2 * kk, idesc_dw, kk > 0 ? 1u : 0u);
+        tc_commit(&mdone[s]);
+      }
+      // Drain: the last commit covers every MMA issued before it.
+      if (c > 0) mbar_wait(&mdone[(c - 1) % kStages], ((c - 1) / kStages) & 1, a.err);
+    }
+  } else {
+    // ---- warps 0-3: W^T for dX, the in-place SGD update, then the dX epilogue
+    const int t = threadIdx.x;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    bool ok = true;
+    for (int c = 0; c <= nc && ok; ++c) {
+      if (c < nc) {
+        const int s = c % kStages;
+        if (!wait_warp(&full[s], (c / kStages) & 1, a.err)) { ok = false; break; }
+        if (a.has_dx) {
+          const float* src = reinterpret_cast<const float*>(wf(s));
+          uint8_t* dst = wt(s);
+#pragma unroll
+          for (int ob = 0; ob < 8; ++ob) {
+            float v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v[q] = src[(ob * 8 + q) * 128 + t];
+            *reinterpret_cast<uint4*>(dst + sw128_offset(t, ob * 8)) =
+                make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                           pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+          }
+          fence_proxy_async_smem();
+        }
+        mbar_arrive(&conv[s]);
+      }
+      if (c > 0) {
+        const int cp = c - 1, sp = cp % kStages, buf = cp & 1;
+        if (!wait_warp(&mdone[sp], (cp / kStages) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+        float* w = reinterpret_cast<float*>(wf(sp));
+#pragma unroll
+        for (int qb = 0; qb < 4; ++qb) {
+          float d[16];
+          tmem_ld16(tbase + 64 + 64 * buf + 16 * qb, d);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            float* p = w + (qb * 16 + q) * 128 + t;
+            *p = __fsub_rn(*p, __fmul_rn(a.lr, d[q]));
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&tfree[buf]);
+        fence_proxy_async_smem();
+        mbar_arrive(&upd[sp]);
+        if (t == 0) {
+          if (mbar_wait(&upd[sp], (cp / kStages) & 1, a.err)) {
+            tma_store_3d(&tm_w, w, i0, cp * 64, j);
+            tma_store_commit();
+            tma_store_wait_read_all();
+          }
+          mbar_arrive(&empty[sp]);
+        }
+      }
+    }
+    if (t == 0) tma_store_wait_all();
+    if (ok && a.has_dx) {
+      // dX epilogue: TMEM lane t holds dH^T[i0 + t][0 .. Bn)
+      tc_fence_after();
+      const int i = i0 + t;
+      const bool valid = i < a.in;
+      float db = 0.f;
+      for (int cb = 0; cb < a.Bn; cb += 16) {
+        float v[16];
+        tmem_ld16(tbase + cb, v);
+        tmem_ld_wait();
+        if (!valid) continue;
+        uint32_t pk[8];
+#pragma unroll
+        for (int q = 0; q < 16; q += 2) {
+          float dz[2];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int b = cb + q + e;
+            float x = 0.f;
+            if (b < a.B) {
+              const __nv_bfloat16 h = *reinterpret_cast<const __nv_bfloat16*>(ht + sw128_offset(t, b));
+              x = (__bfloat162float(h) > 0.f) ? v[q + e] : 0.f;
+              db = __fadd_rn(db, x);
+            }
+            dz[e] = x;
+          }
+          pk[q / 2] = pack_bf16x2(dz[0], dz[1]);
+          const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
+          if (cb + q < a.B) a.dz_prev[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_in + i] = hh.x;
+          if (cb + q + 1 < a.B) a.dz_prev[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_in + i] = hh.y;
+        }
+        uint4* dst = reinterpret_cast<uint4*>(a.dzt_prev + (static_cast<int64_t>(j) * a.in + i) * a.Kp + cb);
+        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      }
+      if (valid) {
+        float* bp = a.bias_prev + static_cast<int64_t>(j) * a.ld + i;
+        *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kBwdTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ gather
+// H_0[j][b][:] = X[j][(t*B + b) mod N][:], HT_0[j][k][b] = the same; one CTA per
+// (64-feature slice, learner).  Rows b >= B and columns b >= B stay zero.
+__global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __restrict__ X,
+                                                    int64_t N, int d0, int B, int Bn, int Kp,
+                                                    int pitch0, int64_t t,
+                                                    __nv_bfloat16* __restrict__ H0,
+                                                    __nv_bfloat16* __restrict__ HT0) {
+  __shared__ __align__(16) __nv_bfloat16 tile[64][64 + 8];
+  const int j = blockIdx.y, k0 = blockIdx.x * 64;
+  const int nvec = B * 8;                       // 16-byte vectors in the [B][64] slice
+  for (int idx = threadIdx.x; idx < nvec; idx += blockDim.x) {
+    const int b = idx >> 3, v = idx & 7;
+    const int k = k0 + v * 8;
+    uint4 val = make_uint4(0, 0, 0, 0);
+    if (k < d0) {
+      const int64_t row = (t * B + b) % N;
+      val = *reinterpret_cast<const uint4*>(X + (static_cast<int64_t>(j) * N + row) * d0 + k);
+      *reinterpret_cast<uint4*>(H0 + (static_cast<int64_t>(j) * Bn + b) * pitch0 + k) = val;
+    }
+    *reinterpret_cast<uint4*>(&tile[b][v * 8]) = val;
+  }
+  __syncthreads();
+  const int nbv = Bn / 8;                       // 8-column groups of the transposed row
+  for (int idx = threadIdx.x; idx < 64 * nbv; idx += blockDim.x) {
+    const int kk = idx / nbv, bv = idx % nbv;
+    const int k = k0 + kk;
+    if (k >= d0) continue;
+    __align__(16) __nv_bfloat16 vals[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int b = bv * 8 + q;
+      vals[q] = b < B ? tile[b][kk] : __float2bfloat16_rn(0.f);
+    }
+    *reinterpret_cast<uint4*>(HT0 + (static_cast<int64_t>(j) * d0 + k) * Kp + bv * 8) =
+        *reinterpret_cast<uint4*>(vals);
+  }
+}
+
+// ------------------------------------------------------------------ cross-entropy
+// One CTA per learner.  p = softmax(z_b), dZ = (p - onehot(y_b)) / B in fp32;
+// loss_j = mean_b (log sum exp - z_{b,y_b}); b_L -= lr * sum_b dZ (fp32).
+__global__ void __launch_bounds__(256) k_xent_bf16(const float* __restrict__ Z,
+                                                  const int32_t* __restrict__ y, int64_t N,
+                                                  int64_t t, int B, int Bn, int Kp, int C,
+                                                  int pitch_c, float lr, float* bias_L,
+                                                  int64_t ld, __nv_bfloat16* dZ,
+                                                  __nv_bfloat16* dZT, float* loss) {
+  __shared__ float row_max[64], row_sum[64], row_loss[64];
+  __shared__ int row_y[64];
+  const int j = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* Zj = Z + static_cast<int64_t>(j) * B * C;
+  for (int b = warp; b < B; b += blockDim.x / 32) {
+    const float* z = Zj + static_cast<int64_t>(b) * C;
+    float m = -INFINITY;
+    for (int c = lane; c < C; c += 32) m = fmaxf(m, z[c]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+    float s = 0.f;
+    for (int c = lane; c < C; c += 32) s += expf(z[c] - m);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) {
+      const int yb = y[static_cast<int64_t>(j) * N + (t * B + b) % N];
+      row_max[b] = m;
+      row_sum[b] = s;
+      row_y[b] = yb;
+      row_loss[b] = logf(s) + m - z[yb];
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float l = 0.f;
+    for (int b = 0; b < B; ++b) l += row_loss[b];
+    loss[j] = l / B;
+  }
+  const float fB = static_cast<float>(B);
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    float db = 0.f;
+    for (int b0 = 0; b0 < Bn; b0 += 8) {
+      __align__(16) __nv_bfloat16 vals[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int b = b0 + q;
+        float g = 0.f;
+        if (b < B) {
+          const float p = __fdiv_rn(expf(Zj[static_cast<int64_t>(b) * C + c] - row_max[b]), row_sum[b]);
+          g = __fdiv_rn(__fsub_rn(p, row_y[b] == c ? 1.f : 0.f), fB);
+          db = __fadd_rn(db, g);
+          dZ[(static_cast<int64_t>(j) * Bn + b) * pitch_c + c] = __float2bfloat16_rn(g);
+        }
+        vals[q] = __float2bfloat16_rn(g);
+      }
+      *reinterpret_cast<uint4*>(dZT + (static_cast<int64_t>(j) * C + c) * Kp + b0) =
+          *reinterpret_cast<uint4*>(vals);
+    }
+    float* bp = bias_L + static_cast<int64_t>(j) * ld + c;
+    *bp = __fsub_rn(*bp, __fmul_rn(lr, db));
+  }
+}
+
+}  // namespace
+
+int tc_fwd_smem_bytes() { return kFwdSmem; }
+int tc_bwd_smem_bytes() { return kBwdSmem; }
+
+cudaError_t tc_configure() {
+  cudaError_t e = cudaFuncSetAttribute(k_tc_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       kFwdSmem);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmem);
+}
+
+cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
+                              const TcFwdArgs& a, int P, cudaStream_t s) {
+  dim3 grid((a.out + 127) / 128, P);
+  k_tc_forward<<<grid, kThreads, kFwdSmem, s>>>(w_fwd, h_in, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& ht_in,
+                               const CUtensorMap& dz, const CUtensorMap& dzt,
+                               const TcBwdArgs& a, int P, cudaStream_t s) {
+  dim3 grid((a.in + 127) / 128, P);
+  k_tc_backward<<<grid, kThreads, kBwdSmem, s>>>(w_bwd, ht_in, dz, dzt, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
+                               int Kp, int pitch0, int64_t t, int P, __nv_bfloat16* H0,
+                               __nv_bfloat16* HT0, cudaStream_t s) {
+  dim3 grid((d0 + 63) / 64, P);
+  k_gather_bf16<<<grid, 256, 0, s>>>(X, N, d0, B, Bn, Kp, pitch0, t, H0, HT0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+                             int Bn, int Kp, int C, int pitch_c, float lr, float* bias_L,
+                             int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
+                             int P, cudaStream_t s) {
+  k_xent_bf16<<<P, 256, 0, s>>>(Z, y, N, t, B, Bn, Kp, C, pitch_c, lr, bias_L, ld, dZ, dZT, loss);
+  return cudaGetLastError();
+}
+
+}  // namespace ha
