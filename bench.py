@@ -148,12 +148,21 @@ def ncu_traffic(kind: str, workload: str):
 
 
 def launches_per_round(w) -> int:
+    """Kernel launches of one round (every launch is one of this library's kernels)."""
     L = len(w.dims) - 1
     if w.precision == "bf16":
-        per_step = 1 + L + 1 + L
+        steps = range(w.K1 * w.K2)
+        gathers = 0   # the first layer reads X directly unless a batch wraps around N
+        n = 0
+        for t in steps:
+            if (t * w.B) % w.N + w.B > w.N:
+                gathers += 1
+        per_step = L + (0 if w.dims[-1] <= 128 else 1) + L
+        n = w.K1 * w.K2 * per_step + gathers
     else:
         per_step = 1 + L + 1 + L + (L - 1)       # dX is its own launch for layers > 1
-    return w.K1 * w.K2 * per_step + (w.K2 - 1) * (1 if w.S > 1 else 0) + 1
+        n = w.K1 * w.K2 * per_step
+    return n + (w.K2 - 1) * (1 if w.S > 1 else 0) + 1
 
 
 # ----------------------------------------------------------------------------- oracle

@@ -12,6 +12,10 @@ fp32 master weights and, optionally, bf16 GEMM operands with fp32 accumulation):
           weights) are rounded to fp32; products are accumulated in float64 first
   "bf16"  as "fp32", and every operand of a matrix product is first rounded to
           bf16 (round-to-nearest-even): the input X, W_l, H_{l-1} and dZ_l
+  "bf16_acc32"  as "bf16" but each product is accumulated in fp32 (numpy's
+          float32 matrix product, in its own summation order): a second valid
+          order of the same computation, used to measure how far two correct
+          implementations drift apart through rounding-boundary decisions
 Readings: ReLU'(z) is taken as [h > 0] on the stored (operand) activation h;
 the update is w - fl(lr * g), a rounded product followed by a rounded subtraction.
 """
@@ -21,7 +25,7 @@ from typing import List, Sequence, Tuple
 
 import numpy as np
 
-MODES = ("f64", "fp32", "bf16")
+MODES = ("f64", "fp32", "bf16", "bf16_acc32")
 
 
 def bf16_round(x) -> np.ndarray:
@@ -43,6 +47,14 @@ def bf16_round(x) -> np.ndarray:
     return out.view(np.float32).reshape(x.shape)
 
 
+def _mm64(a, b):
+    return a @ b
+
+
+def _mm32(a, b):
+    return (np.asarray(a, np.float32) @ np.asarray(b, np.float32)).astype(np.float64)
+
+
 def _modes(mode: str):
     if mode == "f64":
         def operand(a):
@@ -52,7 +64,7 @@ def _modes(mode: str):
         def operand(a):
             return np.asarray(a, dtype=np.float32).astype(np.float64)
         store = operand
-    elif mode == "bf16":
+    elif mode in ("bf16", "bf16_acc32"):
         def operand(a):
             return bf16_round(np.asarray(a, dtype=np.float32)).astype(np.float64)
 
@@ -60,7 +72,7 @@ def _modes(mode: str):
             return np.asarray(a, dtype=np.float32).astype(np.float64)
     else:
         raise ValueError(f"mode must be one of {MODES}")
-    return operand, store
+    return operand, store, (_mm32 if mode == "bf16_acc32" else _mm64)
 
 
 def softmax_xent_grad(Z: np.ndarray, y: np.ndarray, B: int) -> Tuple[float, np.ndarray]:
@@ -81,19 +93,22 @@ def softmax_xent_grad(Z: np.ndarray, y: np.ndarray, B: int) -> Tuple[float, np.n
 
 
 def mlp_forward_backward(Ws: Sequence[np.ndarray], bs: Sequence[np.ndarray],
-                         X: np.ndarray, y: np.ndarray, mode: str
+                         X: np.ndarray, y: np.ndarray, mode: str, preacts: list | None = None
                          ) -> Tuple[float, List[np.ndarray], List[np.ndarray]]:
     """Loss and gradients (dW_l, db_l) of the mean softmax cross-entropy of a
-    ReLU MLP on one mini-batch X [B, d_0], y [B]."""
-    operand, store = _modes(mode)
+    ReLU MLP on one mini-batch X [B, d_0], y [B].  If ``preacts`` is a list, the
+    pre-activations Z_l of every layer are appended to it (for inspection only)."""
+    operand, store, mm = _modes(mode)
     L = len(Ws)
     B = X.shape[0]
     H = [operand(X)]                     # operand form of every layer input
     Zs = []
     for l in range(L):
-        z = store(H[l] @ operand(Ws[l]).T)
+        z = store(mm(H[l], operand(Ws[l]).T))
         z = store(z + np.asarray(bs[l], dtype=np.float64))
         Zs.append(z)
+        if preacts is not None:
+            preacts.append(z)
         if l < L - 1:
             H.append(operand(store(np.maximum(z, 0.0))))
     loss, dz = softmax_xent_grad(Zs[-1], y, B)
@@ -101,10 +116,10 @@ def mlp_forward_backward(Ws: Sequence[np.ndarray], bs: Sequence[np.ndarray],
     gW: List[np.ndarray] = [None] * L  # type: ignore[list-item]
     gb: List[np.ndarray] = [None] * L  # type: ignore[list-item]
     for l in reversed(range(L)):
-        gW[l] = store(operand(dz).T @ H[l])
+        gW[l] = store(mm(operand(dz).T, H[l]))
         gb[l] = store(dz.sum(axis=0))
         if l > 0:
-            dh = store(operand(dz) @ operand(Ws[l]))     # uses W_l before its update
+            dh = store(mm(operand(dz), operand(Ws[l])))  # uses W_l before its update
             dz = store(dh * (H[l] > 0))
     return loss, gW, gb
 
@@ -127,13 +142,17 @@ class MLPProblem:
     def __init__(self, X: np.ndarray, y: np.ndarray, B: int, n_layers: int, mode: str):
         self.X, self.y, self.B, self.L, self.mode = X, y, B, n_layers, mode
         self.last_loss = np.zeros(X.shape[0])
+        self.last_preacts: dict = {}
 
     def gradients(self, j: int, t: int, params_j: List[np.ndarray]) -> List[np.ndarray]:
         from .algorithm import batch_rows
         rows = batch_rows(t, self.B, self.X.shape[1])
         Ws, bs = params_j[0::2], params_j[1::2]
-        loss, gW, gb = mlp_forward_backward(Ws, bs, self.X[j, rows], self.y[j, rows], self.mode)
+        pre: list = []
+        loss, gW, gb = mlp_forward_backward(Ws, bs, self.X[j, rows], self.y[j, rows], self.mode,
+                                            preacts=pre)
         self.last_loss[j] = loss
+        self.last_preacts[j] = pre
         out = []
         for a, b in zip(gW, gb):
             out += [a, b]

@@ -6,6 +6,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <algorithm>
 #include <string>
 #include <vector>
 
@@ -20,6 +21,7 @@ using ha::TcBwdArgs;
 using ha::TcFwdArgs;
 
 constexpr int64_t kAlign = 1024;
+constexpr int64_t kTargetCtas = 152;   // one wave: the forward kernel fits one CTA per SM
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -61,6 +63,9 @@ struct hier_avg {
   std::vector<int> pitch;                       // per width index l = 0..L
   std::vector<int64_t> off_H, off_HT, off_dZ, off_dZT;
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
+  int64_t off_part = 0, off_cnt = 0;          // split-K partials and tile counters
+  std::vector<int> fwd_splits, fwd_tiles;     // per layer
+  bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
   // binding
   bool bound = false;
   int device = 0;
@@ -71,6 +76,7 @@ struct hier_avg {
   int64_t N = 0;
   cudaStream_t stream = nullptr;
   std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_ht, tm_dz, tm_dzt;
+  CUtensorMap tm_x;                           // X [P][N][d_0] as the first layer's batch tile
   int64_t t = 0;
   // profiling
   bool prof = false;
@@ -168,6 +174,25 @@ int plan_layout(hier_avg* h) {
       h->off_dZ[l] = take(P * h->Bn * h->pitch[l] * 2);
       h->off_dZT[l] = take(P * h->dims[l] * h->Kp * 2);
     }
+    // Split-K plan of the forward GEMMs: about one wave of CTAs on the 152 SMs.
+    // It depends on the shapes only, so the summation order is the same on every GPU.
+    h->fwd_splits.assign(L, 1);
+    h->fwd_tiles.assign(L, 1);
+    int64_t part_bytes = 0, max_tiles = 1;
+    for (int l = 0; l < L; ++l) {
+      const int64_t tiles = (h->dims[l + 1] + 127) / 128, nk = (h->dims[l] + 63) / 64;
+      int64_t splits = kTargetCtas / (tiles * P);   // never more than one wave
+      splits = std::max<int64_t>(1, std::min<int64_t>(splits, nk));
+      const int64_t per = (nk + splits - 1) / splits;
+      splits = (nk + per - 1) / per;
+      h->fwd_splits[l] = static_cast<int>(splits);
+      h->fwd_tiles[l] = static_cast<int>(tiles);
+      if (splits > 1) part_bytes = std::max(part_bytes, P * tiles * splits * 128 * h->Bn * 4);
+      max_tiles = std::max(max_tiles, tiles);
+    }
+    h->fused_xent = h->dims[L] <= 128;
+    h->off_part = take(std::max<int64_t>(part_bytes, 16));
+    h->off_cnt = take(P * max_tiles * 4);
   } else {
     for (int l = 0; l <= L; ++l) h->pitch[l] = h->dims[l];
     for (int l = 0; l < L; ++l) h->off_H[l] = take(P * B * h->dims[l] * 4);
@@ -226,6 +251,13 @@ int build_maps(hier_avg* h) {
                        in, P, Kp * 2, in * Kp * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B)))
       return rc;
   }
+  {
+    const uint64_t d0 = h->dims[0], N = h->N;
+    if ((rc = make_map(h, &h->tm_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, const_cast<void*>(h->X), d0,
+                       N, P, d0 * 2, N * d0 * 2, 64, static_cast<uint32_t>(Bn),
+                       CU_TENSOR_MAP_SWIZZLE_128B)))
+      return rc;
+  }
   for (int l = 1; l <= L; ++l) {
     const uint64_t d = h->dims[l], pd = h->pitch[l];
     if ((rc = make_map(h, &h->tm_dz[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_dZ[l], pd,
@@ -265,12 +297,18 @@ int do_step(hier_avg* h) {
   int rc;
   if (h->prec == HA_PREC_BF16) {
     const int d0 = h->dims[0];
-    rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, [&] {
-      return ha::launch_gather_bf16(static_cast<const __nv_bfloat16*>(h->X), h->N, d0, B, h->Bn,
-                                    h->Kp, h->pitch[0], h->t, P, h->wsp<__nv_bfloat16>(h->off_H[0]),
-                                    h->wsp<__nv_bfloat16>(h->off_HT[0]), s);
-    }, "gather");
-    if (rc) return rc;
+    // The first layer reads its batch tile straight from X unless the batch wraps
+    // around the end of the data set; then the rows are gathered first.
+    const int64_t r0 = (h->t * B) % h->N;
+    const bool x_direct = r0 + B <= h->N;
+    if (!x_direct) {
+      rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, [&] {
+        return ha::launch_gather_bf16(static_cast<const __nv_bfloat16*>(h->X), h->N, d0, B, h->Bn,
+                                      h->Kp, h->pitch[0], h->t, P, h->wsp<__nv_bfloat16>(h->off_H[0]),
+                                      h->wsp<__nv_bfloat16>(h->off_HT[0]), s);
+      }, "gather");
+      if (rc) return rc;
+    }
     for (int l = 0; l < L; ++l) {
       TcFwdArgs a{};
       a.in = h->dims[l];
@@ -280,28 +318,49 @@ int do_step(hier_avg* h) {
       a.Kp = h->Kp;
       a.ld = h->ld;
       a.bias = h->params + h->boff[l];
-      a.relu = l + 1 < L;
-      if (a.relu) {
+      a.splits = h->fwd_splits[l];
+      a.o_tiles = h->fwd_tiles[l];
+      a.part = h->wsp<float>(h->off_part);
+      a.counters = h->wsp<int>(h->off_cnt);
+      a.x_direct = (l == 0 && x_direct) ? 1 : 0;
+      a.x_row0 = static_cast<int>(r0);
+      a.ht0_out = h->wsp<__nv_bfloat16>(h->off_HT[0]);
+      if (l + 1 < L) {
+        a.mode = 0;
         a.h_out = h->wsp<__nv_bfloat16>(h->off_H[l + 1]);
         a.pitch_out = h->pitch[l + 1];
         a.ht_out = h->wsp<__nv_bfloat16>(h->off_HT[l + 1]);
+      } else if (h->fused_xent) {
+        a.mode = 2;
+        a.y = h->y;
+        a.N = h->N;
+        a.t = h->t;
+        a.lr = h->lr;
+        a.pitch_out = h->pitch[L];
+        a.dz_out = h->wsp<__nv_bfloat16>(h->off_dZ[L]);
+        a.dzt_out = h->wsp<__nv_bfloat16>(h->off_dZT[L]);
+        a.loss = h->loss();
       } else {
+        a.mode = 1;
         a.z_out = h->wsp<float>(h->off_Z);
       }
       a.err = h->err_word();
+      const CUtensorMap& hin = a.x_direct ? h->tm_x : h->tm_h[l];
       rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), [&] {
-        return ha::launch_tc_forward(h->tm_wf[l], h->tm_h[l], a, P, s);
+        return ha::launch_tc_forward(h->tm_wf[l], hin, a, P, s);
       }, "forward");
       if (rc) return rc;
     }
     const int C = h->dims[L];
-    rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
-      return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, h->Kp, C,
-                                  h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
-                                  h->wsp<__nv_bfloat16>(h->off_dZ[L]),
-                                  h->wsp<__nv_bfloat16>(h->off_dZT[L]), h->loss(), P, s);
-    }, "xent");
-    if (rc) return rc;
+    if (!h->fused_xent) {
+      rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
+        return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, h->Kp, C,
+                                    h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
+                                    h->wsp<__nv_bfloat16>(h->off_dZ[L]),
+                                    h->wsp<__nv_bfloat16>(h->off_dZT[L]), h->loss(), P, s);
+      }, "xent");
+      if (rc) return rc;
+    }
     for (int l = L - 1; l >= 0; --l) {
       TcBwdArgs a{};
       a.in = h->dims[l];

@@ -32,11 +32,28 @@ struct TcFwdArgs {
   int in, out, B, Bn, Kp;
   int64_t ld;                 // parameter row length (floats)
   const float* bias;          // learner 0's b_l; learner j at + j * ld
-  int relu;                   // 1: hidden layer (ReLU, write H and HT), 0: logits
-  __nv_bfloat16* h_out;       // H_{l+1} [P][Bn][pitch_out]
-  int pitch_out;
-  __nv_bfloat16* ht_out;      // HT_{l+1} [P][out][Kp]
-  float* z_out;               // Z_L [P][B][out]
+  int mode;                   // 0 hidden (ReLU -> H, HT), 1 logits -> z_out, 2 fused softmax-CE
+  __nv_bfloat16* h_out;       // mode 0: H_{l+1} [P][Bn][pitch_out]
+  int pitch_out;              // mode 0: H pitch; mode 2: dZ_L pitch
+  __nv_bfloat16* ht_out;      // mode 0: HT_{l+1} [P][out][Kp]
+  float* z_out;               // mode 1: Z_L [P][B][out]
+  // split-K over the input features: grid.z = splits; partial accumulators go to
+  // part [P][o_tiles][splits][128][Bn] and the last CTA of a tile (counted in
+  // counters [P][o_tiles], reset by that CTA) sums them in split order.
+  int splits, o_tiles;
+  float* part;
+  int* counters;
+  // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)
+  // and the CTAs of output tile 0 also write H_0^T.
+  int x_direct, x_row0;
+  __nv_bfloat16* ht0_out;     // HT_0 [P][in][Kp]
+  // mode 2: labels and outputs of the fused cross-entropy
+  const int32_t* y;
+  int64_t N, t;
+  float lr;
+  __nv_bfloat16* dz_out;      // dZ_L [P][Bn][pitch_out]
+  __nv_bfloat16* dzt_out;     // dZT_L [P][out][Kp]
+  float* loss;                // [P]
   int* err;
 };
 struct TcBwdArgs {

@@ -41,13 +41,23 @@ constexpr int kThreads = 192;          // warps 0-3 convert/epilogue, 4 TMA, 5 M
 constexpr int kConv = 128;
 
 // ------------------------------------------------------------------ forward
+// Shared memory: a 4-deep ring of TMA stages (fp32 W tile + bf16 batch tile) and a
+// double-buffered bf16 A tile that the converter warps fill for the MMA.
+constexpr int kFwdStages = 4;
 constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile
-constexpr int kFwdWbf = 128 * 64 * 2;                  // 16 KB bf16 A tile
 constexpr int kFwdH = 64 * 128;                        //  8 KB bf16 B tile (Bn <= 64)
-constexpr int kFwdStage = kFwdWf32 + kFwdWbf + kFwdH;  // 56 KB
-constexpr int kFwdBarOff = kStages * kFwdStage;
+constexpr int kFwdStage = kFwdWf32 + kFwdH;            // 40 KB
+constexpr int kFwdWbf = 128 * 64 * 2;                  // 16 KB bf16 A tile (x2)
+constexpr int kFwdWbfOff = kFwdStages * kFwdStage;
+constexpr int kFwdBarOff = kFwdWbfOff + 2 * kFwdWbf;
 constexpr int kFwdSmem = kFwdBarOff + 256 + 1024;      // + barriers + alignment slack
-constexpr uint32_t kFwdTmemCols = 64;
+// The tensor core's fp32 accumulation loses precision roughly in proportion to the
+// number of MMAs chained into one accumulator, so the accumulator is promoted:
+// every kSegChunks chunks (16 MMAs) the partial sum is folded into fp32 registers
+// with IEEE adds, in chunk order, while the MMAs continue in the other TMEM buffer.
+constexpr int kSegChunks = 4;
+constexpr uint32_t kFwdTmemCols = 128;   // two accumulator buffers of 64 columns
+constexpr int kFwdHidden = 0, kFwdLogits = 1, kFwdXent = 2;   // TcFwdArgs::mode
 
 // Bounded wait whose outcome is made uniform across the warp, so that a warp never
 // reaches a .sync.aligned tcgen05 instruction with only some of its lanes.
@@ -61,28 +71,107 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((a + 1023) & ~uintptr_t(1023));
 }
 
+// Epilogue of the last layer when every class fits in one 128-row tile: the
+// softmax cross-entropy gradient straight from the accumulator (no logits
+// round trip).  Thread t owns class t's logits z[0..Bn); the work is spread
+// over all threads: column statistics (one thread per sample), gradients (all
+// class x sample pairs), then per-class bias sums in sample order.
+__device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, const float* z,
+                                              float* sm) {
+  constexpr int ZP = 65;
+  float* zs = sm;                  // [128][ZP] logits, class-major
+  float* gs = sm + 128 * ZP;       // [128][ZP] gradients
+  float* stat = gs + 128 * ZP;     // max[64], sum[64], label[64], loss[64]
+  const int C = a.out, B = a.B;
+  if (t < C) {
+#pragma unroll
+    for (int b = 0; b < 64; ++b)
+      if (b < a.Bn) zs[t * ZP + b] = z[b];
+  }
+  named_barrier_sync(1, kConv);
+  if (t < B) {
+    float m = -INFINITY;
+    for (int c = 0; c < C; ++c) m = fmaxf(m, zs[c * ZP + t]);
+    float s = 0.f;
+    for (int c = 0; c < C; ++c) s += expf(zs[c * ZP + t] - m);
+    const int yb = a.y[static_cast<int64_t>(j) * a.N + (a.t * B + t) % a.N];
+    stat[t] = m;
+    stat[64 + t] = s;
+    stat[128 + t] = __int_as_float(yb);
+    stat[192 + t] = logf(s) + m - zs[yb * ZP + t];
+  }
+  named_barrier_sync(1, kConv);
+  const float fB = static_cast<float>(B);
+  for (int e = t; e < C * B; e += kConv) {
+    const int c = e / B, b = e - c * B;
+    const float p = __fdiv_rn(expf(zs[c * ZP + b] - stat[b]), stat[64 + b]);
+    const float g = __fdiv_rn(__fsub_rn(p, __float_as_int(stat[128 + b]) == c ? 1.f : 0.f), fB);
+    gs[c * ZP + b] = g;
+    a.dz_out[(static_cast<int64_t>(j) * a.Bn + b) * a.pitch_out + c] = __float2bfloat16_rn(g);
+  }
+  named_barrier_sync(1, kConv);
+  if (t == 0) {
+    float l = 0.f;
+    for (int b = 0; b < B; ++b) l += stat[192 + b];
+    a.loss[j] = l / B;
+  }
+  if (t < C) {
+    float db = 0.f;
+    for (int b0 = 0; b0 < a.Bn; b0 += 8) {
+      uint32_t pk[4];
+#pragma unroll
+      for (int q = 0; q < 8; q += 2) {
+        const int b = b0 + q;
+        const float g0 = b < B ? gs[t * ZP + b] : 0.f;
+        const float g1 = b + 1 < B ? gs[t * ZP + b + 1] : 0.f;
+        if (b < B) db = __fadd_rn(db, g0);
+        if (b + 1 < B) db = __fadd_rn(db, g1);
+        pk[q / 2] = pack_bf16x2(g0, g1);
+      }
+      *reinterpret_cast<uint4*>(a.dzt_out + (static_cast<int64_t>(j) * C + t) * a.Kp + b0) =
+          make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    }
+    float* bp = const_cast<float*>(a.bias) + static_cast<int64_t>(j) * a.ld + t;
+    *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
                  const TcFwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.y, o0 = blockIdx.x * 128;
-  const int nk = (a.in + 63) / 64;
+  const int j = blockIdx.y, tile = blockIdx.x, o0 = tile * 128, split = blockIdx.z;
+  const int nk_all = (a.in + 63) / 64;
+  const int per = (nk_all + a.splits - 1) / a.splits;
+  const int c_begin = split * per;
+  const int nk = min(nk_all, c_begin + per) - c_begin;   // >= 1 by the host's choice of splits
+  const int h_row0 = a.x_direct ? a.x_row0 : 0;           // batch rows inside the H (or X) map
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kFwdBarOff);
-  uint64_t* conv = full + kStages;
-  uint64_t* empty = conv + kStages;
-  uint64_t* done = empty + kStages;
+  uint64_t* empty = full + kFwdStages;
+  uint64_t* conv = empty + kFwdStages;   // [2] A tile written
+  uint64_t* wfree = conv + 2;            // [2] A tile consumed by the MMA
+  uint64_t* accf = wfree + 2;            // [2] accumulator segment complete
+  uint64_t* accr = accf + 2;             // [2] accumulator segment drained
+  uint64_t* done = accr + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  int* last_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  int* all_ok = last_flag + 1;
   auto wf = [&](int s) { return smem + s * kFwdStage; };
-  auto wb = [&](int s) { return smem + s * kFwdStage + kFwdWf32; };
-  auto hb = [&](int s) { return smem + s * kFwdStage + kFwdWf32 + kFwdWbf; };
+  auto hb = [&](int s) { return smem + s * kFwdStage + kFwdWf32; };
+  auto wb = [&](int b) { return smem + kFwdWbfOff + b * kFwdWbf; };
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kFwdStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&conv[s], kConv);
       mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&conv[b], kConv);
+      mbar_init(&wfree[b], 1);
+      mbar_init(&accf[b], 1);
+      mbar_init(&accr[b], kConv);
     }
     mbar_init(done, 1);
     fence_barrier_init();
@@ -102,43 +191,76 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_prefetch_desc(&tm_h);
       int issued = 0;
       for (int c = 0; c < nk; ++c) {
-        const int s = c % kStages;
-        if (c >= kStages && !mbar_wait(&empty[s], ((c / kStages) - 1) & 1, a.err)) break;
+        const int s = c % kFwdStages;
+        if (c >= kFwdStages && !mbar_wait(&empty[s], ((c / kFwdStages) - 1) & 1, a.err)) break;
         mbar_arrive_expect_tx(&full[s], kFwdWf32 + a.Bn * 128);
-        tma_load_3d(wf(s), &tm_w, &full[s], c * 64, o0, j);
-        tma_load_3d(hb(s), &tm_h, &full[s], c * 64, 0, j);
+        tma_load_3d(wf(s), &tm_w, &full[s], (c_begin + c) * 64, o0, j);
+        tma_load_3d(hb(s), &tm_h, &full[s], (c_begin + c) * 64, h_row0, j);
         issued = c + 1;
       }
       // Every load issued must have landed before the CTA may exit.
-      for (int c = issued - kStages > 0 ? issued - kStages : 0; c < issued; ++c)
-        mbar_wait(&full[c % kStages], (c / kStages) & 1, a.err);
+      for (int c = issued - kFwdStages > 0 ? issued - kFwdStages : 0; c < issued; ++c)
+        mbar_wait(&full[c % kFwdStages], (c / kFwdStages) & 1, a.err);
     }
   } else if (warp == 5) {
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_bf16(128, a.Bn);
       for (int c = 0; c < nk; ++c) {
-        const int s = c % kStages;
-        if (!mbar_wait(&conv[s], (c / kStages) & 1, a.err)) break;
+        const int s = c % kFwdStages, b = c & 1;
+        const int seg = c / kSegChunks, ab = seg & 1, first = c % kSegChunks == 0;
+        if (first && seg >= 2 && !mbar_wait(&accr[ab], ((seg >> 1) - 1) & 1, a.err)) break;
+        if (!mbar_wait(&conv[b], (c >> 1) & 1, a.err)) break;
         tc_fence_after();
-        const uint64_t ad = umma_desc_sw128(smem_u32(wb(s)));
+        const uint64_t ad = umma_desc_sw128(smem_u32(wb(b)));
         const uint64_t bd = umma_desc_sw128(smem_u32(hb(s)));
+        const uint32_t d = tmem + 64 * ab;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
-          tc_mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (c > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
         tc_commit(&empty[s]);
+        tc_commit(&wfree[b]);
+        if (c % kSegChunks == kSegChunks - 1 || c == nk - 1) tc_commit(&accf[ab]);
       }
       tc_commit(done);
       mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
     }
   } else {
-    // ---- warps 0-3: fp32 -> bf16 A tile, then the epilogue
+    // ---- warps 0-3: fp32 -> bf16 A tile (and H_0^T for the first layer), then the epilogue
     const int t = threadIdx.x;
+    const bool write_ht0 = a.x_direct && tile == 0;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    float acc[64];
+#pragma unroll
+    for (int q = 0; q < 64; ++q) acc[q] = 0.f;
+    int drained = 0;   // accumulator segments folded into acc so far
+    const int nseg = (nk + kSegChunks - 1) / kSegChunks;
+    // Fold segment `drained` into the registers (warp-uniform; contains tcgen05.ld).
+    auto drain = [&]() -> bool {
+      const int ab = drained & 1;
+      if (!wait_warp(&accf[ab], (drained >> 1) & 1, a.err)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int cb = 0; cb < 64; cb += 16) {
+        if (cb < a.Bn) {
+          float v[16];
+          tmem_ld16(tbase + 64 * ab + cb, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 16; ++q) acc[cb + q] = __fadd_rn(acc[cb + q], v[q]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&accr[ab]);
+      ++drained;
+      return true;
+    };
     bool ok = true;
     for (int c = 0; c < nk; ++c) {
-      const int s = c % kStages;
-      if (!wait_warp(&full[s], (c / kStages) & 1, a.err)) { ok = false; break; }
+      const int s = c % kFwdStages, bb = c & 1;
+      if (!wait_warp(&full[s], (c / kFwdStages) & 1, a.err)) { ok = false; break; }
+      if (c >= 2 && !wait_warp(&wfree[bb], ((c >> 1) - 1) & 1, a.err)) { ok = false; break; }
       const float4* src = reinterpret_cast<const float4*>(wf(s));
-      uint8_t* dst = wb(s);
+      uint8_t* dst = wb(bb);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         const int f = t + kConv * i;        // float4 index in the [128][64] fp32 tile
@@ -149,40 +271,115 @@ __global__ void __launch_bounds__(kThreads, 1)
         pk.y = pack_bf16x2(v.z, v.w);
         *reinterpret_cast<uint2*>(dst + sw128_offset(r, k)) = pk;
       }
+      if (write_ht0) {
+        // H_0^T[k][b] for this chunk's 64 features, from the staged batch tile
+        // (rows b >= B of the tile belong to later samples and are written as 0).
+        const uint8_t* hs = hb(s);
+        const int kk = t & 63;
+        const int k = (c_begin + c) * 64 + kk;
+        if (k < a.in) {
+          for (int b0 = (t >> 6) * 8; b0 < a.Bn; b0 += 16) {
+            uint32_t pk[4];
+#pragma unroll
+            for (int q = 0; q < 8; q += 2) {
+              const int b = b0 + q;
+              const uint16_t lo = b < a.B ? *reinterpret_cast<const uint16_t*>(hs + sw128_offset(b, kk)) : 0;
+              const uint16_t hi = b + 1 < a.B ? *reinterpret_cast<const uint16_t*>(hs + sw128_offset(b + 1, kk)) : 0;
+              pk[q / 2] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+            }
+            *reinterpret_cast<uint4*>(a.ht0_out + (static_cast<int64_t>(j) * a.in + k) * a.Kp + b0) =
+                make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        }
+      }
       fence_proxy_async_smem();
-      mbar_arrive(&conv[s]);
+      mbar_arrive(&conv[bb]);
+      // one segment behind the MMAs: fold the segment completed a while ago
+      if (c % kSegChunks == kSegChunks - 1 && c / kSegChunks >= 1 && drained < c / kSegChunks)
+        if (!drain()) { ok = false; break; }
     }
+    while (ok && drained < nseg)
+      if (!drain()) ok = false;
     if (ok) ok = wait_warp(done, 0, a.err);
     tc_fence_after();
     const int o = o0 + t;
     const bool valid = o < a.out;
-    const float bias = valid ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
-    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
-    for (int cb = 0; cb < a.Bn; cb += 16) {
-      float v[16];
-      tmem_ld16(tbase + cb, v);
-      tmem_ld_wait();
-      if (!ok || !valid) continue;
-      if (a.relu) {
-        uint32_t pk[8];
+    bool finish = true;
+    if (a.splits > 1) {
+      // Split-K: publish this CTA's partial; the last CTA of the tile sums all
+      // partials in split order (deterministic) and runs the epilogue.
+      float* part = a.part + ((static_cast<int64_t>(j) * a.o_tiles + tile) * a.splits) * 128 * a.Bn;
+      float4* mine = reinterpret_cast<float4*>(part + (static_cast<int64_t>(split) * 128 + t) * a.Bn);
 #pragma unroll
-        for (int q = 0; q < 16; q += 2) {
-          const float h0 = fmaxf(__fadd_rn(v[q], bias), 0.f);
-          const float h1 = fmaxf(__fadd_rn(v[q + 1], bias), 0.f);
-          const bool in0 = cb + q < a.B, in1 = cb + q + 1 < a.B;
-          pk[q / 2] = pack_bf16x2(in0 ? h0 : 0.f, in1 ? h1 : 0.f);
-          const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
-          if (in0) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] = hh.x;
-          if (in1) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_out + o] = hh.y;
+      for (int q = 0; q < 64; q += 4)
+        if (q < a.Bn) mine[q / 4] = make_float4(acc[q], acc[q + 1], acc[q + 2], acc[q + 3]);
+      __threadfence();
+      named_barrier_sync(1, kConv);
+      if (t == 0) {
+        int* cnt = a.counters + static_cast<int64_t>(j) * a.o_tiles + tile;
+        const int prev = atomicAdd(cnt, 1);
+        *last_flag = (prev == a.splits - 1);
+        if (prev == a.splits - 1) *cnt = 0;     // ready for the next launch
+      }
+      named_barrier_sync(1, kConv);
+      finish = *last_flag != 0;
+      if (finish) {
+        __threadfence();
+#pragma unroll
+        for (int q = 0; q < 64; ++q) acc[q] = 0.f;
+        for (int sp = 0; sp < a.splits; ++sp) {
+          const float4* src = reinterpret_cast<const float4*>(part + (static_cast<int64_t>(sp) * 128 + t) * a.Bn);
+#pragma unroll
+          for (int q = 0; q < 64; q += 4) {
+            if (q >= a.Bn) break;
+            const float4 v = __ldcg(src + q / 4);
+            acc[q] = __fadd_rn(acc[q], v.x);
+            acc[q + 1] = __fadd_rn(acc[q + 1], v.y);
+            acc[q + 2] = __fadd_rn(acc[q + 2], v.z);
+            acc[q + 3] = __fadd_rn(acc[q + 3], v.w);
+          }
         }
-        uint4* dst = reinterpret_cast<uint4*>(a.ht_out + (static_cast<int64_t>(j) * a.out + o) * a.Kp + cb);
-        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-      } else {
+      }
+    }
+    // A timed-out wait in any converter warp makes the whole group skip the
+    // epilogue (which contains group barriers).
+    if (t == 0) *all_ok = 1;
+    named_barrier_sync(1, kConv);
+    if (!ok) atomicAnd(all_ok, 0);
+    named_barrier_sync(1, kConv);
+    ok = *all_ok != 0;
+    if (finish && ok) {
+      const float bias = valid ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
+      if (a.mode == kFwdXent) {
 #pragma unroll
-        for (int q = 0; q < 16; ++q)
-          if (cb + q < a.B)
-            a.z_out[(static_cast<int64_t>(j) * a.B + cb + q) * a.out + o] = __fadd_rn(v[q], bias);
+        for (int q = 0; q < 64; ++q) acc[q] = __fadd_rn(acc[q], bias);
+        xent_epilogue(a, j, t, acc, reinterpret_cast<float*>(smem));
+      } else if (valid) {
+#pragma unroll
+        for (int cb = 0; cb < 64; cb += 16) {
+          if (cb >= a.Bn) break;
+          if (a.mode == kFwdHidden) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int q = 0; q < 16; q += 2) {
+              const float h0 = fmaxf(__fadd_rn(acc[cb + q], bias), 0.f);
+              const float h1 = fmaxf(__fadd_rn(acc[cb + q + 1], bias), 0.f);
+              const bool in0 = cb + q < a.B, in1 = cb + q + 1 < a.B;
+              pk[q / 2] = pack_bf16x2(in0 ? h0 : 0.f, in1 ? h1 : 0.f);
+              const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
+              if (in0) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] = hh.x;
+              if (in1) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_out + o] = hh.y;
+            }
+            uint4* dst = reinterpret_cast<uint4*>(a.ht_out + (static_cast<int64_t>(j) * a.out + o) * a.Kp + cb);
+            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          } else {
+#pragma unroll
+            for (int q = 0; q < 16; ++q)
+              if (cb + q < a.B)
+                a.z_out[(static_cast<int64_t>(j) * a.B + cb + q) * a.out + o] = __fadd_rn(acc[cb + q], bias);
+          }
+        }
       }
     }
   }
@@ -204,7 +401,7 @@ constexpr int kBwdStage = kBwdWf32 + kBwdWT + kBwdDZ + kBwdDZT;   // 64 KB
 constexpr int kBwdHT = 128 * 128;                      // 16 KB bf16 H^T [128 i][64 b]
 constexpr int kBwdBarOff = kStages * kBwdStage + kBwdHT;
 constexpr int kBwdSmem = kBwdBarOff + 256 + 1024;
-constexpr uint32_t kBwdTmemCols = 256;                 // dX at 0, dW buffers at 64, 128
+constexpr uint32_t kBwdTmemCols = 256;   // dX buffers at columns 0 and 192, dW buffers at 64, 128
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_tc_backward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_ht,
@@ -223,7 +420,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tfree = empty + kStages;   // [2]
   uint64_t* htfull = tfree + 2;
   uint64_t* upd = htfull + 1;         // [kStages] updated chunk ready for the TMA store
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(upd + kStages);
+  uint64_t* xf = upd + kStages;       // [2] dX accumulator segment complete
+  uint64_t* xr = xf + 2;              // [2] dX accumulator segment drained
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xr + 2);
   auto wf = [&](int s) { return smem + s * kBwdStage; };
   auto wt = [&](int s) { return smem + s * kBwdStage + kBwdWf32; };
   auto dzb = [&](int s) { return smem + s * kBwdStage + kBwdWf32 + kBwdWT; };
@@ -240,6 +439,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&tfree[1], kConv);
     mbar_init(htfull, 1);
     for (int s = 0; s < kStages; ++s) mbar_init(&upd[s], kConv);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&xf[b], 1);
+      mbar_init(&xr[b], kConv);
+    }
     fence_barrier_init();
   }
   if (warp == 5) {
@@ -284,6 +487,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int c = 0;
       for (; ok && c < nc; ++c) {
         const int s = c % kStages, buf = c & 1;
+        const int seg = c / kSegChunks, xb = seg & 1, first = c % kSegChunks == 0;
+        if (a.has_dx && first && seg >= 2 && !mbar_wait(&xr[xb], ((seg >> 1) - 1) & 1, a.err)) break;
         if (!mbar_wait(&conv[s], (c / kStages) & 1, a.err)) break;
         if (c >= 2 && !mbar_wait(&tfree[buf], ((c / 2) - 1) & 1, a.err)) break;
         tc_fence_after();
@@ -292,12 +497,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t bd = umma_desc_sw128(smem_u32(dzb(s)));
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
-            tc_mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc_dx, (c > 0 || kk > 0) ? 1u : 0u);
+            tc_mma_bf16(tmem + 192 * xb, ad + 2 * kk, bd + 2 * kk, idesc_dx,
+                        (!first || kk > 0) ? 1u : 0u);
         }
         const uint64_t bd = umma_desc_sw128(smem_u32(dztb(s)));
         for (int kk = 0; kk < kb; ++kk)
           tc_mma_bf16(tmem + 64 + 64 * buf, hd + 2 * kk, bd + 2 * kk, idesc_dw, kk > 0 ? 1u : 0u);
         tc_commit(&mdone[s]);
+        if (a.has_dx && (c % kSegChunks == kSegChunks - 1 || c == nc - 1)) tc_commit(&xf[xb]);
       }
       // Drain: the last commit covers every MMA issued before it.
       if (c > 0) mbar_wait(&mdone[(c - 1) % kStages], ((c - 1) / kStages) & 1, a.err);
@@ -306,6 +513,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---- warps 0-3: W^T for dX, the in-place SGD update, then the dX epilogue
     const int t = threadIdx.x;
     const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    // dX accumulator promoted to registers segment by segment (see kSegChunks)
+    float accx[64];
+#pragma unroll
+    for (int q = 0; q < 64; ++q) accx[q] = 0.f;
+    int drained = 0;
+    const int nseg = a.has_dx ? (nc + kSegChunks - 1) / kSegChunks : 0;
+    auto drain = [&]() -> bool {
+      const int xb = drained & 1;
+      if (!wait_warp(&xf[xb], (drained >> 1) & 1, a.err)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int cb = 0; cb < 64; cb += 16) {
+        if (cb < a.Bn) {
+          float v[16];
+          tmem_ld16(tbase + 192 * xb + cb, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 16; ++q) accx[cb + q] = __fadd_rn(accx[cb + q], v[q]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&xr[xb]);
+      ++drained;
+      return true;
+    };
     bool ok = true;
     for (int c = 0; c <= nc && ok; ++c) {
       if (c < nc) {
@@ -355,20 +587,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           mbar_arrive(&empty[sp]);
         }
+        if (a.has_dx && cp % kSegChunks == kSegChunks - 1 && cp / kSegChunks >= 1 &&
+            drained < cp / kSegChunks)
+          if (!drain()) { ok = false; break; }
       }
     }
+    while (ok && drained < nseg)
+      if (!drain()) ok = false;
     if (t == 0) tma_store_wait_all();
     if (ok && a.has_dx) {
-      // dX epilogue: TMEM lane t holds dH^T[i0 + t][0 .. Bn)
-      tc_fence_after();
+      // dX epilogue: thread t holds dH^T[i0 + t][0 .. Bn) in accx
       const int i = i0 + t;
       const bool valid = i < a.in;
       float db = 0.f;
-      for (int cb = 0; cb < a.Bn; cb += 16) {
-        float v[16];
-        tmem_ld16(tbase + cb, v);
-        tmem_ld_wait();
-        if (!valid) continue;
+#pragma unroll
+      for (int cb = 0; cb < 64; cb += 16) {
+        if (cb >= a.Bn || !valid) break;
+        const float* v = accx + cb;
         uint32_t pk[8];
 #pragma unroll
         for (int q = 0; q < 16; q += 2) {
@@ -448,19 +683,25 @@ __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __rest
 }
 
 // ------------------------------------------------------------------ cross-entropy
-// One CTA per learner.  p = softmax(z_b), dZ = (p - onehot(y_b)) / B in fp32;
-// loss_j = mean_b (log sum exp - z_{b,y_b}); b_L -= lr * sum_b dZ (fp32).
-__global__ void __launch_bounds__(256) k_xent_bf16(const float* __restrict__ Z,
-                                                  const int32_t* __restrict__ y, int64_t N,
-                                                  int64_t t, int B, int Bn, int Kp, int C,
-                                                  int pitch_c, float lr, float* bias_L,
-                                                  int64_t ld, __nv_bfloat16* dZ,
-                                                  __nv_bfloat16* dZT, float* loss) {
+// Softmax cross-entropy gradient when the classes span several output tiles.
+// Grid (P, class slices of 256).  Every CTA computes the per-sample statistics
+// (max, sum of exponentials over all C classes; warp per sample), then each
+// thread owns one class of its slice: dZ = (p - onehot(y_b)) / B in fp32 for
+// every sample, the bf16 operands dZ and dZ^T, and b_L -= lr * sum_b dZ (summed
+// in sample order).  Slice 0 also writes the learner's mean loss.
+constexpr int kXentThreads = 256;
+__global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restrict__ Z,
+                                                           const int32_t* __restrict__ y,
+                                                           int64_t N, int64_t t, int B, int Bn,
+                                                           int Kp, int C, int pitch_c, float lr,
+                                                           float* bias_L, int64_t ld,
+                                                           __nv_bfloat16* dZ, __nv_bfloat16* dZT,
+                                                           float* loss) {
   __shared__ float row_max[64], row_sum[64], row_loss[64];
   __shared__ int row_y[64];
   const int j = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* Zj = Z + static_cast<int64_t>(j) * B * C;
-  for (int b = warp; b < B; b += blockDim.x / 32) {
+  for (int b = warp; b < B; b += kXentThreads / 32) {
     const float* z = Zj + static_cast<int64_t>(b) * C;
     float m = -INFINITY;
     for (int c = lane; c < C; c += 32) m = fmaxf(m, z[c]);
@@ -479,19 +720,23 @@ __global__ void __launch_bounds__(256) k_xent_bf16(const float* __restrict__ Z,
     }
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (blockIdx.y == 0 && threadIdx.x == 0) {
     float l = 0.f;
     for (int b = 0; b < B; ++b) l += row_loss[b];
     loss[j] = l / B;
   }
+  const int c = blockIdx.y * kXentThreads + threadIdx.x;
+  if (c >= C) return;
   const float fB = static_cast<float>(B);
-  for (int c = threadIdx.x; c < C; c += blockDim.x) {
-    float db = 0.f;
-    for (int b0 = 0; b0 < Bn; b0 += 8) {
-      __align__(16) __nv_bfloat16 vals[8];
+  float db = 0.f;
+  for (int b0 = 0; b0 < Bn; b0 += 8) {
+    uint32_t pk[4];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int b = b0 + q;
+    for (int q = 0; q < 8; q += 2) {
+      float g2[2];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int b = b0 + q + e;
         float g = 0.f;
         if (b < B) {
           const float p = __fdiv_rn(expf(Zj[static_cast<int64_t>(b) * C + c] - row_max[b]), row_sum[b]);
@@ -499,14 +744,15 @@ __global__ void __launch_bounds__(256) k_xent_bf16(const float* __restrict__ Z,
           db = __fadd_rn(db, g);
           dZ[(static_cast<int64_t>(j) * Bn + b) * pitch_c + c] = __float2bfloat16_rn(g);
         }
-        vals[q] = __float2bfloat16_rn(g);
+        g2[e] = g;
       }
-      *reinterpret_cast<uint4*>(dZT + (static_cast<int64_t>(j) * C + c) * Kp + b0) =
-          *reinterpret_cast<uint4*>(vals);
+      pk[q / 2] = pack_bf16x2(g2[0], g2[1]);
     }
-    float* bp = bias_L + static_cast<int64_t>(j) * ld + c;
-    *bp = __fsub_rn(*bp, __fmul_rn(lr, db));
+    *reinterpret_cast<uint4*>(dZT + (static_cast<int64_t>(j) * C + c) * Kp + b0) =
+        make_uint4(pk[0], pk[1], pk[2], pk[3]);
   }
+  float* bp = bias_L + static_cast<int64_t>(j) * ld + c;
+  *bp = __fsub_rn(*bp, __fmul_rn(lr, db));
 }
 
 }  // namespace
@@ -523,7 +769,7 @@ cudaError_t tc_configure() {
 
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s) {
-  dim3 grid((a.out + 127) / 128, P);
+  dim3 grid(a.o_tiles, P, a.splits);
   k_tc_forward<<<grid, kThreads, kFwdSmem, s>>>(w_fwd, h_in, a);
   return cudaGetLastError();
 }
@@ -548,7 +794,8 @@ cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_
                              int Bn, int Kp, int C, int pitch_c, float lr, float* bias_L,
                              int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
                              int P, cudaStream_t s) {
-  k_xent_bf16<<<P, 256, 0, s>>>(Z, y, N, t, B, Bn, Kp, C, pitch_c, lr, bias_L, ld, dZ, dZT, loss);
+  dim3 grid(P, (C + kXentThreads - 1) / kXentThreads);
+  k_xent_bf16<<<grid, kXentThreads, 0, s>>>(Z, y, N, t, B, Bn, Kp, C, pitch_c, lr, bias_L, ld, dZ, dZT, loss);
   return cudaGetLastError();
 }
 

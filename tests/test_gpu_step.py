@@ -1,8 +1,17 @@
 """GPU parity of the learner step and of whole rounds (Algorithm 1, Sec. 3.1):
 the CUDA path, called through the C ABI, against the oracle on the same seeded
-inputs.  fp32 path: max relative error 1e-5; bf16-operand path: 1e-2 against
-an oracle that rounds the same operands to bf16.  The error is normwise per
-parameter tensor, max|gpu - oracle| / max|oracle|."""
+inputs.  Errors are normwise per parameter tensor, max|gpu - oracle| / max|oracle|.
+
+Tolerances.  fp32 path: 1e-5.  bf16-operand path: 1e-2 for the parameters after a
+step, against an oracle that rounds the same operands to bf16.  A bf16 rounding or
+ReLU decision taken on a value within rounding distance of its threshold can go
+either way under two valid fp32 accumulation orders, and such flips propagate
+through the layers (a 1-ulp bf16 flip in H_l moves Z_{l+1} by ~1e-4 relative,
+which flips more decisions there).  The spread this causes is measured, not
+guessed: the oracle is run a second time with fp32 accumulation ("bf16_acc32"),
+and the GPU must be within max(tolerance, SPREAD * that oracle-vs-oracle error).
+The update w_new - w_old itself is checked the same way (2e-2 floor), in the max
+norm and in the Frobenius norm."""
 import numpy as np
 import pytest
 import torch
@@ -15,6 +24,8 @@ from paper_1903_05133_gb300.inputs import initial_layers, learner_data, perturbe
 pytestmark = pytest.mark.gpu
 
 TOL = {"fp32": 1e-5, "bf16": 1e-2}
+UPDATE_TOL = {"fp32": 1e-5, "bf16": 2e-2}
+SPREAD = 3.0
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -27,12 +38,24 @@ def rel_err(got: np.ndarray, want: np.ndarray) -> float:
     return float(np.max(np.abs(got.astype(np.float64) - want.astype(np.float64))) / max(scale, 1e-30))
 
 
-def setup(w: configs.Workload, layers=None, N=None, data_device="cpu"):
+def frob_err(got: np.ndarray, want: np.ndarray) -> float:
+    d = np.linalg.norm((got.astype(np.float64) - want.astype(np.float64)).ravel())
+    return float(d / max(np.linalg.norm(want.astype(np.float64).ravel()), 1e-30))
+
+
+def setup(w: configs.Workload, layers=None, N=None, data_device="cpu", perturb=None):
     X, y = learner_data(w, device=data_device, N=N)
     if layers is None:
-        layers = initial_layers(w)
+        layers = initial_layers(w, device=data_device)
     ha = HierAvg(w.P, w.S, w.K1, w.K2, w.lr, w.B, w.dims, w.precision)
     params = ha.pack(layers)
+    if perturb is not None:
+        # distinct learner states with nonzero biases, drawn on the GPU
+        g = torch.Generator(device="cuda")
+        g.manual_seed(1234)
+        for Wl, bl in ha.unpack(params):
+            Wl.add_(torch.randn(Wl.shape, generator=g, device="cuda"), alpha=perturb[0])
+            bl.add_(torch.randn(bl.shape, generator=g, device="cuda"), alpha=perturb[1])
     ha.bind(params, X.cuda(), y.cuda())
     return ha, X, y
 
@@ -46,30 +69,75 @@ def oracle_params(ha: HierAvg, params_gpu: torch.Tensor, learners=None):
     return out
 
 
-def make_oracle(w, ha, X, y, params, learners=None):
+def make_oracle(w, ha, X, y, params, learners=None, mode=None):
     learners = list(range(w.P)) if learners is None else learners
-    Xn = X[learners].float().numpy()
-    yn = y[learners].numpy().astype(np.int64)
-    mode = "fp32" if w.precision == "fp32" else "bf16"
+    Xn = X[learners].float().cpu().numpy()
+    yn = y[learners].cpu().numpy().astype(np.int64)
+    if mode is None:
+        mode = "fp32" if w.precision == "fp32" else "bf16"
     prob = oracle.MLPProblem(Xn, yn, w.B, len(w.dims) - 1, mode)
     o = oracle.HierAvgOracle(len(learners), w.S if len(learners) % w.S == 0 else 1, w.K1, w.K2,
                              w.lr, prob, params, mode)
     return o
 
 
-def compare(ha, o, learners=None, tol=None, before=None, delta_tol=None):
+# A ReLU decision on a pre-activation within rounding distance of zero can go
+# either way even when both sides accumulate to ~1e-7; it swaps one sample's term
+# in one row of that layer's update.  Rows beyond the limit are accepted only if
+# the oracle's own pre-activation in that row is near zero, and only a few.
+NEAR_ZERO = 1e-3          # |z| <= NEAR_ZERO * max|z| of the layer
+MAX_FLIP_ROWS = 0.01      # at most this fraction of rows (and at least 3)
+
+
+def _explained(o, k, L, bad):
+    """Rows flagged `bad` ([learners, out]) of tensor k explained by near-zero
+    pre-activations of the layer that tensor feeds."""
+    layer = k // 2
+    if layer >= L - 1 or not getattr(o.problem, "last_preacts", None):
+        return False
+    near = np.array([np.any(np.abs(o.problem.last_preacts[jj][layer]) <=
+                            NEAR_ZERO * np.max(np.abs(o.problem.last_preacts[jj][layer])), axis=0)
+                     for jj in range(bad.shape[0])])
+    return bool(np.all(near[bad])) and bad.sum() <= max(3, MAX_FLIP_ROWS * bad.size)
+
+
+def _check(name, k, g, want, ref, lim_floor, fn, o, L, report):
+    e = fn(g, want)
+    lim = max(lim_floor, SPREAD * fn(ref, want)) if ref is not None else lim_floor
+    if report is not None:
+        report.append((k, name, e, lim))
+    if e <= lim:
+        return e
+    if fn is rel_err:
+        scale = np.max(np.abs(want))
+        rows = np.max(np.abs(g - want).reshape(g.shape[0], g.shape[1], -1), axis=2) / scale
+        if _explained(o, k, L, rows > lim):
+            return e
+    raise AssertionError(f"tensor {k}: {name} err {e:.3e} > {lim:.3e}")
+
+
+def compare(ha, o, learners=None, tol=None, before=None, o_ref=None, report=None):
+    """Check the GPU parameters against oracle `o` (and, with `before`, the update
+    itself).  With a second-order oracle `o_ref`, bf16 tolerances widen to SPREAD
+    times the oracle-vs-oracle error; rows beyond that must be explained by
+    near-zero ReLU inputs."""
     tol = TOL[ha.precision] if tol is None else tol
+    utol = UPDATE_TOL[ha.precision]
+    learners = list(range(ha.P)) if learners is None else learners
     got = oracle_params(ha, ha.params, learners)
     worst = 0.0
     for k, (g, want) in enumerate(zip(got, o.params)):
-        e = rel_err(g, want)
-        worst = max(worst, e)
-        assert e <= tol, f"tensor {k}: rel err {e:.3e} > {tol}"
-        if before is not None and delta_tol is not None:
-            dg, do = g.astype(np.float64) - before[k], want.astype(np.float64) - before[k]
-            if np.max(np.abs(do)) > 0:
-                ed = rel_err(dg, do)
-                assert ed <= delta_tol, f"tensor {k}: update rel err {ed:.3e} > {delta_tol}"
+        g, want = g.astype(np.float64), want.astype(np.float64)
+        ref = o_ref.params[k].astype(np.float64) if o_ref is not None else None
+        worst = max(worst, _check("param", k, g, want, ref, tol, rel_err, o, ha.L, report))
+        if before is None:
+            continue
+        b0 = before[k]
+        if np.max(np.abs(want - b0)) == 0:
+            continue
+        rb = ref - b0 if ref is not None else None
+        for name, fn in (("update-max", rel_err), ("update-frob", frob_err)):
+            _check(name, k, g - b0, want - b0, rb, utol, fn, o, ha.L, report)
     return worst
 
 
@@ -92,10 +160,13 @@ def test_one_step_from_distinct_learners(w):
     ha, X, y = setup(w, layers)
     start = oracle_params(ha, ha.params)
     o = make_oracle(w, ha, X, y, start)
+    o_ref = make_oracle(w, ha, X, y, start, mode="bf16_acc32") if w.precision == "bf16" else None
     ha.step()
     ha.check()
     o.step()
-    compare(ha, o, before=[a.astype(np.float64) for a in start], delta_tol=TOL[w.precision] * 2)
+    if o_ref is not None:
+        o_ref.step()
+    compare(ha, o, before=[a.astype(np.float64) for a in start], o_ref=o_ref)
     gl = ha.losses().numpy()
     assert np.allclose(gl, o.problem.last_loss, rtol=1e-3, atol=1e-4)
 
@@ -132,11 +203,12 @@ def test_literal_sequence_equals_round():
     assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
 
 
-def _force(o, ha):
-    """Load the GPU's current learner state into the oracle (teacher forcing)."""
+def _force(ha, *oracles):
+    """Load the GPU's current learner state into the oracles (teacher forcing)."""
     state = oracle_params(ha, ha.params)
-    o.params = [a.copy() for a in state]
-    o.t = ha.get_step()
+    for o in oracles:
+        o.params = [a.copy() for a in state]
+        o.t = ha.get_step()
     return [a.astype(np.float64) for a in state]
 
 
@@ -146,14 +218,16 @@ def test_round_teacher_forced(w):
     # (1e-2, and the update itself within 2e-2), every average bit-exact.
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
+    o_ref = make_oracle(w, ha, X, y, oracle_params(ha, ha.params), mode="bf16_acc32")
     worst = 0.0
     for b in range(w.K2):
         for k in range(w.K1):
-            before = _force(o, ha)
+            before = _force(ha, o, o_ref)
             ha.step()
             o.step()
-            worst = max(worst, compare(ha, o, before=before, delta_tol=2 * TOL["bf16"]))
-        _force(o, ha)
+            o_ref.step()
+            worst = max(worst, compare(ha, o, before=before, o_ref=o_ref))
+        _force(ha, o)
         if b + 1 < w.K2:
             ha.local_average()
             o.local_average()
@@ -169,23 +243,20 @@ def test_round_teacher_forced(w):
     print(f"{w.name}: worst per-step rel err {worst:.3e}")
 
 
-# After K1*K2 compounded steps the two sides differ by more than one step's
-# rounding: valid accumulation orders differ, so a few ReLU-mask and bf16
-# rounding decisions near their thresholds flip and propagate.  Biases start at
-# zero, so their normwise scale is small and they show it first.  The end-to-end
-# round is therefore held to 5e-2; the contract (1e-2 per step) is checked above.
-E2E_TOL = 5e-2
-
-
 def test_mlp512_round_end_to_end():
+    # A whole round without teacher forcing: decision flips compound over the
+    # K1*K2 steps, so the bound is SPREAD times the oracle-vs-oracle drift.
     w = configs.MLP512_P16
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
+    o_ref = make_oracle(w, ha, X, y, oracle_params(ha, ha.params), mode="bf16_acc32")
     ha.round()
     o.round()
+    o_ref.round()
     ha.check()
-    worst = compare(ha, o, tol=E2E_TOL)
-    print(f"{w.name}: end-to-end round rel err {worst:.3e}")
+    report = []
+    compare(ha, o, o_ref=o_ref, report=report)
+    print(w.name, "end-to-end:", [(k, f"{e:.2e}", f"{lim:.2e}") for k, _, e, lim in report])
 
 
 @pytest.mark.parametrize("w", [configs.MLP2048_P64, configs.MLP4096_P32], ids=lambda w: w.name)
@@ -193,15 +264,19 @@ def test_full_size_step_sampled(w):
     # Full-size model, P and B (the launch configuration the bench times); the
     # oracle recomputes the first and the last learner one by one.
     w = w.replace(N=4 * w.B)
-    ha, X, y = setup(w)
+    ha, X, y = setup(w, data_device="cuda", perturb=(0.002, 0.05))
     learners = [0, w.P - 1]
     start = oracle_params(ha, ha.params, learners)
     o = make_oracle(w, ha, X, y, start, learners)
+    o_ref = make_oracle(w, ha, X, y, start, learners, mode="bf16_acc32")
     ha.step()
     ha.check()
     o.step()
-    compare(ha, o, learners, before=[a.astype(np.float64) for a in start],
-            delta_tol=TOL["bf16"] * 2)
+    o_ref.step()
+    report = []
+    compare(ha, o, learners, before=[a.astype(np.float64) for a in start], o_ref=o_ref,
+            report=report)
+    print(w.name, [(k, kind, f"{e:.2e}", f"{lim:.2e}") for k, kind, e, lim in report])
 
 
 def test_round_host_matches_device_round():

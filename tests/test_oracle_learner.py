@@ -106,7 +106,7 @@ def test_mlp_gradient_against_autograd():
         assert np.allclose(gb[l], tb[l].grad.numpy(), rtol=1e-12, atol=1e-14)
 
 
-@pytest.mark.parametrize("mode,tol", [("fp32", 1e-5), ("bf16", 3e-2)])
+@pytest.mark.parametrize("mode,tol", [("fp32", 1e-5), ("bf16", 3e-2), ("bf16_acc32", 3e-2)])
 def test_reduced_precision_modes_track_f64(mode, tol):
     Ws, bs, X, y = _tiny_net((64, 48, 10), 16, 13)
     X = ln.bf16_round(X.astype(np.float32)).astype(np.float64)
