@@ -157,7 +157,11 @@ def launches_per_round(w) -> int:
         for t in steps:
             if (t * w.B) % w.N + w.B > w.N:
                 gathers += 1
-        per_step = L + (0 if w.dims[-1] <= 128 else 1) + L
+        C, din = w.dims[-1], w.dims[-2]
+        if C <= 16 and din % 64 == 0 and w.B <= 64:      # fused last-layer kernel
+            per_step = (L - 1) + 1 + (L - 1)
+        else:
+            per_step = L + (0 if C <= 128 else 1) + L
         n = w.K1 * w.K2 * per_step + gathers
     else:
         per_step = 1 + L + 1 + L + (L - 1)       # dX is its own launch for layers > 1
@@ -280,10 +284,20 @@ def run_ours(args):
     per_round = w.samples_per_round
     value = ws * per_round * args.steps / T
 
-    kinds = ["gather", "forward", "xent", "backward", "local_avg", "global_avg"]
+    kinds = ["gather", "forward", "xent", "backward", "local_avg", "global_avg", "head"]
     prof = {k: ha.profile_read(k) for k in kinds}
     ha.profile(False)
-    main_kinds = ["forward", "backward", "local_avg", "global_avg", "xent", "gather"]
+    # the same rounds again without per-kernel events (host-overhead check, untimed)
+    plain_ms = []
+    for k in range(min(args.steps, 10)):
+        flush.zero_()
+        a_ev, b_ev = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_ev.record()
+        ha.round()
+        b_ev.record()
+        torch.cuda.synchronize()
+        plain_ms.append(a_ev.elapsed_time(b_ev))
+    main_kinds = ["forward", "backward", "local_avg", "global_avg", "xent", "gather", "head"]
     dom = max(main_kinds, key=lambda k: prof[k][0])
     pk, pk_src = peaks()
     dom_ms, dom_n, dom_bytes = prof[dom]
@@ -318,6 +332,7 @@ def run_ours(args):
                           "frac_of_measured_hbm": (avg_by / (avg_ms / 1e3) / 1e9 / pk["hbm_gbs"]) if avg_ms > 0 else None,
                           "frac_of_8TBps": (avg_by / (avg_ms / 1e3) / 8e12) if avg_ms > 0 else None},
             "kernels": kernels,
+            "ms_per_step_without_kernel_events": statistics.median(plain_ms),
             "gpu_launches": launches_per_round(w) * args.steps,
             "clocks": clocks}
 

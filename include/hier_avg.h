@@ -83,7 +83,7 @@ typedef struct hier_avg hier_avg;
  *   precision           : HA_PREC_FP32 or HA_PREC_BF16
  * Errors: HA_EINVAL for P, S, K1, K2, B < 1, P % S != 0, non-finite lr, bad dims or
  * precision; HA_EUNSUPPORTED for a shape the kernels do not cover (BF16: B > 64 or
- * an input width d_0 .. d_{L-1} not a multiple of 8; FP32: B > 1024). */
+ * an input width d_0 .. d_{L-1} not a multiple of 8; either: P > 65535). */
 int hier_avg_create(int P, int S, int K1, int K2, float lr, int B, const int* dims,
                     int n_dims, int precision, hier_avg** out);
 
@@ -158,7 +158,8 @@ int hier_avg_check(hier_avg* h);
 #define HA_KERNEL_BACKWARD      3   /* fused dX + dW + SGD update            */
 #define HA_KERNEL_LOCAL_AVG     4
 #define HA_KERNEL_GLOBAL_AVG    5   /* fused last local + global average     */
-#define HA_KERNEL_KINDS         6
+#define HA_KERNEL_HEAD          6   /* fused last layer (<= 16 classes)      */
+#define HA_KERNEL_KINDS         7
 int hier_avg_profile(hier_avg* h, int enable);
 
 /* Synchronise and read kind's totals since profiling was enabled: summed event

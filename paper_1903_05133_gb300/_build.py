@@ -19,7 +19,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libhier_avg.so")
 
-SOURCES = ["hier_avg_api.cu", "avg_kernels.cu", "step_tc.cu", "step_fp32.cu"]
+SOURCES = ["hier_avg_api.cu", "avg_kernels.cu", "step_tc.cu", "step_head.cu", "step_fp32.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-ftz=false",
           "-prec-div=true", "-prec-sqrt=true", f"-I{INCLUDE}", f"-I{CSRC}"]

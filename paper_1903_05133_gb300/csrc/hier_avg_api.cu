@@ -66,6 +66,7 @@ struct hier_avg {
   int64_t off_part = 0, off_cnt = 0;          // split-K partials and tile counters
   std::vector<int> fwd_splits, fwd_tiles;     // per layer
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
+  bool head = false;                          // d_L <= 16: fused last-layer kernel
   // binding
   bool bound = false;
   int device = 0;
@@ -191,6 +192,7 @@ int plan_layout(hier_avg* h) {
       max_tiles = std::max(max_tiles, tiles);
     }
     h->fused_xent = h->dims[L] <= 128;
+    h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B));
     h->off_part = take(std::max<int64_t>(part_bytes, 16));
     h->off_cnt = take(P * max_tiles * 4);
   } else {
@@ -309,7 +311,8 @@ int do_step(hier_avg* h) {
       }, "gather");
       if (rc) return rc;
     }
-    for (int l = 0; l < L; ++l) {
+    const int n_fwd = h->head ? L - 1 : L;
+    for (int l = 0; l < n_fwd; ++l) {
       TcFwdArgs a{};
       a.in = h->dims[l];
       a.out = h->dims[l + 1];
@@ -352,7 +355,34 @@ int do_step(hier_avg* h) {
       if (rc) return rc;
     }
     const int C = h->dims[L];
-    if (!h->fused_xent) {
+    if (h->head) {
+      ha::HeadArgs a{};
+      a.C = C;
+      a.in = h->dims[L - 1];
+      a.B = B;
+      a.Bn = h->Bn;
+      a.Kp = h->Kp;
+      a.pitch_in = h->pitch[L - 1];
+      a.ld = h->ld;
+      a.N = h->N;
+      a.t = h->t;
+      a.lr = h->lr;
+      a.W = h->params + h->woff[L - 1];
+      a.bias = h->params + h->boff[L - 1];
+      a.x_rows = L == 1;
+      a.H = L == 1 ? static_cast<const __nv_bfloat16*>(h->X) : h->wsp<__nv_bfloat16>(h->off_H[L - 1]);
+      a.y = h->y;
+      a.has_dx = L > 1;
+      if (L > 1) {
+        a.bias_prev = h->params + h->boff[L - 2];
+        a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[L - 1]);
+        a.dzt_prev = h->wsp<__nv_bfloat16>(h->off_dZT[L - 1]);
+      }
+      a.loss = h->loss();
+      const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0));
+      rc = h->timed(HA_KERNEL_HEAD, hb, [&] { return ha::launch_head(a, P, s); }, "head");
+      if (rc) return rc;
+    } else if (!h->fused_xent) {
       rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
         return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, h->Kp, C,
                                     h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
@@ -361,7 +391,7 @@ int do_step(hier_avg* h) {
       }, "xent");
       if (rc) return rc;
     }
-    for (int l = L - 1; l >= 0; --l) {
+    for (int l = h->head ? L - 2 : L - 1; l >= 0; --l) {
       TcBwdArgs a{};
       a.in = h->dims[l];
       a.out = h->dims[l + 1];
@@ -581,6 +611,7 @@ int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t w
   if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_bytes, h->stream), "bind: memset"))) return rc;
   if (h->prec == HA_PREC_BF16) {
     if ((rc = h->cuda(ha::tc_configure(), "bind: kernel attributes"))) return rc;
+    if ((rc = h->cuda(ha::head_configure(), "bind: kernel attributes"))) return rc;
     if ((rc = build_maps(h))) return rc;
   }
   h->bound = true;

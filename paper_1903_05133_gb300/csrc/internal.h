@@ -86,6 +86,28 @@ cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_
                              int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
                              int P, cudaStream_t s);
 
+// Fused last layer for <= 16 classes (forward, softmax CE, backward), one CTA per
+// learner on CUDA cores.
+struct HeadArgs {
+  int C, in, B, Bn, Kp, pitch_in;
+  int64_t ld, N, t;
+  float lr;
+  float* W;                   // learner 0's W_L [C][in] (fp32 master)
+  float* bias;                // learner 0's b_L
+  const __nv_bfloat16* H;     // H_{L-1} [P][Bn][pitch_in], or X [P][N][in] when x_rows
+  int x_rows;
+  const int32_t* y;
+  int has_dx;                 // write dZ_{L-1} / dZT_{L-1} and update b_{L-1}
+  float* bias_prev;
+  __nv_bfloat16* dz_prev;     // [P][Bn][pitch_in]
+  __nv_bfloat16* dzt_prev;    // [P][in][Kp]
+  float* loss;                // [P]
+};
+bool head_supported(int C, int in, int B);
+int head_smem_bytes(int C, int in, int B);
+cudaError_t head_configure();   // raises the dynamic shared-memory limit once
+cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s);
+
 // ----------------------------------------------------------------- fp32 CUDA-core step
 // Buffers: H_l [P][B][d_l] fp32, Z_L [P][B][d_L], dZ_l [P][B][d_l] fp32.
 cudaError_t launch_gather_f32(const float* X, int64_t N, int d0, int B, int64_t t, int P,

@@ -147,13 +147,28 @@ SMALL_BF16 = configs.Workload("tiny_mlp_bf16", P=4, S=2, K1=2, K2=2, rounds=1,
 RAGGED_BF16 = configs.Workload("ragged_mlp_bf16", P=6, S=3, K1=1, K2=2, rounds=1,
                                dims=(264, 136, 200, 13), precision="bf16", N=50, B=20, lr=0.05,
                                sigma_mu=0.1, init="he")
+SOFTMAX_BF16 = configs.Workload("softmax_bf16", P=4, S=2, K1=2, K2=2, rounds=1, dims=(256, 10),
+                                precision="bf16", N=64, B=16, lr=0.05, sigma_mu=0.1, init="he")
+WIDE_SOFTMAX_BF16 = configs.Workload("softmax_bf16_c40", P=4, S=2, K1=1, K2=2, rounds=1,
+                                     dims=(256, 40), precision="bf16", N=48, B=16, lr=0.05,
+                                     sigma_mu=0.1, init="he")
+MANY_CLASSES_BF16 = configs.Workload("mlp_bf16_c300", P=4, S=4, K1=1, K2=2, rounds=1,
+                                     dims=(128, 64, 300), precision="bf16", N=64, B=32, lr=0.05,
+                                     sigma_mu=0.1, init="he")
 SMALL_FP32 = configs.Workload("tiny_mlp_fp32", P=4, S=2, K1=2, K2=2, rounds=1,
                               dims=(100, 37, 10), precision="fp32", N=40, B=7, lr=0.05,
                               sigma_mu=0.1, init="he")
 
 
-@pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, RAGGED_BF16,
-                               configs.MLP512_P16], ids=lambda w: w.name)
+# Last-layer paths: fused head kernel (<= 16 classes; SMALL_BF16, SOFTMAX_BF16 which
+# reads X directly, the 16-learner MLP), tensor-core forward with the CE in its
+# epilogue (RAGGED_BF16: 13 classes over a 200-wide ragged input; WIDE_SOFTMAX_BF16),
+# and the standalone CE kernel (MANY_CLASSES_BF16: 300 classes over 3 tiles).
+STEP_CASES = [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16, WIDE_SOFTMAX_BF16,
+              RAGGED_BF16, MANY_CLASSES_BF16, configs.MLP512_P16]
+
+
+@pytest.mark.parametrize("w", STEP_CASES, ids=lambda w: w.name)
 def test_one_step_from_distinct_learners(w):
     # Learners start from different parameters, so every learner's step is checked.
     layers = perturbed_layers(w, 0.01, seed=1)
@@ -171,16 +186,21 @@ def test_one_step_from_distinct_learners(w):
     assert np.allclose(gl, o.problem.last_loss, rtol=1e-3, atol=1e-4)
 
 
-@pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, RAGGED_BF16],
+@pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16,
+                               WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16],
                          ids=lambda w: w.name)
 def test_full_run_against_oracle(w):
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
+    o_ref = (make_oracle(w, ha, X, y, oracle_params(ha, ha.params), mode="bf16_acc32")
+             if w.precision == "bf16" else None)
     for _ in range(w.rounds):
         ha.round()
         o.round()
+        if o_ref is not None:
+            o_ref.round()
     ha.check()
-    compare(ha, o)
+    compare(ha, o, o_ref=o_ref)
     # every learner holds the same parameters after the global average
     p = ha.params.cpu().numpy().view(np.uint32)
     assert np.all(p == p[0])
