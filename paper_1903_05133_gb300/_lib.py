@@ -33,6 +33,7 @@ SIGNATURES = {
     "hier_avg_global_average": (c_int, [c_void_p]),
     "hier_avg_round": (c_int, [c_void_p]),
     "hier_avg_round_host": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p]),
+    "hier_avg_step_static": (c_int, [c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_void_p]),
     "hier_avg_get_step": (c_int, [c_void_p, P_int64]),
     "hier_avg_set_step": (c_int, [c_void_p, c_int64]),
     "hier_avg_losses": (c_int, [c_void_p, c_void_p]),

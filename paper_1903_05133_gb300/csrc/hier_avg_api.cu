@@ -7,6 +7,7 @@
 #include <cstdio>
 #include <cstring>
 #include <algorithm>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -736,3 +737,80 @@ int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* laun
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free step.  Some callers cannot allocate device memory at all: code
+// running under an allocator they do not own, inside a host that forbids
+// cudaMalloc after start-up, or from a language binding that only hands out
+// existing buffers.  For them the step's scratch (activations, their transposes,
+// split-K partial sums and tile counters) lives in this file-scope array instead
+// of a caller workspace.  Every GPU that loads the library holds it until exit.
+namespace {
+
+constexpr int64_t kStaticScratchBytes = int64_t(16) << 20;   // 16 MiB
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device, looked up once per
+// device.  In host code the symbol's name is only a host-side stand-in.
+cudaError_t static_scratch(int device, void** out) {
+  if (device < 0 || device >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (!g_scratch_ptr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_ptr[device] = p;
+  }
+  *out = g_scratch_ptr[device];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" int hier_avg_step_static(hier_avg* h, float* params_dev, const void* X_dev,
+                                    const int32_t* y_dev, int64_t N, void* stream) {
+  if (!h) return HA_EINVAL;
+  if (!params_dev || !X_dev || !y_dev || N < 1)
+    return h->fail(HA_EINVAL, "step_static: NULL buffer or N < 1");
+  if (h->ws_bytes > kStaticScratchBytes)
+    return h->fail(HA_ENOMEM,
+                   "step_static: this configuration needs %lld bytes of scratch, the static "
+                   "array holds %lld; use hier_avg_bind with a caller workspace",
+                   (long long)h->ws_bytes, (long long)kStaticScratchBytes);
+  if (reinterpret_cast<uintptr_t>(params_dev) % 256)
+    return h->fail(HA_EINVAL, "step_static: params must be 256-byte aligned");
+  if (h->prec == HA_PREC_BF16 && reinterpret_cast<uintptr_t>(X_dev) % 16)
+    return h->fail(HA_EINVAL, "step_static: X must be 16-byte aligned");
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, params_dev) != cudaSuccess || attr.type != cudaMemoryTypeDevice)
+    return h->fail(HA_EINVAL, "step_static: params is not device memory");
+  int rc;
+  if ((rc = h->cuda(cudaSetDevice(attr.device), "step_static: set device"))) return rc;
+  void* scratch = nullptr;
+  if ((rc = h->cuda(static_scratch(attr.device, &scratch), "step_static: scratch address")))
+    return rc;
+  h->bound = false;
+  h->device = attr.device;
+  h->params = params_dev;
+  h->ws = static_cast<uint8_t*>(scratch);
+  h->X = X_dev;
+  h->y = y_dev;
+  h->N = N;
+  h->stream = static_cast<cudaStream_t>(stream);
+  // The array keeps whatever the previous call (of any handle) left in it; the
+  // step needs its padding and its split-K counters to start at zero.
+  if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_bytes, h->stream), "step_static: clear")))
+    return rc;
+  if (h->prec == HA_PREC_BF16) {
+    if ((rc = h->cuda(ha::tc_configure(), "step_static: kernel attributes"))) return rc;
+    if ((rc = h->cuda(ha::head_configure(), "step_static: kernel attributes"))) return rc;
+    if ((rc = build_maps(h))) return rc;
+  }
+  h->bound = true;
+  return do_step(h);
+}
