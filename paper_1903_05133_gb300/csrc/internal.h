@@ -86,8 +86,8 @@ cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_
                              int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
                              int P, cudaStream_t s);
 
-// Fused last layer for <= 16 classes (forward, softmax CE, backward), one CTA per
-// learner on CUDA cores.
+// Small last layer (<= 16 classes) on CUDA cores: a per-learner forward + softmax-CE
+// kernel and a per-feature-slice backward kernel, linked by the scratch `gq`.
 struct HeadArgs {
   int C, in, B, Bn, Kp, pitch_in;
   int64_t ld, N, t;
@@ -102,9 +102,10 @@ struct HeadArgs {
   __nv_bfloat16* dz_prev;     // [P][Bn][pitch_in]
   __nv_bfloat16* dzt_prev;    // [P][in][Kp]
   float* loss;                // [P]
+  float* gq;                  // scratch: bf16-rounded CE gradient [P][Bn][16]
 };
 bool head_supported(int C, int in, int B);
-int head_smem_bytes(int C, int in, int B);
+int head_scratch_floats(int P, int Bn);
 cudaError_t head_configure();   // raises the dynamic shared-memory limit once
 cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s);
 

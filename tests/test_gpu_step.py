@@ -155,17 +155,20 @@ WIDE_SOFTMAX_BF16 = configs.Workload("softmax_bf16_c40", P=4, S=2, K1=1, K2=2, r
 MANY_CLASSES_BF16 = configs.Workload("mlp_bf16_c300", P=4, S=4, K1=1, K2=2, rounds=1,
                                      dims=(128, 64, 300), precision="bf16", N=64, B=32, lr=0.05,
                                      sigma_mu=0.1, init="he")
+HEAD_C13 = configs.Workload("mlp_bf16_c13", P=4, S=2, K1=1, K2=2, rounds=1, dims=(192, 128, 13),
+                            precision="bf16", N=48, B=24, lr=0.05, sigma_mu=0.1, init="he")
 SMALL_FP32 = configs.Workload("tiny_mlp_fp32", P=4, S=2, K1=2, K2=2, rounds=1,
                               dims=(100, 37, 10), precision="fp32", N=40, B=7, lr=0.05,
                               sigma_mu=0.1, init="he")
 
 
-# Last-layer paths: fused head kernel (<= 16 classes; SMALL_BF16, SOFTMAX_BF16 which
-# reads X directly, the 16-learner MLP), tensor-core forward with the CE in its
+# Last-layer paths: CUDA-core head kernels (<= 16 classes; SMALL_BF16, SOFTMAX_BF16 which
+# reads X directly, the 16-learner MLP, HEAD_C13 with a class count that is not the
+# specialised 10), tensor-core forward with the CE in its
 # epilogue (RAGGED_BF16: 13 classes over a 200-wide ragged input; WIDE_SOFTMAX_BF16),
 # and the standalone CE kernel (MANY_CLASSES_BF16: 300 classes over 3 tiles).
-STEP_CASES = [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16, WIDE_SOFTMAX_BF16,
-              RAGGED_BF16, MANY_CLASSES_BF16, configs.MLP512_P16]
+STEP_CASES = [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16, HEAD_C13,
+              WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16, configs.MLP512_P16]
 
 
 @pytest.mark.parametrize("w", STEP_CASES, ids=lambda w: w.name)
@@ -187,7 +190,7 @@ def test_one_step_from_distinct_learners(w):
 
 
 @pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16,
-                               WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16],
+                               HEAD_C13, WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16],
                          ids=lambda w: w.name)
 def test_full_run_against_oracle(w):
     ha, X, y = setup(w)
