@@ -141,7 +141,7 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host,
  * own, or a binding that only passes existing buffers).  The paper has no
  * counterpart: this is a property of the library, not of the method.
  * The caller passes the inputs and outputs (params_dev [P, ld] updated in place,
- * X_dev, y_dev, N as for hier_avg_bind); the step's scratch lives in one 16 MiB
+ * X_dev, y_dev, N as for hier_avg_bind); the step's scratch lives in one 32 MiB
  * array that the library holds in every GPU's memory until the process exits.
  * The call binds the handle to these buffers and to that array, clears the part
  * of the array the step uses, takes the step at the handle's counter t and
@@ -153,7 +153,7 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host,
  *     threads) race on it.  After a call, later hier_avg_step / round calls of
  *     the same handle also use the array until hier_avg_bind is called again.
  * Errors: HA_ENOMEM (with a message naming both sizes) when the configuration
- * needs more than 16 MiB of scratch (hier_avg_workspace_bytes), HA_EINVAL for
+ * needs more than 32 MiB of scratch (hier_avg_workspace_bytes), HA_EINVAL for
  * NULL or misaligned buffers or N < 1, HA_ECUDA. */
 int hier_avg_step_static(hier_avg* h, float* params_dev, const void* X_dev,
                          const int32_t* y_dev, int64_t N, void* stream);

@@ -22,7 +22,7 @@ using ha::TcBwdArgs;
 using ha::TcFwdArgs;
 
 constexpr int64_t kAlign = 1024;
-constexpr int64_t kTargetCtas = 152;   // one wave: the forward kernel fits one CTA per SM
+constexpr int64_t kTargetCtas = 152;   // persistent forward: one CTA per SM of a GB300
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -66,7 +66,7 @@ struct hier_avg {
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
   int64_t off_part = 0, off_cnt = 0;          // split-K partials and tile counters
   int64_t off_gq = 0;                         // small-head CE gradient
-  std::vector<int> fwd_splits, fwd_tiles;     // per layer
+  std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
   bool head = false;                          // d_L <= 16: fused last-layer kernel
   // binding
@@ -177,27 +177,25 @@ int plan_layout(hier_avg* h) {
       h->off_dZ[l] = take(P * h->Bn * h->pitch[l] * 2);
       h->off_dZT[l] = take(P * h->dims[l] * h->Kp * 2);
     }
-    // Split-K plan of the forward GEMMs: about one wave of CTAs on the 152 SMs.
-    // It depends on the shapes only, so the summation order is the same on every GPU.
-    h->fwd_splits.assign(L, 1);
+    // Stream-K plan of the forward GEMMs: at most one persistent CTA per SM of a
+    // GB300 (152).  It depends on the shapes only, so the summation order of split
+    // tiles is the same on every GPU.
+    h->fwd_ctas.assign(L, 1);
     h->fwd_tiles.assign(L, 1);
-    int64_t part_bytes = 0, max_tiles = 1;
+    int64_t part_bytes = 16, max_tiles = 1;
     for (int l = 0; l < L; ++l) {
       const int64_t tiles = (h->dims[l + 1] + 127) / 128, nk = (h->dims[l] + 63) / 64;
-      int64_t splits = kTargetCtas / (tiles * P);   // never more than one wave
-      splits = std::max<int64_t>(1, std::min<int64_t>(splits, nk));
-      const int64_t per = (nk + splits - 1) / splits;
-      splits = (nk + per - 1) / per;
-      h->fwd_splits[l] = static_cast<int>(splits);
+      const int64_t units = tiles * P * nk;
+      h->fwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, units));
       h->fwd_tiles[l] = static_cast<int>(tiles);
-      if (splits > 1) part_bytes = std::max(part_bytes, P * tiles * splits * 128 * h->Bn * 4);
-      max_tiles = std::max(max_tiles, tiles);
+      part_bytes = std::max(part_bytes, int64_t(h->fwd_ctas[l]) * 128 * h->Bn * 4);
+      max_tiles = std::max(max_tiles, tiles * P);
     }
     h->fused_xent = h->dims[L] <= 128;
     h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B));
-    h->off_part = take(std::max<int64_t>(part_bytes, 16));
+    h->off_part = take(part_bytes);
     h->off_gq = take(h->head ? int64_t(ha::head_scratch_floats(h->P, h->Bn)) * 4 : 16);
-    h->off_cnt = take(P * max_tiles * 4);
+    h->off_cnt = take(max_tiles * 4);
   } else {
     for (int l = 0; l <= L; ++l) h->pitch[l] = h->dims[l];
     for (int l = 0; l < L; ++l) h->off_H[l] = take(P * B * h->dims[l] * 4);
@@ -324,8 +322,9 @@ int do_step(hier_avg* h) {
       a.Kp = h->Kp;
       a.ld = h->ld;
       a.bias = h->params + h->boff[l];
-      a.splits = h->fwd_splits[l];
+      a.ctas = h->fwd_ctas[l];
       a.o_tiles = h->fwd_tiles[l];
+      a.n_tiles = h->fwd_tiles[l] * P;
       a.part = h->wsp<float>(h->off_part);
       a.counters = h->wsp<int>(h->off_cnt);
       a.x_direct = (l == 0 && x_direct) ? 1 : 0;
@@ -750,7 +749,7 @@ int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* laun
 // of a caller workspace.  Every GPU that loads the library holds it until exit.
 namespace {
 
-constexpr int64_t kStaticScratchBytes = int64_t(16) << 20;   // 16 MiB
+constexpr int64_t kStaticScratchBytes = int64_t(32) << 20;   // 32 MiB
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];

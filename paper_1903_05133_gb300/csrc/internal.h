@@ -37,10 +37,12 @@ struct TcFwdArgs {
   int pitch_out;              // mode 0: H pitch; mode 2: dZ_L pitch
   __nv_bfloat16* ht_out;      // mode 0: HT_{l+1} [P][out][Kp]
   float* z_out;               // mode 1: Z_L [P][B][out]
-  // split-K over the input features: grid.z = splits; partial accumulators go to
-  // part [P][o_tiles][splits][128][Bn] and the last CTA of a tile (counted in
-  // counters [P][o_tiles], reset by that CTA) sums them in split order.
-  int splits, o_tiles;
+  // persistent stream-K schedule: `ctas` CTAs share the n_tiles x ceil(in/64) units
+  // (tile = learner x 128 outputs) evenly.  A split tile is finished by the CTA that
+  // holds its first chunk; each other contributor writes its partial to its slot of
+  // part [ctas][128][Bn] and bumps counters[tile] (reset to 0 by the finisher), and
+  // the finisher adds the partials in CTA order.
+  int ctas, n_tiles, o_tiles;
   float* part;
   int* counters;
   // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)

@@ -56,6 +56,27 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* e
   }
 }
 
+// ------------------------------------------------ cross-CTA flags (global)
+// Add to a global counter with release order (prior writes of this thread, and
+// those it has observed, are visible before the new value); nothing is returned.
+__device__ __forceinline__ void red_release_add(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Wait, bounded, until *p == want, reading with acquire order.
+__device__ __forceinline__ bool spin_acquire_eq(const int* p, int want, int* err) {
+  const long long t0 = clock64();
+  while (true) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    if (v == want) return true;
+    if (clock64() - t0 > kWaitLimitCycles) {
+      if (err) atomicOr(err, HA_DEVERR_TIMEOUT);
+      return false;
+    }
+    __nanosleep(32);
+  }
+}
+
 // ---------------------------------------------------------------- fences
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

@@ -41,23 +41,56 @@ constexpr int kThreads = 192;          // warps 0-3 convert/epilogue, 4 TMA, 5 M
 constexpr int kConv = 128;
 
 // ------------------------------------------------------------------ forward
-// Shared memory: a 4-deep ring of TMA stages (fp32 W tile + bf16 batch tile) and a
-// double-buffered bf16 A tile that the converter warps fill for the MMA.
-constexpr int kFwdStages = 4;
+// Persistent stream-K forward.  The work of one layer is a list of units
+// u = (tile, chunk): tile = (learner j, 128 output features), chunk = 64 input
+// features.  CTA g of G owns the contiguous units [g*U/G, (g+1)*U/G), so every SM
+// streams the same number of chunks and the TMA ring runs straight across tile
+// boundaries.  A tile whose chunks are spread over several CTAs is finished by
+// the contributor that arrives last: it sums the published partial accumulators
+// in CTA order (deterministic) and runs the epilogue.
+// Warps 0-7 convert the fp32 weight tiles to bf16 and own the accumulator rows:
+// warp w serves TMEM lanes 32*(w%4).., and the two warps on the same lanes split
+// the batch columns in interleaved 16-column blocks (group w/4 takes blocks
+// 2m + w/4).  Warp 8 issues TMA, warp 9 the MMAs.
+// Shared memory: two TMA rings, the fp32 weight tiles (released by the converter
+// warps as soon as they have read them, so conversion and MMA latency stay out of
+// the weight stream) and the bf16 batch tiles (released by the MMA); a
+// double-buffered bf16 A tile the converter warps fill for the MMA; and (fused
+// cross-entropy only) a staging area for the epilogue.  The MMA of chunk i waits
+// for batch tile i, which is reloaded only after the MMA nh chunks earlier, so the
+// batch ring takes all the shared memory left (its tiles are Bn x 128 bytes).
+constexpr int kFwdConv = 256;
+constexpr int kFwdThreads = kFwdConv + 64;
+constexpr int kFwdWRingMax = 5, kFwdHRingMax = 8;
 constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile
-constexpr int kFwdH = 64 * 128;                        //  8 KB bf16 B tile (Bn <= 64)
-constexpr int kFwdStage = kFwdWf32 + kFwdH;            // 40 KB
 constexpr int kFwdWbf = 128 * 64 * 2;                  // 16 KB bf16 A tile (x2)
-constexpr int kFwdWbfOff = kFwdStages * kFwdStage;
-constexpr int kFwdBarOff = kFwdWbfOff + 2 * kFwdWbf;
-constexpr int kFwdSmem = kFwdBarOff + 256 + 1024;      // + barriers + alignment slack
+constexpr int kFwdSmemMax = 227 * 1024;
+constexpr int kXentSmem = (2 * 128 * 65 + 4 * 64) * 4; // logits, gradients, statistics
 // The tensor core's fp32 accumulation loses precision roughly in proportion to the
 // number of MMAs chained into one accumulator, so the accumulator is promoted:
 // every kSegChunks chunks (16 MMAs) the partial sum is folded into fp32 registers
 // with IEEE adds, in chunk order, while the MMAs continue in the other TMEM buffer.
 constexpr int kSegChunks = 4;
 constexpr uint32_t kFwdTmemCols = 128;   // two accumulator buffers of 64 columns
-constexpr int kFwdHidden = 0, kFwdLogits = 1, kFwdXent = 2;   // TcFwdArgs::mode
+constexpr int kFwdHidden = 0, kFwdXent = 2;   // TcFwdArgs::mode (1 = logits)
+
+// Layout: W ring | A tiles | epilogue staging (mode 2) | batch ring | barriers.
+__host__ __device__ constexpr int fwd_wring(int mode) { return mode == 2 ? 3 : 5; }
+__host__ __device__ constexpr int fwd_h_off(int mode) {
+  return fwd_wring(mode) * kFwdWf32 + 2 * kFwdWbf + (mode == 2 ? kXentSmem : 0);
+}
+__host__ __device__ constexpr int fwd_hring(int mode, int Bn) {
+  return (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode)) / (Bn * 128) < kFwdHRingMax
+             ? (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode)) / (Bn * 128)
+             : kFwdHRingMax;
+}
+__host__ __device__ constexpr int fwd_bar_off(int mode, int Bn) {
+  return fwd_h_off(mode) + fwd_hring(mode, Bn) * Bn * 128;
+}
+__host__ __device__ constexpr int fwd_smem(int mode, int Bn) { return fwd_bar_off(mode, Bn) + 512 + 1024; }
+static_assert(fwd_hring(2, 64) >= 3 && fwd_hring(0, 64) >= 4 && fwd_smem(2, 64) <= kFwdSmemMax &&
+                  fwd_smem(0, 64) <= kFwdSmemMax && fwd_smem(0, 16) <= kFwdSmemMax,
+              "forward shared-memory plan");
 
 // Bounded wait whose outcome is made uniform across the warp, so that a warp never
 // reaches a .sync.aligned tcgen05 instruction with only some of its lanes.
@@ -71,24 +104,44 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((a + 1023) & ~uintptr_t(1023));
 }
 
+// A barrier of the converter threads on an mbarrier, bounded like every other
+// wait.  `phase` counts this thread's uses.
+struct GroupSync {
+  uint64_t* bar;
+  uint32_t phase;
+  int* err;
+  __device__ __forceinline__ bool operator()() {
+    mbar_arrive(bar);
+    const bool ok = mbar_wait(bar, phase & 1, err);
+    ++phase;
+    return ok;
+  }
+};
+
 // Epilogue of the last layer when every class fits in one 128-row tile: the
 // softmax cross-entropy gradient straight from the accumulator (no logits
-// round trip).  Thread t owns class t's logits z[0..Bn); the work is spread
-// over all threads: column statistics (one thread per sample), gradients (all
-// class x sample pairs), then per-class bias sums in sample order.
-__device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, const float* z,
-                                              float* sm) {
+// round trip).  Row r = class, group gr holds the column blocks 2m + gr of it
+// (blocks of 16 samples) in acc[16m ..].  Work is then spread over all converter
+// threads: column statistics, all class x sample gradients, per-class bias sums
+// in sample order.
+__device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, int r, int gr,
+                                              const float* acc, float* sm, GroupSync& gsync) {
   constexpr int ZP = 65;
   float* zs = sm;                  // [128][ZP] logits, class-major
   float* gs = sm + 128 * ZP;       // [128][ZP] gradients
   float* stat = gs + 128 * ZP;     // max[64], sum[64], label[64], loss[64]
   const int C = a.out, B = a.B;
-  if (t < C) {
+  if (r < C) {
 #pragma unroll
-    for (int b = 0; b < 64; ++b)
-      if (b < a.Bn) zs[t * ZP + b] = z[b];
+    for (int m = 0; m < 2; ++m) {
+      const int cb = (2 * m + gr) * 16;
+      if (cb < a.Bn) {
+#pragma unroll
+        for (int q = 0; q < 16; ++q) zs[r * ZP + cb + q] = acc[16 * m + q];
+      }
+    }
   }
-  named_barrier_sync(1, kConv);
+  gsync();
   if (t < B) {
     float m = -INFINITY;
     for (int c = 0; c < C; ++c) m = fmaxf(m, zs[c * ZP + t]);
@@ -100,16 +153,16 @@ __device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, 
     stat[128 + t] = __int_as_float(yb);
     stat[192 + t] = logf(s) + m - zs[yb * ZP + t];
   }
-  named_barrier_sync(1, kConv);
+  gsync();
   const float fB = static_cast<float>(B);
-  for (int e = t; e < C * B; e += kConv) {
+  for (int e = t; e < C * B; e += kFwdConv) {
     const int c = e / B, b = e - c * B;
     const float p = __fdiv_rn(expf(zs[c * ZP + b] - stat[b]), stat[64 + b]);
     const float g = __fdiv_rn(__fsub_rn(p, __float_as_int(stat[128 + b]) == c ? 1.f : 0.f), fB);
     gs[c * ZP + b] = g;
     a.dz_out[(static_cast<int64_t>(j) * a.Bn + b) * a.pitch_out + c] = __float2bfloat16_rn(g);
   }
-  named_barrier_sync(1, kConv);
+  gsync();
   if (t == 0) {
     float l = 0.f;
     for (int b = 0; b < B; ++b) l += stat[192 + b];
@@ -134,49 +187,76 @@ __device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, 
     float* bp = const_cast<float*>(a.bias) + static_cast<int64_t>(j) * a.ld + t;
     *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
   }
+  gsync();   // the staging area is reused by the next tile
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+// First unit of CTA g when U units are split over G CTAs (G <= U).
+__device__ __forceinline__ int unit_begin(int g, int U, int G) {
+  return static_cast<int>(static_cast<int64_t>(g) * U / G);
+}
+// The CTA that owns unit u.
+__device__ __forceinline__ int cta_of(int u, int U, int G) {
+  int g = static_cast<int>(static_cast<int64_t>(u) * G / U);
+  while (g + 1 < G && unit_begin(g + 1, U, G) <= u) ++g;
+  while (g > 0 && unit_begin(g, U, G) > u) --g;
+  return g;
+}
+
+__global__ void __launch_bounds__(kFwdThreads, 1)
     k_tc_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
                  const TcFwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.y, tile = blockIdx.x, o0 = tile * 128, split = blockIdx.z;
-  const int nk_all = (a.in + 63) / 64;
-  const int per = (nk_all + a.splits - 1) / a.splits;
-  const int c_begin = split * per;
-  const int nk = min(nk_all, c_begin + per) - c_begin;   // >= 1 by the host's choice of splits
+  const int g = blockIdx.x, G = gridDim.x;
+  const int nk = (a.in + 63) / 64;
+  const int U = a.n_tiles * nk;
+  const int u0 = unit_begin(g, U, G), u1 = unit_begin(g + 1, U, G);
+  const int n_local = u1 - u0;
+  const int nw = fwd_wring(a.mode), nh = fwd_hring(a.mode, a.Bn);
+  const int hbytes = a.Bn * 128;
   const int h_row0 = a.x_direct ? a.x_row0 : 0;           // batch rows inside the H (or X) map
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kFwdBarOff);
-  uint64_t* empty = full + kFwdStages;
-  uint64_t* conv = empty + kFwdStages;   // [2] A tile written
-  uint64_t* wfree = conv + 2;            // [2] A tile consumed by the MMA
-  uint64_t* accf = wfree + 2;            // [2] accumulator segment complete
-  uint64_t* accr = accf + 2;             // [2] accumulator segment drained
-  uint64_t* done = accr + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
-  int* last_flag = reinterpret_cast<int*>(tmem_slot + 1);
-  int* all_ok = last_flag + 1;
-  auto wf = [&](int s) { return smem + s * kFwdStage; };
-  auto hb = [&](int s) { return smem + s * kFwdStage + kFwdWf32; };
-  auto wb = [&](int b) { return smem + kFwdWbfOff + b * kFwdWbf; };
+  const int tile0 = u0 / nk, c0 = u0 - tile0 * nk;         // first unit's tile and chunk
+  uint8_t* wbf_base = smem + nw * kFwdWf32;
+  uint8_t* xent_sm = wbf_base + 2 * kFwdWbf;
+  uint8_t* h_base = smem + fwd_h_off(a.mode);
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + fwd_bar_off(a.mode, a.Bn));
+  uint64_t* wempty = wfull + kFwdWRingMax;  // weight tile read by every converter warp
+  uint64_t* hfull = wempty + kFwdWRingMax;
+  uint64_t* hempty = hfull + kFwdHRingMax;  // batch tile consumed by the MMA
+  uint64_t* conv = hempty + kFwdHRingMax;   // [2] A tile written
+  uint64_t* wfree = conv + 2;              // [2] A tile consumed by the MMA
+  uint64_t* accf = wfree + 2;              // [2] accumulator segment complete
+  uint64_t* accr = accf + 2;               // [2] accumulator segment drained
+  uint64_t* gbar = accr + 2;               // converter-group barrier
+  uint64_t* done = gbar + 1;
+  uint64_t* pready = done + 1;             // this CTA's split-tile partial is written
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
+  auto wf = [&](int s) { return smem + s * kFwdWf32; };
+  auto hb = [&](int s) { return h_base + s * hbytes; };
+  auto wb = [&](int b) { return wbf_base + b * kFwdWbf; };
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kFwdStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int s = 0; s < kFwdWRingMax; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], kFwdConv / 32);   // one arrival per converter warp
+    }
+    for (int s = 0; s < kFwdHRingMax; ++s) {
+      mbar_init(&hfull[s], 1);
+      mbar_init(&hempty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&conv[b], kConv);
+      mbar_init(&conv[b], kFwdConv / 32);
       mbar_init(&wfree[b], 1);
       mbar_init(&accf[b], 1);
-      mbar_init(&accr[b], kConv);
+      mbar_init(&accr[b], kFwdConv);
     }
+    mbar_init(gbar, kFwdConv);
     mbar_init(done, 1);
+    mbar_init(pready, kFwdConv / 32);
     fence_barrier_init();
   }
-  if (warp == 5) {
+  if (warp == 9) {
     tmem_alloc(tmem_slot, kFwdTmemCols);
     tmem_relinquish();
   }
@@ -185,68 +265,94 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 4) {
-    if (lane == 0) {
-      tma_prefetch_desc(&tm_w);
-      tma_prefetch_desc(&tm_h);
-      int issued = 0;
-      for (int c = 0; c < nk; ++c) {
-        const int s = c % kFwdStages;
-        if (c >= kFwdStages && !mbar_wait(&empty[s], ((c / kFwdStages) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&full[s], kFwdWf32 + a.Bn * 128);
-        tma_load_3d(wf(s), &tm_w, &full[s], (c_begin + c) * 64, o0, j);
-        tma_load_3d(hb(s), &tm_h, &full[s], (c_begin + c) * 64, h_row0, j);
-        issued = c + 1;
+  if (warp == 8) {
+    // Lane 0 streams the weight tiles, lane 1 the batch tiles: each ring runs as
+    // far ahead as its own consumer allows.
+    if (lane < 2) {
+      const bool wside = lane == 0;
+      const int n = wside ? nw : nh;
+      uint64_t* fullb = wside ? wfull : hfull;
+      uint64_t* emptyb = wside ? wempty : hempty;
+      if (wside) tma_prefetch_desc(&tm_w);
+      else tma_prefetch_desc(&tm_h);
+      int issued = 0, tau = tile0, c = c0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+        const int s = i % n;
+        if (i >= n && !mbar_wait(&emptyb[s], ((i / n) - 1) & 1, a.err)) break;
+        if (wside) {
+          mbar_arrive_expect_tx(&fullb[s], kFwdWf32);
+          tma_load_3d(wf(s), &tm_w, &fullb[s], c * 64, ot * 128, j);
+        } else {
+          mbar_arrive_expect_tx(&fullb[s], a.Bn * 128);
+          tma_load_3d(hb(s), &tm_h, &fullb[s], c * 64, h_row0, j);
+        }
+        issued = i + 1;
+        if (++c == nk) { c = 0; ++tau; }
       }
       // Every load issued must have landed before the CTA may exit.
-      for (int c = issued - kFwdStages > 0 ? issued - kFwdStages : 0; c < issued; ++c)
-        mbar_wait(&full[c % kFwdStages], (c / kFwdStages) & 1, a.err);
+      for (int i = issued - n > 0 ? issued - n : 0; i < issued; ++i)
+        mbar_wait(&fullb[i % n], (i / n) & 1, a.err);
+    } else if (lane == 2 && c0 != 0 && n_local > 0) {
+      // The first tile began in an earlier CTA, which finishes it: once the
+      // converter warps have written this CTA's partial, publish it (release
+      // order makes the partial visible before the count).
+      if (mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
     }
-  } else if (warp == 5) {
+  } else if (warp == 9) {
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_bf16(128, a.Bn);
-      for (int c = 0; c < nk; ++c) {
-        const int s = c % kFwdStages, b = c & 1;
-        const int seg = c / kSegChunks, ab = seg & 1, first = c % kSegChunks == 0;
-        if (first && seg >= 2 && !mbar_wait(&accr[ab], ((seg >> 1) - 1) & 1, a.err)) break;
-        if (!mbar_wait(&conv[b], (c >> 1) & 1, a.err)) break;
+      int q = -1, c = c0, p = 0;        // accumulator segment index, chunk, position in run
+      for (int i = 0; i < n_local; ++i) {
+        const bool tlast = i == n_local - 1 || c == nk - 1;
+        const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+        const int sh = i % nh, b = i & 1;
+        if (first) ++q;
+        const int ab = q & 1;
+        if (first && q >= 2 && !mbar_wait(&accr[ab], ((q >> 1) - 1) & 1, a.err)) break;
+        if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) break;
+        if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) break;
         tc_fence_after();
         const uint64_t ad = umma_desc_sw128(smem_u32(wb(b)));
-        const uint64_t bd = umma_desc_sw128(smem_u32(hb(s)));
+        const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh)));
         const uint32_t d = tmem + 64 * ab;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
           tc_mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
-        tc_commit(&empty[s]);
+        tc_commit(&hempty[sh]);
         tc_commit(&wfree[b]);
-        if (c % kSegChunks == kSegChunks - 1 || c == nk - 1) tc_commit(&accf[ab]);
+        if (last) tc_commit(&accf[ab]);
+        ++p;
+        if (++c == nk) { c = 0; p = 0; }
       }
       tc_commit(done);
       mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
     }
   } else {
-    // ---- warps 0-3: fp32 -> bf16 A tile (and H_0^T for the first layer), then the epilogue
+    // ---- warps 0-7: fp32 -> bf16 A tile (and H_0^T for the first layer), the
+    // accumulator drains and the tile epilogues
     const int t = threadIdx.x;
-    const bool write_ht0 = a.x_direct && tile == 0;
-    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
-    float acc[64];
+    const int r = t & 127, gr = t >> 7;                    // accumulator row, column group
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+    GroupSync gsync{gbar, 0, a.err};
+    float acc[32];                                         // blocks 2m + gr, m = 0, 1
 #pragma unroll
-    for (int q = 0; q < 64; ++q) acc[q] = 0.f;
-    int drained = 0;   // accumulator segments folded into acc so far
-    const int nseg = (nk + kSegChunks - 1) / kSegChunks;
+    for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+    int qc = -1, drained = 0;
     // Fold segment `drained` into the registers (warp-uniform; contains tcgen05.ld).
     auto drain = [&]() -> bool {
       const int ab = drained & 1;
       if (!wait_warp(&accf[ab], (drained >> 1) & 1, a.err)) return false;
       tc_fence_after();
 #pragma unroll
-      for (int cb = 0; cb < 64; cb += 16) {
+      for (int m = 0; m < 2; ++m) {
+        const int cb = (2 * m + gr) * 16;
         if (cb < a.Bn) {
           float v[16];
           tmem_ld16(tbase + 64 * ab + cb, v);
           tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 16; ++q) acc[cb + q] = __fadd_rn(acc[cb + q], v[q]);
+          for (int q = 0; q < 16; ++q) acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v[q]);
         }
       }
       tc_fence_before();
@@ -254,31 +360,131 @@ __global__ void __launch_bounds__(kThreads, 1)
       ++drained;
       return true;
     };
+    // Tile tau is complete in this CTA's registers (or in this CTA's part of it).
+    // A tile split over CTAs g_first .. g_last is finished by g_first, the CTA that
+    // holds its first chunk and, in stream-K order, reaches it last; every other
+    // contributor writes its partial to its own slot and publishes it without
+    // waiting.  The finisher adds the partials in CTA order.
+    auto tile_end = [&](int tau, bool whole, float bias) -> bool {
+      const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+      if (!whole) {
+        if (tau * nk < u0) {
+          float* mine = a.part + (static_cast<int64_t>(g) * 128 + r) * a.Bn;
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int cb = (2 * m + gr) * 16;
+            if (cb < a.Bn) {
+#pragma unroll
+              for (int q = 0; q < 16; q += 4)
+                __stcg(reinterpret_cast<float4*>(mine + cb + q),
+                       make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                                   acc[16 * m + q + 3]));
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(pready);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+          return true;
+        }
+        const int g_last = cta_of((tau + 1) * nk - 1, U, G);
+        if (t == 0) {
+          const bool ok = spin_acquire_eq(a.counters + tau, g_last - g, a.err);
+          if (ok) a.counters[tau] = 0;   // ready for the next launch
+        }
+        if (!gsync()) return false;
+        for (int gg = g + 1; gg <= g_last; ++gg) {
+          const float* src = a.part + (static_cast<int64_t>(gg) * 128 + r) * a.Bn;
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int cb = (2 * m + gr) * 16;
+            if (cb < a.Bn) {
+#pragma unroll
+              for (int q = 0; q < 16; q += 4) {
+                const float4 v = __ldcg(reinterpret_cast<const float4*>(src + cb + q));
+                acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v.x);
+                acc[16 * m + q + 1] = __fadd_rn(acc[16 * m + q + 1], v.y);
+                acc[16 * m + q + 2] = __fadd_rn(acc[16 * m + q + 2], v.z);
+                acc[16 * m + q + 3] = __fadd_rn(acc[16 * m + q + 3], v.w);
+              }
+            }
+          }
+        }
+      }
+      const int o = ot * 128 + r;
+      const bool valid = o < a.out;
+      if (a.mode == kFwdXent) {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) acc[q] = __fadd_rn(acc[q], bias);
+        xent_epilogue(a, j, t, r, gr, acc, reinterpret_cast<float*>(xent_sm), gsync);
+      } else if (valid) {
+#pragma unroll
+        for (int m = 0; m < 2; ++m) {
+          const int cb = (2 * m + gr) * 16;
+          if (cb >= a.Bn) break;
+          if (a.mode == kFwdHidden) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int q = 0; q < 16; q += 2) {
+              const float h0 = fmaxf(__fadd_rn(acc[16 * m + q], bias), 0.f);
+              const float h1 = fmaxf(__fadd_rn(acc[16 * m + q + 1], bias), 0.f);
+              const bool in0 = cb + q < a.B, in1 = cb + q + 1 < a.B;
+              pk[q / 2] = pack_bf16x2(in0 ? h0 : 0.f, in1 ? h1 : 0.f);
+              const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
+              if (in0) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] = hh.x;
+              if (in1) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_out + o] = hh.y;
+            }
+            uint4* dst = reinterpret_cast<uint4*>(a.ht_out + (static_cast<int64_t>(j) * a.out + o) * a.Kp + cb);
+            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          } else {
+#pragma unroll
+            for (int q = 0; q < 16; ++q)
+              if (cb + q < a.B)
+                a.z_out[(static_cast<int64_t>(j) * a.B + cb + q) * a.out + o] = __fadd_rn(acc[16 * m + q], bias);
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+      return true;
+    };
     bool ok = true;
-    for (int c = 0; c < nk; ++c) {
-      const int s = c % kFwdStages, bb = c & 1;
-      if (!wait_warp(&full[s], (c / kFwdStages) & 1, a.err)) { ok = false; break; }
-      if (c >= 2 && !wait_warp(&wfree[bb], ((c >> 1) - 1) & 1, a.err)) { ok = false; break; }
-      const float4* src = reinterpret_cast<const float4*>(wf(s));
+    int tau = tile0, c = c0, p = 0;
+    float tbias = 0.f;                 // bias of row r of the current tile, loaded early
+    for (int i = 0; i < n_local && ok; ++i) {
+      const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+      const bool tlast = i == n_local - 1 || c == nk - 1;
+      if (p == 0) {
+        const int o = ot * 128 + r;
+        tbias = o < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
+      }
+      const int sw = i % nw, sh = i % nh, bb = i & 1;
+      if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+      if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+      const float* src = reinterpret_cast<const float*>(wf(sw));
       uint8_t* dst = wb(bb);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int f = t + kConv * i;        // float4 index in the [128][64] fp32 tile
-        const int r = f >> 4, k = (f & 15) * 4;
-        const float4 v = src[f];
-        uint2 pk;
-        pk.x = pack_bf16x2(v.x, v.y);
-        pk.y = pack_bf16x2(v.z, v.w);
-        *reinterpret_cast<uint2*>(dst + sw128_offset(r, k)) = pk;
+      for (int v = 0; v < 4; ++v) {
+        const int f = t + kFwdConv * v;      // group of 8 floats in the [128][64] fp32 tile
+        const int row = f >> 3, k = (f & 7) * 8;
+        const float4 x0 = *reinterpret_cast<const float4*>(src + row * 64 + k);
+        const float4 x1 = *reinterpret_cast<const float4*>(src + row * 64 + k + 4);
+        *reinterpret_cast<uint4*>(dst + sw128_offset(row, k)) =
+            make_uint4(pack_bf16x2(x0.x, x0.y), pack_bf16x2(x0.z, x0.w), pack_bf16x2(x1.x, x1.y),
+                       pack_bf16x2(x1.z, x1.w));
       }
-      if (write_ht0) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&wempty[sw]);   // the fp32 tile is no longer needed
+      if (a.x_direct && ot == 0) {
         // H_0^T[k][b] for this chunk's 64 features, from the staged batch tile
         // (rows b >= B of the tile belong to later samples and are written as 0).
-        const uint8_t* hs = hb(s);
+        if (!wait_warp(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
+        const uint8_t* hs = hb(sh);
         const int kk = t & 63;
-        const int k = (c_begin + c) * 64 + kk;
+        const int k = c * 64 + kk;
         if (k < a.in) {
-          for (int b0 = (t >> 6) * 8; b0 < a.Bn; b0 += 16) {
+          for (int b0 = (t >> 6) * 8; b0 < a.Bn; b0 += 32) {
             uint32_t pk[4];
 #pragma unroll
             for (int q = 0; q < 8; q += 2) {
@@ -293,99 +499,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       fence_proxy_async_smem();
-      mbar_arrive(&conv[bb]);
-      // one segment behind the MMAs: fold the segment completed a while ago
-      if (c % kSegChunks == kSegChunks - 1 && c / kSegChunks >= 1 && drained < c / kSegChunks)
-        if (!drain()) { ok = false; break; }
-    }
-    while (ok && drained < nseg)
-      if (!drain()) ok = false;
-    if (ok) ok = wait_warp(done, 0, a.err);
-    tc_fence_after();
-    const int o = o0 + t;
-    const bool valid = o < a.out;
-    bool finish = true;
-    if (a.splits > 1) {
-      // Split-K: publish this CTA's partial; the last CTA of the tile sums all
-      // partials in split order (deterministic) and runs the epilogue.
-      float* part = a.part + ((static_cast<int64_t>(j) * a.o_tiles + tile) * a.splits) * 128 * a.Bn;
-      float4* mine = reinterpret_cast<float4*>(part + (static_cast<int64_t>(split) * 128 + t) * a.Bn);
-#pragma unroll
-      for (int q = 0; q < 64; q += 4)
-        if (q < a.Bn) mine[q / 4] = make_float4(acc[q], acc[q + 1], acc[q + 2], acc[q + 3]);
-      __threadfence();
-      named_barrier_sync(1, kConv);
-      if (t == 0) {
-        int* cnt = a.counters + static_cast<int64_t>(j) * a.o_tiles + tile;
-        const int prev = atomicAdd(cnt, 1);
-        *last_flag = (prev == a.splits - 1);
-        if (prev == a.splits - 1) *cnt = 0;     // ready for the next launch
-      }
-      named_barrier_sync(1, kConv);
-      finish = *last_flag != 0;
-      if (finish) {
-        __threadfence();
-#pragma unroll
-        for (int q = 0; q < 64; ++q) acc[q] = 0.f;
-        for (int sp = 0; sp < a.splits; ++sp) {
-          const float4* src = reinterpret_cast<const float4*>(part + (static_cast<int64_t>(sp) * 128 + t) * a.Bn);
-#pragma unroll
-          for (int q = 0; q < 64; q += 4) {
-            if (q >= a.Bn) break;
-            const float4 v = __ldcg(src + q / 4);
-            acc[q] = __fadd_rn(acc[q], v.x);
-            acc[q + 1] = __fadd_rn(acc[q + 1], v.y);
-            acc[q + 2] = __fadd_rn(acc[q + 2], v.z);
-            acc[q + 3] = __fadd_rn(acc[q + 3], v.w);
-          }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&conv[bb]);
+      if (p % kSegChunks == 0) ++qc;
+      if (tlast) {
+        while (ok && drained <= qc)
+          if (!drain()) ok = false;
+        if (ok) {
+          const bool whole = (tau != tile0 || c0 == 0) && c == nk - 1;
+          ok = __all_sync(0xffffffffu, tile_end(tau, whole, tbias));
         }
+      } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
+        if (!drain()) ok = false;   // one segment behind the MMAs
       }
-    }
-    // A timed-out wait in any converter warp makes the whole group skip the
-    // epilogue (which contains group barriers).
-    if (t == 0) *all_ok = 1;
-    named_barrier_sync(1, kConv);
-    if (!ok) atomicAnd(all_ok, 0);
-    named_barrier_sync(1, kConv);
-    ok = *all_ok != 0;
-    if (finish && ok) {
-      const float bias = valid ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
-      if (a.mode == kFwdXent) {
-#pragma unroll
-        for (int q = 0; q < 64; ++q) acc[q] = __fadd_rn(acc[q], bias);
-        xent_epilogue(a, j, t, acc, reinterpret_cast<float*>(smem));
-      } else if (valid) {
-#pragma unroll
-        for (int cb = 0; cb < 64; cb += 16) {
-          if (cb >= a.Bn) break;
-          if (a.mode == kFwdHidden) {
-            uint32_t pk[8];
-#pragma unroll
-            for (int q = 0; q < 16; q += 2) {
-              const float h0 = fmaxf(__fadd_rn(acc[cb + q], bias), 0.f);
-              const float h1 = fmaxf(__fadd_rn(acc[cb + q + 1], bias), 0.f);
-              const bool in0 = cb + q < a.B, in1 = cb + q + 1 < a.B;
-              pk[q / 2] = pack_bf16x2(in0 ? h0 : 0.f, in1 ? h1 : 0.f);
-              const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
-              if (in0) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] = hh.x;
-              if (in1) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_out + o] = hh.y;
-            }
-            uint4* dst = reinterpret_cast<uint4*>(a.ht_out + (static_cast<int64_t>(j) * a.out + o) * a.Kp + cb);
-            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-          } else {
-#pragma unroll
-            for (int q = 0; q < 16; ++q)
-              if (cb + q < a.B)
-                a.z_out[(static_cast<int64_t>(j) * a.B + cb + q) * a.out + o] = __fadd_rn(acc[cb + q], bias);
-          }
-        }
-      }
+      ++p;
+      if (++c == nk) { c = 0; p = 0; ++tau; }
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == 9) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kFwdTmemCols);
@@ -757,21 +890,32 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
 
 }  // namespace
 
-int tc_fwd_smem_bytes() { return kFwdSmem; }
+int tc_fwd_smem_bytes() { return kFwdSmemMax; }
 int tc_bwd_smem_bytes() { return kBwdSmem; }
 
 cudaError_t tc_configure() {
   cudaError_t e = cudaFuncSetAttribute(k_tc_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       kFwdSmem);
+                                       kFwdSmemMax);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmem);
 }
 
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s) {
-  dim3 grid(a.o_tiles, P, a.splits);
-  k_tc_forward<<<grid, kThreads, kFwdSmem, s>>>(w_fwd, h_in, a);
-  return cudaGetLastError();
+  (void)P;
+  // Cooperative: the finisher of a split tile waits for the other contributors,
+  // so every CTA of the grid must be resident at once (the launch fails otherwise).
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.ctas);
+  cfg.blockDim = dim3(kFwdThreads);
+  cfg.dynamicSmemBytes = fwd_smem(a.mode, a.Bn);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_tc_forward, w_fwd, h_in, a);
 }
 
 cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& ht_in,

@@ -64,7 +64,7 @@ def test_static_step_matches_bound_step(lib, w):
 def test_static_step_rejects_large_configurations(lib):
     w = configs.MLP2048_P64                          # needs ~181 MiB of scratch
     h = HierAvg(w.P, w.S, w.K1, w.K2, w.lr, w.B, w.dims, w.precision)
-    assert h.workspace_bytes > 16 << 20
+    assert h.workspace_bytes > 32 << 20
     params = torch.zeros(w.P, h.ld, device="cuda")
     X = torch.zeros(w.P, 2, w.dims[0], dtype=torch.bfloat16, device="cuda")
     y = torch.zeros(w.P, 2, dtype=torch.int32, device="cuda")
@@ -72,4 +72,4 @@ def test_static_step_rejects_large_configurations(lib):
                                   ctypes.c_void_p(X.data_ptr()), ctypes.c_void_p(y.data_ptr()),
                                   2, None)
     assert rc == -2                                  # HA_ENOMEM
-    assert b"16777216" in lib.hier_avg_last_error(h.h)
+    assert b"33554432" in lib.hier_avg_last_error(h.h)
