@@ -60,13 +60,14 @@ struct hier_avg {
   int64_t D = 0, ld = 0;
   std::vector<int64_t> woff, boff;
   // workspace layout
-  int Bn = 0, Kp = 0;
+  int Bn = 0;
   std::vector<int> pitch;                       // per width index l = 0..L
-  std::vector<int64_t> off_H, off_HT, off_dZ, off_dZT;
+  std::vector<int64_t> off_H, off_dZ;
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
-  int64_t off_part = 0, off_cnt = 0;          // split-K partials and tile counters
+  int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
   int64_t off_gq = 0;                         // small-head CE gradient
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
+  std::vector<int> bwd_ctas, bwd_tiles;       // per layer: stream-K CTAs, input slices
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
   bool head = false;                          // d_L <= 16: fused last-layer kernel
   // binding
@@ -78,7 +79,7 @@ struct hier_avg {
   const int32_t* y = nullptr;
   int64_t N = 0;
   cudaStream_t stream = nullptr;
-  std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_ht, tm_dz, tm_dzt;
+  std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_dz;
   CUtensorMap tm_x;                           // X [P][N][d_0] as the first layer's batch tile
   int64_t t = 0;
   // profiling
@@ -161,35 +162,31 @@ int plan_layout(hier_avg* h) {
     return o;
   };
   h->off_H.assign(L + 1, 0);
-  h->off_HT.assign(L + 1, 0);
   h->off_dZ.assign(L + 1, 0);
-  h->off_dZT.assign(L + 1, 0);
   h->pitch.assign(L + 1, 0);
   if (h->prec == HA_PREC_BF16) {
     h->Bn = static_cast<int>(round_up(B, 16));
-    h->Kp = 64;
     for (int l = 0; l <= L; ++l) h->pitch[l] = static_cast<int>(round_up(h->dims[l], 64));
-    for (int l = 0; l < L; ++l) {
-      h->off_H[l] = take(P * h->Bn * h->pitch[l] * 2);
-      h->off_HT[l] = take(P * h->dims[l] * h->Kp * 2);
-    }
-    for (int l = 1; l <= L; ++l) {
-      h->off_dZ[l] = take(P * h->Bn * h->pitch[l] * 2);
-      h->off_dZT[l] = take(P * h->dims[l] * h->Kp * 2);
-    }
-    // Stream-K plan of the forward GEMMs: at most one persistent CTA per SM of a
-    // GB300 (152).  It depends on the shapes only, so the summation order of split
-    // tiles is the same on every GPU.
+    for (int l = 0; l < L; ++l) h->off_H[l] = take(P * h->Bn * h->pitch[l] * 2);
+    for (int l = 1; l <= L; ++l) h->off_dZ[l] = take(P * h->Bn * h->pitch[l] * 2);
+    // Stream-K plans of the forward and backward GEMMs: at most one persistent CTA
+    // per SM of a GB300 (152).  They depend on the shapes only, so the summation
+    // order of split tiles is the same on every GPU.  Forward tile = 128 outputs x
+    // 64-input chunks; backward tile = 128 inputs x 64-output chunks.
     h->fwd_ctas.assign(L, 1);
     h->fwd_tiles.assign(L, 1);
+    h->bwd_ctas.assign(L, 1);
+    h->bwd_tiles.assign(L, 1);
     int64_t part_bytes = 16, max_tiles = 1;
     for (int l = 0; l < L; ++l) {
-      const int64_t tiles = (h->dims[l + 1] + 127) / 128, nk = (h->dims[l] + 63) / 64;
-      const int64_t units = tiles * P * nk;
-      h->fwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, units));
-      h->fwd_tiles[l] = static_cast<int>(tiles);
-      part_bytes = std::max(part_bytes, int64_t(h->fwd_ctas[l]) * 128 * h->Bn * 4);
-      max_tiles = std::max(max_tiles, tiles * P);
+      const int64_t in = h->dims[l], out = h->dims[l + 1];
+      const int64_t ftiles = (out + 127) / 128, btiles = (in + 127) / 128;
+      h->fwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, ftiles * P * ((in + 63) / 64)));
+      h->fwd_tiles[l] = static_cast<int>(ftiles);
+      h->bwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, btiles * P * ((out + 63) / 64)));
+      h->bwd_tiles[l] = static_cast<int>(btiles);
+      part_bytes = std::max(part_bytes, int64_t(std::max(h->fwd_ctas[l], h->bwd_ctas[l])) * 128 * h->Bn * 4);
+      max_tiles = std::max(max_tiles, std::max(ftiles, btiles) * P);
     }
     h->fused_xent = h->dims[L] <= 128;
     h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B));
@@ -231,16 +228,14 @@ int build_maps(hier_avg* h) {
   h->tm_wf.resize(L);
   h->tm_wb.resize(L);
   h->tm_h.resize(L);
-  h->tm_ht.resize(L);
   h->tm_dz.resize(L + 1);
-  h->tm_dzt.resize(L + 1);
-  const uint64_t P = h->P, Bn = h->Bn, Kp = h->Kp;
+  const uint64_t P = h->P, Bn = h->Bn;
   int rc;
   for (int l = 0; l < L; ++l) {
     const uint64_t in = h->dims[l], out = h->dims[l + 1];
     float* W = h->params + h->woff[l];
     if ((rc = make_map(h, &h->tm_wf[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
-                       h->ld * 4, 64, 128, CU_TENSOR_MAP_SWIZZLE_NONE)))
+                       h->ld * 4, 32, 128, CU_TENSOR_MAP_SWIZZLE_128B)))
       return rc;
     if ((rc = make_map(h, &h->tm_wb[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
                        h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
@@ -249,9 +244,6 @@ int build_maps(hier_avg* h) {
     if ((rc = make_map(h, &h->tm_h[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_H[l], pin,
                        Bn, P, pin * 2, Bn * pin * 2, 64, static_cast<uint32_t>(Bn),
                        CU_TENSOR_MAP_SWIZZLE_128B)))
-      return rc;
-    if ((rc = make_map(h, &h->tm_ht[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_HT[l], Kp,
-                       in, P, Kp * 2, in * Kp * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B)))
       return rc;
   }
   {
@@ -266,9 +258,6 @@ int build_maps(hier_avg* h) {
     if ((rc = make_map(h, &h->tm_dz[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_dZ[l], pd,
                        Bn, P, pd * 2, Bn * pd * 2, 64, static_cast<uint32_t>(Bn),
                        CU_TENSOR_MAP_SWIZZLE_128B)))
-      return rc;
-    if ((rc = make_map(h, &h->tm_dzt[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_dZT[l],
-                       Kp, d, P, Kp * 2, d * Kp * 2, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B)))
       return rc;
   }
   return HA_OK;
@@ -285,13 +274,13 @@ int check_bound(hier_avg* h) {
 double bytes_forward(const hier_avg* h, int l) {
   const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
-  return P * (in * out * 4.0 + out * 4.0 + B * in * act + B * out * (l + 1 == h->L ? 4.0 : 2 * act));
+  return P * (in * out * 4.0 + out * 4.0 + B * in * act + B * out * (l + 1 == h->L ? 4.0 : act));
 }
 double bytes_backward(const hier_avg* h, int l) {
   const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
-  const double dx = l > 0 ? (B * in * act * 2 + in * 8.0) : 0.0;
-  return P * (in * out * 8.0 + B * in * act + 2 * B * out * act + dx);
+  const double dx = l > 0 ? (B * in * act + in * 8.0) : 0.0;
+  return P * (in * out * 8.0 + B * in * act + B * out * act + dx);
 }
 
 int do_step(hier_avg* h) {
@@ -307,8 +296,7 @@ int do_step(hier_avg* h) {
     if (!x_direct) {
       rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, [&] {
         return ha::launch_gather_bf16(static_cast<const __nv_bfloat16*>(h->X), h->N, d0, B, h->Bn,
-                                      h->Kp, h->pitch[0], h->t, P, h->wsp<__nv_bfloat16>(h->off_H[0]),
-                                      h->wsp<__nv_bfloat16>(h->off_HT[0]), s);
+                                      h->pitch[0], h->t, P, h->wsp<__nv_bfloat16>(h->off_H[0]), s);
       }, "gather");
       if (rc) return rc;
     }
@@ -319,7 +307,6 @@ int do_step(hier_avg* h) {
       a.out = h->dims[l + 1];
       a.B = B;
       a.Bn = h->Bn;
-      a.Kp = h->Kp;
       a.ld = h->ld;
       a.bias = h->params + h->boff[l];
       a.ctas = h->fwd_ctas[l];
@@ -329,12 +316,10 @@ int do_step(hier_avg* h) {
       a.counters = h->wsp<int>(h->off_cnt);
       a.x_direct = (l == 0 && x_direct) ? 1 : 0;
       a.x_row0 = static_cast<int>(r0);
-      a.ht0_out = h->wsp<__nv_bfloat16>(h->off_HT[0]);
       if (l + 1 < L) {
         a.mode = 0;
         a.h_out = h->wsp<__nv_bfloat16>(h->off_H[l + 1]);
         a.pitch_out = h->pitch[l + 1];
-        a.ht_out = h->wsp<__nv_bfloat16>(h->off_HT[l + 1]);
       } else if (h->fused_xent) {
         a.mode = 2;
         a.y = h->y;
@@ -343,7 +328,6 @@ int do_step(hier_avg* h) {
         a.lr = h->lr;
         a.pitch_out = h->pitch[L];
         a.dz_out = h->wsp<__nv_bfloat16>(h->off_dZ[L]);
-        a.dzt_out = h->wsp<__nv_bfloat16>(h->off_dZT[L]);
         a.loss = h->loss();
       } else {
         a.mode = 1;
@@ -363,7 +347,6 @@ int do_step(hier_avg* h) {
       a.in = h->dims[L - 1];
       a.B = B;
       a.Bn = h->Bn;
-      a.Kp = h->Kp;
       a.pitch_in = h->pitch[L - 1];
       a.ld = h->ld;
       a.N = h->N;
@@ -378,7 +361,6 @@ int do_step(hier_avg* h) {
       if (L > 1) {
         a.bias_prev = h->params + h->boff[L - 2];
         a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[L - 1]);
-        a.dzt_prev = h->wsp<__nv_bfloat16>(h->off_dZT[L - 1]);
       }
       a.loss = h->loss();
       a.gq = h->wsp<float>(h->off_gq);
@@ -387,10 +369,9 @@ int do_step(hier_avg* h) {
       if (rc) return rc;
     } else if (!h->fused_xent) {
       rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
-        return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, h->Kp, C,
+        return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, C,
                                     h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
-                                    h->wsp<__nv_bfloat16>(h->off_dZ[L]),
-                                    h->wsp<__nv_bfloat16>(h->off_dZT[L]), h->loss(), P, s);
+                                    h->wsp<__nv_bfloat16>(h->off_dZ[L]), h->loss(), P, s);
       }, "xent");
       if (rc) return rc;
     }
@@ -400,7 +381,6 @@ int do_step(hier_avg* h) {
       a.out = h->dims[l + 1];
       a.B = B;
       a.Bn = h->Bn;
-      a.Kp = h->Kp;
       a.ld = h->ld;
       a.lr = h->lr;
       a.has_dx = l > 0;
@@ -408,12 +388,20 @@ int do_step(hier_avg* h) {
         a.bias_prev = h->params + h->boff[l - 1];
         a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[l]);
         a.pitch_in = h->pitch[l];
-        a.dzt_prev = h->wsp<__nv_bfloat16>(h->off_dZT[l]);
       }
+      // H_{l-1}: the layer's input rows, straight from X for the first layer when
+      // the forward read them there too.
+      const bool from_x = l == 0 && x_direct;
+      a.h_row0 = from_x ? static_cast<int>(r0) : 0;
+      a.ctas = h->bwd_ctas[l];
+      a.s_tiles = h->bwd_tiles[l];
+      a.n_tiles = h->bwd_tiles[l] * P;
+      a.part = h->wsp<float>(h->off_part);
+      a.counters = h->wsp<int>(h->off_cnt);
       a.err = h->err_word();
+      const CUtensorMap& hin = from_x ? h->tm_x : h->tm_h[l];
       rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
-        return ha::launch_tc_backward(h->tm_wb[l], h->tm_ht[l], h->tm_dz[l + 1], h->tm_dzt[l + 1],
-                                      a, P, s);
+        return ha::launch_tc_backward(h->tm_wb[l], hin, h->tm_dz[l + 1], a, P, s);
       }, "backward");
       if (rc) return rc;
     }

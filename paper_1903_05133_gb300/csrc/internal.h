@@ -22,20 +22,18 @@ cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, 
 // Activation buffers of the bf16 path (all zero-initialised once; kernels only
 // ever write the valid region, so the padding stays zero):
 //   H_l   [P][Bn][pitch(d_l)]  bf16  layer-l input rows (batch-major)
-//   HT_l  [P][d_l][Kp]         bf16  the same, transposed (feature-major)
 //   dZ_l  [P][Bn][pitch(d_l)]  bf16  gradient w.r.t. the pre-activation of layer l
-//   dZT_l [P][d_l][Kp]         bf16  transposed
 //   Z_L   [P][B][d_L]          fp32  logits of the last layer
-// Bn = B rounded up to 16 (the MMA N extent), Kp = 64 (B <= 64), pitch(d) = d
-// rounded up to 64.
+// Bn = B rounded up to 16 (the MMA N extent, B <= 64), pitch(d) = d rounded up to
+// 64.  The backward reads H and dZ as stored (MN-major operands), so no transposed
+// copies exist.
 struct TcFwdArgs {
-  int in, out, B, Bn, Kp;
+  int in, out, B, Bn;
   int64_t ld;                 // parameter row length (floats)
   const float* bias;          // learner 0's b_l; learner j at + j * ld
-  int mode;                   // 0 hidden (ReLU -> H, HT), 1 logits -> z_out, 2 fused softmax-CE
+  int mode;                   // 0 hidden (ReLU -> H), 1 logits -> z_out, 2 fused softmax-CE
   __nv_bfloat16* h_out;       // mode 0: H_{l+1} [P][Bn][pitch_out]
   int pitch_out;              // mode 0: H pitch; mode 2: dZ_L pitch
-  __nv_bfloat16* ht_out;      // mode 0: HT_{l+1} [P][out][Kp]
   float* z_out;               // mode 1: Z_L [P][B][out]
   // persistent stream-K schedule: `ctas` CTAs share the n_tiles x ceil(in/64) units
   // (tile = learner x 128 outputs) evenly.  A split tile is finished by the CTA that
@@ -46,27 +44,29 @@ struct TcFwdArgs {
   float* part;
   int* counters;
   // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)
-  // and the CTAs of output tile 0 also write H_0^T.
   int x_direct, x_row0;
-  __nv_bfloat16* ht0_out;     // HT_0 [P][in][Kp]
   // mode 2: labels and outputs of the fused cross-entropy
   const int32_t* y;
   int64_t N, t;
   float lr;
   __nv_bfloat16* dz_out;      // dZ_L [P][Bn][pitch_out]
-  __nv_bfloat16* dzt_out;     // dZT_L [P][out][Kp]
   float* loss;                // [P]
   int* err;
 };
 struct TcBwdArgs {
-  int in, out, B, Bn, Kp;
+  int in, out, B, Bn;
   int64_t ld;
   float lr;
   int has_dx;                 // compute dZ_{l-1} (every layer but the first)
   float* bias_prev;           // learner 0's b_{l-1}
   __nv_bfloat16* dz_prev;     // dZ_{l-1} [P][Bn][pitch_in]
   int pitch_in;
-  __nv_bfloat16* dzt_prev;    // dZT_{l-1} [P][in][Kp]
+  int h_row0;                 // first batch row of H_{l-1} in its tensor map (X rows for l = 0)
+  // persistent stream-K schedule over n_tiles = P x ceil(in/128) tiles x ceil(out/64)
+  // chunks, same partial/counter protocol as the forward
+  int ctas, n_tiles, s_tiles;
+  float* part;
+  int* counters;
   int* err;
 };
 int tc_fwd_smem_bytes();
@@ -74,24 +74,21 @@ int tc_bwd_smem_bytes();
 cudaError_t tc_configure();   // raises the dynamic shared-memory limits once
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s);
-cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& ht_in,
-                               const CUtensorMap& dz, const CUtensorMap& dzt,
-                               const TcBwdArgs& a, int P, cudaStream_t s);
-// Mini-batch fetch for the bf16 path: rows (t*B + b) mod N of X -> H_0 and HT_0.
+cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
+                               const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s);
+// Mini-batch fetch for the bf16 path: rows (t*B + b) mod N of X -> H_0.
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
-                               int Kp, int pitch0, int64_t t, int P, __nv_bfloat16* H0,
-                               __nv_bfloat16* HT0, cudaStream_t s);
+                               int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s);
 // Softmax cross-entropy gradient of the last layer (bf16 operands out), loss, and
 // the SGD update of the last bias.
 cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
-                             int Bn, int Kp, int C, int pitch_c, float lr, float* bias_L,
-                             int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
-                             int P, cudaStream_t s);
+                             int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
+                             __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s);
 
 // Small last layer (<= 16 classes) on CUDA cores: a per-learner forward + softmax-CE
 // kernel and a per-feature-slice backward kernel, linked by the scratch `gq`.
 struct HeadArgs {
-  int C, in, B, Bn, Kp, pitch_in;
+  int C, in, B, Bn, pitch_in;
   int64_t ld, N, t;
   float lr;
   float* W;                   // learner 0's W_L [C][in] (fp32 master)
@@ -99,10 +96,9 @@ struct HeadArgs {
   const __nv_bfloat16* H;     // H_{L-1} [P][Bn][pitch_in], or X [P][N][in] when x_rows
   int x_rows;
   const int32_t* y;
-  int has_dx;                 // write dZ_{L-1} / dZT_{L-1} and update b_{L-1}
+  int has_dx;                 // write dZ_{L-1} and update b_{L-1}
   float* bias_prev;
   __nv_bfloat16* dz_prev;     // [P][Bn][pitch_in]
-  __nv_bfloat16* dzt_prev;    // [P][in][Kp]
   float* loss;                // [P]
   float* gq;                  // scratch: bf16-rounded CE gradient [P][Bn][16]
 };

@@ -166,38 +166,26 @@ __global__ void __launch_bounds__(kBwdCols) k_head_bwd(const HeadArgs a) {
 #pragma unroll
     for (int q = 0; q < 8; ++q)
       h[q] = b0 + q < B ? __bfloat162float(head_row(a, j, b0 + q)[k]) : 0.f;
-    uint32_t pk[4];
 #pragma unroll
-    for (int q = 0; q < 8; q += 2) {
-      float dz2[2];
+    for (int q = 0; q < 8; ++q) {
+      const int b = b0 + q;
+      if (b < B) {
+        float dh = 0.f;
 #pragma unroll
-      for (int e2 = 0; e2 < 2; ++e2) {
-        const int b = b0 + q + e2;
-        float dz = 0.f;
-        if (b < B) {
-          float dh = 0.f;
-#pragma unroll
-          for (int c = 0; c < CM; ++c) {
-            if (CT > 0 || c < C) {
-              const float g = gq[b * kHeadMaxC + c];
-              dw[c] = fmaf(g, h[q + e2], dw[c]);
-              dh = fmaf(g, wk[c], dh);
-            }
-          }
-          if (a.has_dx) {
-            dz = h[q + e2] > 0.f ? dh : 0.f;
-            db = __fadd_rn(db, dz);
-            a.dz_prev[(static_cast<int64_t>(j) * a.Bn + b) * a.pitch_in + k] = __float2bfloat16_rn(dz);
+        for (int c = 0; c < CM; ++c) {
+          if (CT > 0 || c < C) {
+            const float g = gq[b * kHeadMaxC + c];
+            dw[c] = fmaf(g, h[q], dw[c]);
+            dh = fmaf(g, wk[c], dh);
           }
         }
-        dz2[e2] = dz;
+        if (a.has_dx) {
+          const float dz = h[q] > 0.f ? dh : 0.f;
+          db = __fadd_rn(db, dz);
+          a.dz_prev[(static_cast<int64_t>(j) * a.Bn + b) * a.pitch_in + k] = __float2bfloat16_rn(dz);
+        }
       }
-      const __nv_bfloat162 pr = __floats2bfloat162_rn(dz2[0], dz2[1]);
-      pk[q / 2] = *reinterpret_cast<const uint32_t*>(&pr);
     }
-    if (a.has_dx)
-      *reinterpret_cast<uint4*>(a.dzt_prev + (static_cast<int64_t>(j) * in + k) * a.Kp + b0) =
-          make_uint4(pk[0], pk[1], pk[2], pk[3]);
   }
 #pragma unroll
   for (int c = 0; c < CM; ++c)

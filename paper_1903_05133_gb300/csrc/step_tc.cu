@@ -36,9 +36,6 @@
 namespace ha {
 namespace {
 
-constexpr int kStages = 3;
-constexpr int kThreads = 192;          // warps 0-3 convert/epilogue, 4 TMA, 5 MMA
-constexpr int kConv = 128;
 
 // ------------------------------------------------------------------ forward
 // Persistent stream-K forward.  The work of one layer is a list of units
@@ -46,24 +43,25 @@ constexpr int kConv = 128;
 // features.  CTA g of G owns the contiguous units [g*U/G, (g+1)*U/G), so every SM
 // streams the same number of chunks and the TMA ring runs straight across tile
 // boundaries.  A tile whose chunks are spread over several CTAs is finished by
-// the contributor that arrives last: it sums the published partial accumulators
-// in CTA order (deterministic) and runs the epilogue.
+// the CTA that holds its first chunk (see tile_end) with the partials of the
+// others added in CTA order (deterministic).
 // Warps 0-7 convert the fp32 weight tiles to bf16 and own the accumulator rows:
-// warp w serves TMEM lanes 32*(w%4).., and the two warps on the same lanes split
-// the batch columns in interleaved 16-column blocks (group w/4 takes blocks
-// 2m + w/4).  Warp 8 issues TMA, warp 9 the MMAs.
-// Shared memory: two TMA rings, the fp32 weight tiles (released by the converter
-// warps as soon as they have read them, so conversion and MMA latency stay out of
-// the weight stream) and the bf16 batch tiles (released by the MMA); a
-// double-buffered bf16 A tile the converter warps fill for the MMA; and (fused
-// cross-entropy only) a staging area for the epilogue.  The MMA of chunk i waits
-// for batch tile i, which is reloaded only after the MMA nh chunks earlier, so the
-// batch ring takes all the shared memory left (its tiles are Bn x 128 bytes).
+// warp w serves TMEM lanes 32*(w%4).., converts K half w/4 of those 32 rows, and
+// the two warps on the same lanes split the batch columns in interleaved 16-column
+// blocks (group w/4 takes blocks 2m + w/4).  Warp 8 issues TMA, warp 9 the MMAs.
+// The bf16 A tile (128 rows x 64 K) lives in tensor memory, double-buffered, so
+// shared memory holds only the two TMA rings: the fp32 weight tiles (two
+// 128-byte-swizzled 128 x 32 boxes per chunk, released by the converter warps as
+// soon as they have read them, so conversion and MMA latency stay out of the
+// weight stream) and the bf16 batch tiles (Bn x 128 bytes, released by the MMA),
+// plus (fused cross-entropy only) a staging area for the epilogue.  A chunk takes
+// about 4 us from TMA issue to arrival under full load, so both rings are as deep
+// as shared memory allows.
 constexpr int kFwdConv = 256;
 constexpr int kFwdThreads = kFwdConv + 64;
-constexpr int kFwdWRingMax = 5, kFwdHRingMax = 8;
-constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile
-constexpr int kFwdWbf = 128 * 64 * 2;                  // 16 KB bf16 A tile (x2)
+constexpr int kFwdWRingMax = 6, kFwdHRingMax = 8;
+constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile (2 boxes)
+constexpr int kFwdWBox = 128 * 32 * 4;                 // one 128 x 32 fp32 box
 constexpr int kFwdSmemMax = 227 * 1024;
 constexpr int kXentSmem = (2 * 128 * 65 + 4 * 64) * 4; // logits, gradients, statistics
 // The tensor core's fp32 accumulation loses precision roughly in proportion to the
@@ -71,25 +69,31 @@ constexpr int kXentSmem = (2 * 128 * 65 + 4 * 64) * 4; // logits, gradients, sta
 // every kSegChunks chunks (16 MMAs) the partial sum is folded into fp32 registers
 // with IEEE adds, in chunk order, while the MMAs continue in the other TMEM buffer.
 constexpr int kSegChunks = 4;
-constexpr uint32_t kFwdTmemCols = 128;   // two accumulator buffers of 64 columns
+// TMEM columns: accumulators at 0 and 64, bf16 A tiles (32 columns each) at 128, 160.
+constexpr uint32_t kFwdTmemCols = 256;
+constexpr uint32_t kFwdTmemA = 128;
 constexpr int kFwdHidden = 0, kFwdXent = 2;   // TcFwdArgs::mode (1 = logits)
 
-// Layout: W ring | A tiles | epilogue staging (mode 2) | batch ring | barriers.
-__host__ __device__ constexpr int fwd_wring(int mode) { return mode == 2 ? 3 : 5; }
-__host__ __device__ constexpr int fwd_h_off(int mode) {
-  return fwd_wring(mode) * kFwdWf32 + 2 * kFwdWbf + (mode == 2 ? kXentSmem : 0);
+// Layout: W ring | epilogue staging (mode 2) | batch ring | barriers.
+__host__ __device__ constexpr int fwd_wring(int mode, int Bn) {
+  return mode == 2 ? 3 : (Bn <= 32 ? 6 : 5);
+}
+__host__ __device__ constexpr int fwd_h_off(int mode, int Bn) {
+  return fwd_wring(mode, Bn) * kFwdWf32 + (mode == 2 ? kXentSmem : 0);
 }
 __host__ __device__ constexpr int fwd_hring(int mode, int Bn) {
-  return (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode)) / (Bn * 128) < kFwdHRingMax
-             ? (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode)) / (Bn * 128)
+  return (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode, Bn)) / (Bn * 128) < kFwdHRingMax
+             ? (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode, Bn)) / (Bn * 128)
              : kFwdHRingMax;
 }
 __host__ __device__ constexpr int fwd_bar_off(int mode, int Bn) {
-  return fwd_h_off(mode) + fwd_hring(mode, Bn) * Bn * 128;
+  return fwd_h_off(mode, Bn) + fwd_hring(mode, Bn) * Bn * 128;
 }
 __host__ __device__ constexpr int fwd_smem(int mode, int Bn) { return fwd_bar_off(mode, Bn) + 512 + 1024; }
-static_assert(fwd_hring(2, 64) >= 3 && fwd_hring(0, 64) >= 4 && fwd_smem(2, 64) <= kFwdSmemMax &&
-                  fwd_smem(0, 64) <= kFwdSmemMax && fwd_smem(0, 16) <= kFwdSmemMax,
+static_assert(fwd_hring(2, 64) >= 6 && fwd_hring(0, 64) == 8 && fwd_hring(0, 32) == 8 &&
+                  fwd_smem(2, 64) <= kFwdSmemMax && fwd_smem(0, 64) <= kFwdSmemMax &&
+                  fwd_smem(0, 48) <= kFwdSmemMax && fwd_smem(0, 32) <= kFwdSmemMax &&
+                  fwd_smem(0, 16) <= kFwdSmemMax && fwd_smem(2, 16) <= kFwdSmemMax,
               "forward shared-memory plan");
 
 // Bounded wait whose outcome is made uniform across the warp, so that a warp never
@@ -170,20 +174,7 @@ __device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, 
   }
   if (t < C) {
     float db = 0.f;
-    for (int b0 = 0; b0 < a.Bn; b0 += 8) {
-      uint32_t pk[4];
-#pragma unroll
-      for (int q = 0; q < 8; q += 2) {
-        const int b = b0 + q;
-        const float g0 = b < B ? gs[t * ZP + b] : 0.f;
-        const float g1 = b + 1 < B ? gs[t * ZP + b + 1] : 0.f;
-        if (b < B) db = __fadd_rn(db, g0);
-        if (b + 1 < B) db = __fadd_rn(db, g1);
-        pk[q / 2] = pack_bf16x2(g0, g1);
-      }
-      *reinterpret_cast<uint4*>(a.dzt_out + (static_cast<int64_t>(j) * C + t) * a.Kp + b0) =
-          make_uint4(pk[0], pk[1], pk[2], pk[3]);
-    }
+    for (int b = 0; b < B; ++b) db = __fadd_rn(db, gs[t * ZP + b]);
     float* bp = const_cast<float*>(a.bias) + static_cast<int64_t>(j) * a.ld + t;
     *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
   }
@@ -213,18 +204,17 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   const int U = a.n_tiles * nk;
   const int u0 = unit_begin(g, U, G), u1 = unit_begin(g + 1, U, G);
   const int n_local = u1 - u0;
-  const int nw = fwd_wring(a.mode), nh = fwd_hring(a.mode, a.Bn);
+  const int nw = fwd_wring(a.mode, a.Bn), nh = fwd_hring(a.mode, a.Bn);
   const int hbytes = a.Bn * 128;
   const int h_row0 = a.x_direct ? a.x_row0 : 0;           // batch rows inside the H (or X) map
   const int tile0 = u0 / nk, c0 = u0 - tile0 * nk;         // first unit's tile and chunk
-  uint8_t* wbf_base = smem + nw * kFwdWf32;
-  uint8_t* xent_sm = wbf_base + 2 * kFwdWbf;
-  uint8_t* h_base = smem + fwd_h_off(a.mode);
+  uint8_t* xent_sm = smem + nw * kFwdWf32;
+  uint8_t* h_base = smem + fwd_h_off(a.mode, a.Bn);
   uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + fwd_bar_off(a.mode, a.Bn));
   uint64_t* wempty = wfull + kFwdWRingMax;  // weight tile read by every converter warp
   uint64_t* hfull = wempty + kFwdWRingMax;
   uint64_t* hempty = hfull + kFwdHRingMax;  // batch tile consumed by the MMA
-  uint64_t* conv = hempty + kFwdHRingMax;   // [2] A tile written
+  uint64_t* conv = hempty + kFwdHRingMax;   // [2] A tile written to TMEM
   uint64_t* wfree = conv + 2;              // [2] A tile consumed by the MMA
   uint64_t* accf = wfree + 2;              // [2] accumulator segment complete
   uint64_t* accr = accf + 2;               // [2] accumulator segment drained
@@ -234,7 +224,6 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
   auto wf = [&](int s) { return smem + s * kFwdWf32; };
   auto hb = [&](int s) { return h_base + s * hbytes; };
-  auto wb = [&](int b) { return wbf_base + b * kFwdWbf; };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kFwdWRingMax; ++s) {
@@ -283,6 +272,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         if (wside) {
           mbar_arrive_expect_tx(&fullb[s], kFwdWf32);
           tma_load_3d(wf(s), &tm_w, &fullb[s], c * 64, ot * 128, j);
+          tma_load_3d(wf(s) + kFwdWBox, &tm_w, &fullb[s], c * 64 + 32, ot * 128, j);
         } else {
           mbar_arrive_expect_tx(&fullb[s], a.Bn * 128);
           tma_load_3d(hb(s), &tm_h, &fullb[s], c * 64, h_row0, j);
@@ -313,12 +303,12 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) break;
         if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) break;
         tc_fence_after();
-        const uint64_t ad = umma_desc_sw128(smem_u32(wb(b)));
+        const uint32_t at = tmem + kFwdTmemA + 32 * b;
         const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh)));
         const uint32_t d = tmem + 64 * ab;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk)
-          tc_mma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
+          tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
         tc_commit(&hempty[sh]);
         tc_commit(&wfree[b]);
         if (last) tc_commit(&accf[ab]);
@@ -423,20 +413,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           const int cb = (2 * m + gr) * 16;
           if (cb >= a.Bn) break;
           if (a.mode == kFwdHidden) {
-            uint32_t pk[8];
 #pragma unroll
-            for (int q = 0; q < 16; q += 2) {
-              const float h0 = fmaxf(__fadd_rn(acc[16 * m + q], bias), 0.f);
-              const float h1 = fmaxf(__fadd_rn(acc[16 * m + q + 1], bias), 0.f);
-              const bool in0 = cb + q < a.B, in1 = cb + q + 1 < a.B;
-              pk[q / 2] = pack_bf16x2(in0 ? h0 : 0.f, in1 ? h1 : 0.f);
-              const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
-              if (in0) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] = hh.x;
-              if (in1) a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_out + o] = hh.y;
-            }
-            uint4* dst = reinterpret_cast<uint4*>(a.ht_out + (static_cast<int64_t>(j) * a.out + o) * a.Kp + cb);
-            dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            for (int q = 0; q < 16; ++q)
+              if (cb + q < a.B)
+                a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] =
+                    __float2bfloat16_rn(fmaxf(__fadd_rn(acc[16 * m + q], bias), 0.f));
           } else {
 #pragma unroll
             for (int q = 0; q < 16; ++q)
@@ -462,43 +443,26 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       const int sw = i % nw, sh = i % nh, bb = i & 1;
       if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
       if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
-      const float* src = reinterpret_cast<const float*>(wf(sw));
-      uint8_t* dst = wb(bb);
+      tc_fence_after();
+      {
+        // Row 32*(warp%4) + lane, K half warp/4: 32 floats from the swizzled box
+        // (16-byte chunk q of row r sits at chunk q ^ (r%8)), packed to bf16 pairs,
+        // stored as 16 TMEM columns of this lane.
+        const int row = 32 * (warp & 3) + lane, half = warp >> 2;
+        const uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
+        uint32_t pk[16];
 #pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        const int f = t + kFwdConv * v;      // group of 8 floats in the [128][64] fp32 tile
-        const int row = f >> 3, k = (f & 7) * 8;
-        const float4 x0 = *reinterpret_cast<const float4*>(src + row * 64 + k);
-        const float4 x1 = *reinterpret_cast<const float4*>(src + row * 64 + k + 4);
-        *reinterpret_cast<uint4*>(dst + sw128_offset(row, k)) =
-            make_uint4(pack_bf16x2(x0.x, x0.y), pack_bf16x2(x0.z, x0.w), pack_bf16x2(x1.x, x1.y),
-                       pack_bf16x2(x1.z, x1.w));
+        for (int q = 0; q < 8; ++q) {
+          const float4 x = *reinterpret_cast<const float4*>(src + ((q ^ (row & 7)) << 4));
+          pk[2 * q] = pack_bf16x2(x.x, x.y);
+          pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
+        }
+        tmem_st16(tbase + kFwdTmemA + 32 * bb + 16 * half, pk);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&wempty[sw]);   // the fp32 tile is no longer needed
-      if (a.x_direct && ot == 0) {
-        // H_0^T[k][b] for this chunk's 64 features, from the staged batch tile
-        // (rows b >= B of the tile belong to later samples and are written as 0).
-        if (!wait_warp(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
-        const uint8_t* hs = hb(sh);
-        const int kk = t & 63;
-        const int k = c * 64 + kk;
-        if (k < a.in) {
-          for (int b0 = (t >> 6) * 8; b0 < a.Bn; b0 += 32) {
-            uint32_t pk[4];
-#pragma unroll
-            for (int q = 0; q < 8; q += 2) {
-              const int b = b0 + q;
-              const uint16_t lo = b < a.B ? *reinterpret_cast<const uint16_t*>(hs + sw128_offset(b, kk)) : 0;
-              const uint16_t hi = b + 1 < a.B ? *reinterpret_cast<const uint16_t*>(hs + sw128_offset(b + 1, kk)) : 0;
-              pk[q / 2] = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
-            }
-            *reinterpret_cast<uint4*>(a.ht0_out + (static_cast<int64_t>(j) * a.in + k) * a.Kp + b0) =
-                make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          }
-        }
-      }
-      fence_proxy_async_smem();
+      tmem_st_wait();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&conv[bb]);
       if (p % kSegChunks == 0) ++qc;
@@ -526,56 +490,107 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 }
 
 // ------------------------------------------------------------------ backward
+// Persistent stream-K backward of one layer.  Unit u = (tile, chunk): tile = (learner
+// j, input features i0 .. i0+127), chunk = output rows o0 .. o0+63 of W_l.  CTA g of G
+// owns the contiguous units [g*U/G, (g+1)*U/G).  Per unit:
+//   dW^T[i][o] = sum_b H_{l-1}[b][i] dZ_l[b][o]    both operands MN-major, read as stored
+//                                                  (H tile of the tile, dZ tile of the chunk)
+//   W[o][i]   -= lr dW^T[i][o]                     fp32, in shared memory, then TMA-stored
+//   dH^T[i][b] += sum_o W[o][i] dZ_l[b][o]          pre-update weights (A = W^T, bf16, in TMEM)
+// so W is read once and written once.  dH^T of a tile accumulates over its chunks (with
+// the same every-kSegChunks promotion as the forward); a tile split over CTAs is
+// finished, as in the forward, by the CTA holding its first chunk.  The tile epilogue
+// applies the ReLU mask of H_{l-1}, writes dZ_{l-1} and updates b_{l-1}.
+// Warps 0-3: thread t owns input feature i0 + t (TMEM lane t): it converts its column
+// of the fp32 chunk to the bf16 A tile, applies the update and runs the epilogue.
+// Warp 4: lane 0 loads W chunks and H tiles, lane 1 dZ tiles, lane 2 issues the TMA
+// stores of updated chunks (and releases their slots once read), lane 3 publishes a
+// split tile's partial.  Warp 5: the MMAs.
+constexpr int kBwdConv = 128;
+constexpr int kBwdThreads = kBwdConv + 64;
 constexpr int kBwdWf32 = 64 * 128 * 4;                 // 32 KB fp32 W chunk [64 o][128 i]
-constexpr int kBwdWT = 128 * 64 * 2;                   // 16 KB bf16 W^T [128 i][64 o]
-constexpr int kBwdDZ = 64 * 128;                       //  8 KB bf16 dZ [Bn][64 o]
-constexpr int kBwdDZT = 64 * 128;                      //  8 KB bf16 dZ^T [64 o][64 b]
-constexpr int kBwdStage = kBwdWf32 + kBwdWT + kBwdDZ + kBwdDZT;   // 64 KB
-constexpr int kBwdHT = 128 * 128;                      // 16 KB bf16 H^T [128 i][64 b]
-constexpr int kBwdBarOff = kStages * kBwdStage + kBwdHT;
-constexpr int kBwdSmem = kBwdBarOff + 256 + 1024;
-constexpr uint32_t kBwdTmemCols = 256;   // dX buffers at columns 0 and 192, dW buffers at 64, 128
+constexpr int kBwdWRingMax = 5, kBwdZRingMax = 8;
+constexpr int kBwdSmemMax = 227 * 1024;
+// TMEM columns: dH^T accumulators at 0 and 64, dW^T at 128 and 192, W^T (A) at 256, 288.
+constexpr uint32_t kBwdTmemCols = 512;
+constexpr uint32_t kBwdTmemW = 128, kBwdTmemA = 256;
 
-__global__ void __launch_bounds__(kThreads, 1)
-    k_tc_backward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_ht,
-                  const __grid_constant__ CUtensorMap tm_dz, const __grid_constant__ CUtensorMap tm_dzt,
-                  const TcBwdArgs a) {
+// Layout: W ring | 2 H tiles (2 x [Bn][64] bf16 each) | dZ ring ([Bn][64] bf16) | barriers.
+__host__ __device__ constexpr int bwd_wring(int Bn) { return Bn <= 32 ? 5 : 4; }
+__host__ __device__ constexpr int bwd_h_off(int Bn) { return bwd_wring(Bn) * kBwdWf32; }
+__host__ __device__ constexpr int bwd_z_off(int Bn) { return bwd_h_off(Bn) + 2 * 2 * Bn * 128; }
+__host__ __device__ constexpr int bwd_zring(int Bn) {
+  return (kBwdSmemMax - 1024 - 512 - bwd_z_off(Bn)) / (Bn * 128) < kBwdZRingMax
+             ? (kBwdSmemMax - 1024 - 512 - bwd_z_off(Bn)) / (Bn * 128)
+             : kBwdZRingMax;
+}
+__host__ __device__ constexpr int bwd_bar_off(int Bn) { return bwd_z_off(Bn) + bwd_zring(Bn) * Bn * 128; }
+__host__ __device__ constexpr int bwd_smem(int Bn) { return bwd_bar_off(Bn) + 512 + 1024; }
+static_assert(bwd_zring(64) >= 6 && bwd_zring(48) >= 6 && bwd_zring(32) >= 6 && bwd_zring(16) >= 6 &&
+                  bwd_smem(64) <= kBwdSmemMax && bwd_smem(48) <= kBwdSmemMax &&
+                  bwd_smem(32) <= kBwdSmemMax && bwd_smem(16) <= kBwdSmemMax,
+              "backward shared-memory plan");
+
+__global__ void __launch_bounds__(kBwdThreads, 1)
+    k_tc_backward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
+                  const __grid_constant__ CUtensorMap tm_dz, const TcBwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int j = blockIdx.y, i0 = blockIdx.x * 128;
+  const int g = blockIdx.x, G = gridDim.x;
   const int nc = (a.out + 63) / 64;
-  uint8_t* ht = smem + kStages * kBwdStage;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBwdBarOff);
-  uint64_t* conv = full + kStages;
-  uint64_t* mdone = conv + kStages;
-  uint64_t* empty = mdone + kStages;
-  uint64_t* tfree = empty + kStages;   // [2]
-  uint64_t* htfull = tfree + 2;
-  uint64_t* upd = htfull + 1;         // [kStages] updated chunk ready for the TMA store
-  uint64_t* xf = upd + kStages;       // [2] dX accumulator segment complete
-  uint64_t* xr = xf + 2;              // [2] dX accumulator segment drained
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xr + 2);
-  auto wf = [&](int s) { return smem + s * kBwdStage; };
-  auto wt = [&](int s) { return smem + s * kBwdStage + kBwdWf32; };
-  auto dzb = [&](int s) { return smem + s * kBwdStage + kBwdWf32 + kBwdWT; };
-  auto dztb = [&](int s) { return smem + s * kBwdStage + kBwdWf32 + kBwdWT + kBwdDZ; };
+  const int U = a.n_tiles * nc;
+  const int u0 = unit_begin(g, U, G), u1 = unit_begin(g + 1, U, G);
+  const int n_local = u1 - u0;
+  const int nw = bwd_wring(a.Bn), nz = bwd_zring(a.Bn);
+  const int tbytes = a.Bn * 128;                           // one [Bn][64] bf16 tile
+  const int tile0 = u0 / nc, c0 = u0 - tile0 * nc;
+  uint8_t* h_base = smem + bwd_h_off(a.Bn);
+  uint8_t* z_base = smem + bwd_z_off(a.Bn);
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + bwd_bar_off(a.Bn));
+  uint64_t* wempty = wfull + kBwdWRingMax;   // chunk stored back (TMA has read it)
+  uint64_t* upd = wempty + kBwdWRingMax;     // chunk updated in shared memory
+  uint64_t* zfull = upd + kBwdWRingMax;
+  uint64_t* zempty = zfull + kBwdZRingMax;   // dZ tile consumed by both MMAs
+  uint64_t* hfull = zempty + kBwdZRingMax;   // [2]
+  uint64_t* hempty = hfull + 2;              // [2] tile epilogue done
+  uint64_t* conv = hempty + 2;               // [2] W^T written to TMEM
+  uint64_t* afree = conv + 2;                // [2] W^T consumed by the dX MMA
+  uint64_t* dwdone = afree + 2;              // [2] dW^T of the chunk complete
+  uint64_t* dwfree = dwdone + 2;             // [2] dW^T read by the update
+  uint64_t* xf = dwfree + 2;                 // [2] dH^T segment complete
+  uint64_t* xr = xf + 2;                     // [2] dH^T segment drained
+  uint64_t* gbar = xr + 2;
+  uint64_t* done = gbar + 1;
+  uint64_t* pready = done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
+  auto wf = [&](int s) { return smem + s * kBwdWf32; };
+  auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
+  auto zb = [&](int s) { return z_base + s * tbytes; };
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&conv[s], kConv);
-      mbar_init(&mdone[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int s = 0; s < kBwdWRingMax; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], 1);
+      mbar_init(&upd[s], kBwdConv / 32);
     }
-    mbar_init(&tfree[0], kConv);
-    mbar_init(&tfree[1], kConv);
-    mbar_init(htfull, 1);
-    for (int s = 0; s < kStages; ++s) mbar_init(&upd[s], kConv);
+    for (int s = 0; s < kBwdZRingMax; ++s) {
+      mbar_init(&zfull[s], 1);
+      mbar_init(&zempty[s], 1);
+    }
     for (int b = 0; b < 2; ++b) {
+      mbar_init(&hfull[b], 1);
+      mbar_init(&hempty[b], kBwdConv / 32);
+      mbar_init(&conv[b], kBwdConv / 32);
+      mbar_init(&afree[b], 1);
+      mbar_init(&dwdone[b], 1);
+      mbar_init(&dwfree[b], kBwdConv / 32);
       mbar_init(&xf[b], 1);
-      mbar_init(&xr[b], kConv);
+      mbar_init(&xr[b], kBwdConv / 32);
     }
+    mbar_init(gbar, kBwdConv);
+    mbar_init(done, 1);
+    mbar_init(pready, kBwdConv / 32);
     fence_barrier_init();
   }
   if (warp == 5) {
@@ -589,69 +604,114 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 4) {
     if (lane == 0) {
+      // W chunks, and each tile's H tile (two 64-feature boxes) ahead of its first chunk
       tma_prefetch_desc(&tm_w);
-      tma_prefetch_desc(&tm_ht);
-      tma_prefetch_desc(&tm_dz);
-      tma_prefetch_desc(&tm_dzt);
-      mbar_arrive_expect_tx(htfull, kBwdHT);
-      tma_load_3d(ht, &tm_ht, htfull, 0, i0, j);
-      const uint32_t bytes = kBwdWf32 + kBwdDZT + (a.has_dx ? a.Bn * 128 : 0);
-      int issued = 0;
-      for (int c = 0; c < nc; ++c) {
-        const int s = c % kStages;
-        if (c >= kStages && !mbar_wait(&empty[s], ((c / kStages) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&full[s], bytes);
-        tma_load_3d(wf(s), &tm_w, &full[s], i0, c * 64, j);
-        if (a.has_dx) tma_load_3d(dzb(s), &tm_dz, &full[s], c * 64, 0, j);
-        tma_load_3d(dztb(s), &tm_dzt, &full[s], 0, c * 64, j);
-        issued = c + 1;
+      tma_prefetch_desc(&tm_h);
+      int issued = 0, tau = tile0, c = c0, kt = 0;
+      bool ok = true;
+      for (int i = 0; i < n_local && ok; ++i) {
+        const int j = tau / a.s_tiles, i0 = (tau - j * a.s_tiles) * 128;
+        if (i == 0 || c == 0) {
+          const int hbuf = kt & 1;
+          if (kt >= 2 && !mbar_wait(&hempty[hbuf], ((kt >> 1) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&hfull[hbuf], 2 * tbytes);
+          tma_load_3d(hb(hbuf), &tm_h, &hfull[hbuf], i0, a.h_row0, j);
+          tma_load_3d(hb(hbuf) + tbytes, &tm_h, &hfull[hbuf], i0 + 64, a.h_row0, j);
+          ++kt;
+        }
+        const int s = i % nw;
+        if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+        mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
+        tma_load_3d(wf(s), &tm_w, &wfull[s], i0, c * 64, j);
+        issued = i + 1;
+        if (++c == nc) { c = 0; ++tau; }
       }
-      mbar_wait(htfull, 0, a.err);
-      for (int c = issued - kStages > 0 ? issued - kStages : 0; c < issued; ++c)
-        mbar_wait(&full[c % kStages], (c / kStages) & 1, a.err);
+      for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
+        mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
+      for (int k = kt - 2 > 0 ? kt - 2 : 0; k < kt; ++k) mbar_wait(&hfull[k & 1], (k >> 1) & 1, a.err);
+    } else if (lane == 1) {
+      tma_prefetch_desc(&tm_dz);
+      int issued = 0, tau = tile0, c = c0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.s_tiles;
+        const int s = i % nz;
+        if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&zfull[s], tbytes);
+        tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j);
+        issued = i + 1;
+        if (++c == nc) { c = 0; ++tau; }
+      }
+      for (int i = issued - nz > 0 ? issued - nz : 0; i < issued; ++i)
+        mbar_wait(&zfull[i % nz], (i / nz) & 1, a.err);
+    } else if (lane == 2) {
+      // Store each updated chunk; its slot is released once the TMA has read it.
+      int tau = tile0, c = c0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.s_tiles, i0 = (tau - j * a.s_tiles) * 128;
+        const int s = i % nw;
+        if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
+        tma_store_3d(&tm_w, wf(s), i0, c * 64, j);
+        tma_store_commit();
+        tma_store_wait_read_all();
+        mbar_arrive(&wempty[s]);
+        if (++c == nc) { c = 0; ++tau; }
+      }
+      tma_store_wait_all();
+    } else if (lane == 3 && a.has_dx && c0 != 0 && n_local > 0) {
+      if (mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
     }
   } else if (warp == 5) {
     if (lane == 0) {
+      const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
       const uint32_t idesc_dx = umma_idesc_bf16(128, a.Bn);
-      const uint32_t idesc_dw = umma_idesc_bf16(128, 64);
-      const int kb = (a.B + 15) / 16;   // K = B for dW
-      bool ok = mbar_wait(htfull, 0, a.err);
-      const uint64_t hd = umma_desc_sw128(smem_u32(ht));
-      int c = 0;
-      for (; ok && c < nc; ++c) {
-        const int s = c % kStages, buf = c & 1;
-        const int seg = c / kSegChunks, xb = seg & 1, first = c % kSegChunks == 0;
-        if (a.has_dx && first && seg >= 2 && !mbar_wait(&xr[xb], ((seg >> 1) - 1) & 1, a.err)) break;
-        if (!mbar_wait(&conv[s], (c / kStages) & 1, a.err)) break;
-        if (c >= 2 && !mbar_wait(&tfree[buf], ((c / 2) - 1) & 1, a.err)) break;
+      const int kb = a.Bn / 16;   // K = Bn for dW
+      int tau = tile0, c = c0, p = 0, q = -1, kt = -1;
+      for (int i = 0; i < n_local; ++i) {
+        const bool tlast = i == n_local - 1 || c == nc - 1;
+        const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+        const int sz = i % nz, b = i & 1;
+        if (p == 0) {
+          ++kt;
+          if (!mbar_wait(&hfull[kt & 1], (kt >> 1) & 1, a.err)) break;
+        }
+        if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) break;
+        if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) break;
         tc_fence_after();
+        const uint32_t hs = smem_u32(hb(kt & 1)), zs = smem_u32(zb(sz));
+        for (int kk = 0; kk < kb; ++kk)
+          tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
+                      umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+        tc_commit(&dwdone[b]);
         if (a.has_dx) {
-          const uint64_t ad = umma_desc_sw128(smem_u32(wt(s)));
-          const uint64_t bd = umma_desc_sw128(smem_u32(dzb(s)));
+          if (first) ++q;
+          const int xb = q & 1;
+          if (first && q >= 2 && !mbar_wait(&xr[xb], ((q >> 1) - 1) & 1, a.err)) break;
+          if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) break;
+          tc_fence_after();
+          const uint64_t zd = umma_desc_sw128(zs);
 #pragma unroll
           for (int kk = 0; kk < 4; ++kk)
-            tc_mma_bf16(tmem + 192 * xb, ad + 2 * kk, bd + 2 * kk, idesc_dx,
-                        (!first || kk > 0) ? 1u : 0u);
+            tc_mma_bf16_ta(tmem + 64 * xb, tmem + kBwdTmemA + 32 * b + 8 * kk, zd + 2 * kk, idesc_dx,
+                           (!first || kk > 0) ? 1u : 0u);
+          tc_commit(&afree[b]);
+          if (last) tc_commit(&xf[xb]);
         }
-        const uint64_t bd = umma_desc_sw128(smem_u32(dztb(s)));
-        for (int kk = 0; kk < kb; ++kk)
-          tc_mma_bf16(tmem + 64 + 64 * buf, hd + 2 * kk, bd + 2 * kk, idesc_dw, kk > 0 ? 1u : 0u);
-        tc_commit(&mdone[s]);
-        if (a.has_dx && (c % kSegChunks == kSegChunks - 1 || c == nc - 1)) tc_commit(&xf[xb]);
+        tc_commit(&zempty[sz]);
+        ++p;
+        if (++c == nc) { c = 0; p = 0; ++tau; }
       }
-      // Drain: the last commit covers every MMA issued before it.
-      if (c > 0) mbar_wait(&mdone[(c - 1) % kStages], ((c - 1) / kStages) & 1, a.err);
+      tc_commit(done);
+      mbar_wait(done, 0, a.err);
     }
   } else {
-    // ---- warps 0-3: W^T for dX, the in-place SGD update, then the dX epilogue
+    // ---- warps 0-3
     const int t = threadIdx.x;
     const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
-    // dX accumulator promoted to registers segment by segment (see kSegChunks)
-    float accx[64];
+    GroupSync gsync{gbar, 0, a.err};
+    float accx[64];                                // dH^T[i0 + t][0 .. Bn), promoted
 #pragma unroll
     for (int q = 0; q < 64; ++q) accx[q] = 0.f;
-    int drained = 0;
-    const int nseg = a.has_dx ? (nc + kSegChunks - 1) / kSegChunks : 0;
+    int qc = -1, drained = 0;
     auto drain = [&]() -> bool {
       const int xb = drained & 1;
       if (!wait_warp(&xf[xb], (drained >> 1) & 1, a.err)) return false;
@@ -660,111 +720,140 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int cb = 0; cb < 64; cb += 16) {
         if (cb < a.Bn) {
           float v[16];
-          tmem_ld16(tbase + 192 * xb + cb, v);
+          tmem_ld16(tbase + 64 * xb + cb, v);
           tmem_ld_wait();
 #pragma unroll
           for (int q = 0; q < 16; ++q) accx[cb + q] = __fadd_rn(accx[cb + q], v[q]);
         }
       }
       tc_fence_before();
-      mbar_arrive(&xr[xb]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&xr[xb]);
       ++drained;
       return true;
     };
-    bool ok = true;
-    for (int c = 0; c <= nc && ok; ++c) {
-      if (c < nc) {
-        const int s = c % kStages;
-        if (!wait_warp(&full[s], (c / kStages) & 1, a.err)) { ok = false; break; }
-        if (a.has_dx) {
-          const float* src = reinterpret_cast<const float*>(wf(s));
-          uint8_t* dst = wt(s);
+    // End of tile tau in this CTA (has_dx): finish it, or publish this CTA's part.
+    auto tile_end = [&](int tau, bool whole, int kt) -> bool {
+      const int j = tau / a.s_tiles, fi = (tau - j * a.s_tiles) * 128 + t;
+      if (!whole) {
+        if (tau * nc < u0) {
+          float* mine = a.part + (static_cast<int64_t>(g) * 128 + t) * a.Bn;
 #pragma unroll
-          for (int ob = 0; ob < 8; ++ob) {
-            float v[8];
-#pragma unroll
-            for (int q = 0; q < 8; ++q) v[q] = src[(ob * 8 + q) * 128 + t];
-            *reinterpret_cast<uint4*>(dst + sw128_offset(t, ob * 8)) =
-                make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                           pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
-          }
-          fence_proxy_async_smem();
+          for (int cb = 0; cb < 64; cb += 4)
+            if (cb < a.Bn)
+              __stcg(reinterpret_cast<float4*>(mine + cb),
+                     make_float4(accx[cb], accx[cb + 1], accx[cb + 2], accx[cb + 3]));
+          __syncwarp();
+          if (lane == 0) mbar_arrive(pready);
+          return true;
         }
-        mbar_arrive(&conv[s]);
-      }
-      if (c > 0) {
-        const int cp = c - 1, sp = cp % kStages, buf = cp & 1;
-        if (!wait_warp(&mdone[sp], (cp / kStages) & 1, a.err)) { ok = false; break; }
-        tc_fence_after();
-        float* w = reinterpret_cast<float*>(wf(sp));
-#pragma unroll
-        for (int qb = 0; qb < 4; ++qb) {
-          float d[16];
-          tmem_ld16(tbase + 64 + 64 * buf + 16 * qb, d);
-          tmem_ld_wait();
-#pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            float* p = w + (qb * 16 + q) * 128 + t;
-            *p = __fsub_rn(*p, __fmul_rn(a.lr, d[q]));
-          }
-        }
-        tc_fence_before();
-        mbar_arrive(&tfree[buf]);
-        fence_proxy_async_smem();
-        mbar_arrive(&upd[sp]);
+        const int g_last = cta_of((tau + 1) * nc - 1, U, G);
         if (t == 0) {
-          if (mbar_wait(&upd[sp], (cp / kStages) & 1, a.err)) {
-            tma_store_3d(&tm_w, w, i0, cp * 64, j);
-            tma_store_commit();
-            tma_store_wait_read_all();
-          }
-          mbar_arrive(&empty[sp]);
+          const bool ok = spin_acquire_eq(a.counters + tau, g_last - g, a.err);
+          if (ok) a.counters[tau] = 0;
         }
-        if (a.has_dx && cp % kSegChunks == kSegChunks - 1 && cp / kSegChunks >= 1 &&
-            drained < cp / kSegChunks)
-          if (!drain()) { ok = false; break; }
-      }
-    }
-    while (ok && drained < nseg)
-      if (!drain()) ok = false;
-    if (t == 0) tma_store_wait_all();
-    if (ok && a.has_dx) {
-      // dX epilogue: thread t holds dH^T[i0 + t][0 .. Bn) in accx
-      const int i = i0 + t;
-      const bool valid = i < a.in;
-      float db = 0.f;
+        if (!gsync()) return false;
+        for (int gg = g + 1; gg <= g_last; ++gg) {
+          const float* src = a.part + (static_cast<int64_t>(gg) * 128 + t) * a.Bn;
 #pragma unroll
-      for (int cb = 0; cb < 64; cb += 16) {
-        if (cb >= a.Bn || !valid) break;
-        const float* v = accx + cb;
-        uint32_t pk[8];
-#pragma unroll
-        for (int q = 0; q < 16; q += 2) {
-          float dz[2];
-#pragma unroll
-          for (int e = 0; e < 2; ++e) {
-            const int b = cb + q + e;
-            float x = 0.f;
-            if (b < a.B) {
-              const __nv_bfloat16 h = *reinterpret_cast<const __nv_bfloat16*>(ht + sw128_offset(t, b));
-              x = (__bfloat162float(h) > 0.f) ? v[q + e] : 0.f;
-              db = __fadd_rn(db, x);
+          for (int cb = 0; cb < 64; cb += 4) {
+            if (cb < a.Bn) {
+              const float4 v = __ldcg(reinterpret_cast<const float4*>(src + cb));
+              accx[cb] = __fadd_rn(accx[cb], v.x);
+              accx[cb + 1] = __fadd_rn(accx[cb + 1], v.y);
+              accx[cb + 2] = __fadd_rn(accx[cb + 2], v.z);
+              accx[cb + 3] = __fadd_rn(accx[cb + 3], v.w);
             }
-            dz[e] = x;
           }
-          pk[q / 2] = pack_bf16x2(dz[0], dz[1]);
-          const __nv_bfloat162 hh = *reinterpret_cast<__nv_bfloat162*>(&pk[q / 2]);
-          if (cb + q < a.B) a.dz_prev[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_in + i] = hh.x;
-          if (cb + q + 1 < a.B) a.dz_prev[(static_cast<int64_t>(j) * a.Bn + cb + q + 1) * a.pitch_in + i] = hh.y;
         }
-        uint4* dst = reinterpret_cast<uint4*>(a.dzt_prev + (static_cast<int64_t>(j) * a.in + i) * a.Kp + cb);
-        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
       }
-      if (valid) {
-        float* bp = a.bias_prev + static_cast<int64_t>(j) * a.ld + i;
+      // dZ_{l-1}[b][i] = dH[b][i] * (H_{l-1}[b][i] > 0), b < B; b_{l-1}[i] -= lr sum_b.
+      // (The H tile landed long ago; the wait makes the TMA's writes visible here.)
+      if (!wait_warp(&hfull[kt & 1], (kt >> 1) & 1, a.err)) return false;
+      if (fi < a.in) {
+        const uint8_t* hcol = hb(kt & 1) + (t >> 6) * a.Bn * 128;
+        __nv_bfloat16* dz = a.dz_prev + static_cast<int64_t>(j) * a.Bn * a.pitch_in + fi;
+        float db = 0.f;
+#pragma unroll
+        for (int b = 0; b < 64; ++b) {
+          if (b < a.B) {
+            const __nv_bfloat16 hv =
+                *reinterpret_cast<const __nv_bfloat16*>(hcol + sw128_offset(b, t & 63));
+            const float x = __bfloat162float(hv) > 0.f ? accx[b] : 0.f;
+            db = __fadd_rn(db, x);
+            dz[static_cast<int64_t>(b) * a.pitch_in] = __float2bfloat16_rn(x);
+          }
+        }
+        float* bp = a.bias_prev + static_cast<int64_t>(j) * a.ld + fi;
         *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
       }
+      return true;
+    };
+    bool ok = true;
+    int tau = tile0, c = c0, p = 0, kt = -1;
+    for (int i = 0; i < n_local && ok; ++i) {
+      const bool tlast = i == n_local - 1 || c == nc - 1;
+      const int sw = i % nw, b = i & 1;
+      if (p == 0) ++kt;
+      if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+      float* w = reinterpret_cast<float*>(wf(sw));
+      float wv[64];
+#pragma unroll
+      for (int o = 0; o < 64; ++o) wv[o] = w[o * 128 + t];
+      if (a.has_dx) {
+        if (i >= 2 && !wait_warp(&afree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) pk[q] = pack_bf16x2(wv[32 * hh + 2 * q], wv[32 * hh + 2 * q + 1]);
+          tmem_st16(tbase + kBwdTmemA + 32 * b + 16 * hh, pk);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&conv[b]);
+      }
+      if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+      tc_fence_after();
+#pragma unroll
+      for (int qb = 0; qb < 4; ++qb) {
+        float d[16];
+        tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
+        tmem_ld_wait();
+#pragma unroll
+        for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&dwfree[b]);
+#pragma unroll
+      for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&upd[sw]);
+      if (a.has_dx) {
+        if (p % kSegChunks == 0) ++qc;
+        if (tlast) {
+          while (ok && drained <= qc)
+            if (!drain()) ok = false;
+          if (ok) {
+            const bool whole = (tau != tile0 || c0 == 0) && c == nc - 1;
+            ok = __all_sync(0xffffffffu, tile_end(tau, whole, kt));
+#pragma unroll
+            for (int q = 0; q < 64; ++q) accx[q] = 0.f;
+          }
+        } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
+          if (!drain()) ok = false;
+        }
+      }
+      if (tlast) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&hempty[kt & 1]);   // the H tile may be replaced
+      }
+      ++p;
+      if (++c == nc) { c = 0; p = 0; ++tau; }
     }
   }
   tc_fence_before();
@@ -777,41 +866,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ------------------------------------------------------------------ gather
-// H_0[j][b][:] = X[j][(t*B + b) mod N][:], HT_0[j][k][b] = the same; one CTA per
-// (64-feature slice, learner).  Rows b >= B and columns b >= B stay zero.
+// H_0[j][b][:] = X[j][(t*B + b) mod N][:] for b < B, one CTA per (64-feature slice,
+// learner); rows b >= B stay zero.
 __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __restrict__ X,
-                                                    int64_t N, int d0, int B, int Bn, int Kp,
+                                                    int64_t N, int d0, int B, int Bn,
                                                     int pitch0, int64_t t,
-                                                    __nv_bfloat16* __restrict__ H0,
-                                                    __nv_bfloat16* __restrict__ HT0) {
-  __shared__ __align__(16) __nv_bfloat16 tile[64][64 + 8];
+                                                    __nv_bfloat16* __restrict__ H0) {
   const int j = blockIdx.y, k0 = blockIdx.x * 64;
   const int nvec = B * 8;                       // 16-byte vectors in the [B][64] slice
   for (int idx = threadIdx.x; idx < nvec; idx += blockDim.x) {
     const int b = idx >> 3, v = idx & 7;
     const int k = k0 + v * 8;
-    uint4 val = make_uint4(0, 0, 0, 0);
     if (k < d0) {
       const int64_t row = (t * B + b) % N;
-      val = *reinterpret_cast<const uint4*>(X + (static_cast<int64_t>(j) * N + row) * d0 + k);
-      *reinterpret_cast<uint4*>(H0 + (static_cast<int64_t>(j) * Bn + b) * pitch0 + k) = val;
+      *reinterpret_cast<uint4*>(H0 + (static_cast<int64_t>(j) * Bn + b) * pitch0 + k) =
+          *reinterpret_cast<const uint4*>(X + (static_cast<int64_t>(j) * N + row) * d0 + k);
     }
-    *reinterpret_cast<uint4*>(&tile[b][v * 8]) = val;
-  }
-  __syncthreads();
-  const int nbv = Bn / 8;                       // 8-column groups of the transposed row
-  for (int idx = threadIdx.x; idx < 64 * nbv; idx += blockDim.x) {
-    const int kk = idx / nbv, bv = idx % nbv;
-    const int k = k0 + kk;
-    if (k >= d0) continue;
-    __align__(16) __nv_bfloat16 vals[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int b = bv * 8 + q;
-      vals[q] = b < B ? tile[b][kk] : __float2bfloat16_rn(0.f);
-    }
-    *reinterpret_cast<uint4*>(HT0 + (static_cast<int64_t>(j) * d0 + k) * Kp + bv * 8) =
-        *reinterpret_cast<uint4*>(vals);
   }
 }
 
@@ -820,16 +890,14 @@ __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __rest
 // Grid (P, class slices of 256).  Every CTA computes the per-sample statistics
 // (max, sum of exponentials over all C classes; warp per sample), then each
 // thread owns one class of its slice: dZ = (p - onehot(y_b)) / B in fp32 for
-// every sample, the bf16 operands dZ and dZ^T, and b_L -= lr * sum_b dZ (summed
-// in sample order).  Slice 0 also writes the learner's mean loss.
+// every sample, its bf16 copy, and b_L -= lr * sum_b dZ (summed in sample order).  Slice 0 also writes the learner's mean loss.
 constexpr int kXentThreads = 256;
 __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restrict__ Z,
                                                            const int32_t* __restrict__ y,
                                                            int64_t N, int64_t t, int B, int Bn,
-                                                           int Kp, int C, int pitch_c, float lr,
+                                                           int C, int pitch_c, float lr,
                                                            float* bias_L, int64_t ld,
-                                                           __nv_bfloat16* dZ, __nv_bfloat16* dZT,
-                                                           float* loss) {
+                                                           __nv_bfloat16* dZ, float* loss) {
   __shared__ float row_max[64], row_sum[64], row_loss[64];
   __shared__ int row_y[64];
   const int j = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -862,27 +930,11 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
   if (c >= C) return;
   const float fB = static_cast<float>(B);
   float db = 0.f;
-  for (int b0 = 0; b0 < Bn; b0 += 8) {
-    uint32_t pk[4];
-#pragma unroll
-    for (int q = 0; q < 8; q += 2) {
-      float g2[2];
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int b = b0 + q + e;
-        float g = 0.f;
-        if (b < B) {
-          const float p = __fdiv_rn(expf(Zj[static_cast<int64_t>(b) * C + c] - row_max[b]), row_sum[b]);
-          g = __fdiv_rn(__fsub_rn(p, row_y[b] == c ? 1.f : 0.f), fB);
-          db = __fadd_rn(db, g);
-          dZ[(static_cast<int64_t>(j) * Bn + b) * pitch_c + c] = __float2bfloat16_rn(g);
-        }
-        g2[e] = g;
-      }
-      pk[q / 2] = pack_bf16x2(g2[0], g2[1]);
-    }
-    *reinterpret_cast<uint4*>(dZT + (static_cast<int64_t>(j) * C + c) * Kp + b0) =
-        make_uint4(pk[0], pk[1], pk[2], pk[3]);
+  for (int b = 0; b < B; ++b) {
+    const float p = __fdiv_rn(expf(Zj[static_cast<int64_t>(b) * C + c] - row_max[b]), row_sum[b]);
+    const float g = __fdiv_rn(__fsub_rn(p, row_y[b] == c ? 1.f : 0.f), fB);
+    db = __fadd_rn(db, g);
+    dZ[(static_cast<int64_t>(j) * Bn + b) * pitch_c + c] = __float2bfloat16_rn(g);
   }
   float* bp = bias_L + static_cast<int64_t>(j) * ld + c;
   *bp = __fsub_rn(*bp, __fmul_rn(lr, db));
@@ -891,13 +943,14 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
 }  // namespace
 
 int tc_fwd_smem_bytes() { return kFwdSmemMax; }
-int tc_bwd_smem_bytes() { return kBwdSmem; }
+int tc_bwd_smem_bytes() { return kBwdSmemMax; }
 
 cudaError_t tc_configure() {
   cudaError_t e = cudaFuncSetAttribute(k_tc_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        kFwdSmemMax);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmem);
+  return cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kBwdSmemMax);
 }
 
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
@@ -918,28 +971,35 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
   return cudaLaunchKernelEx(&cfg, k_tc_forward, w_fwd, h_in, a);
 }
 
-cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& ht_in,
-                               const CUtensorMap& dz, const CUtensorMap& dzt,
-                               const TcBwdArgs& a, int P, cudaStream_t s) {
-  dim3 grid((a.in + 127) / 128, P);
-  k_tc_backward<<<grid, kThreads, kBwdSmem, s>>>(w_bwd, ht_in, dz, dzt, a);
-  return cudaGetLastError();
+cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
+                               const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s) {
+  (void)P;
+  // Cooperative for the same reason as the forward (split dX tiles).
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.ctas);
+  cfg.blockDim = dim3(kBwdThreads);
+  cfg.dynamicSmemBytes = bwd_smem(a.Bn);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_tc_backward, w_bwd, h_in, dz, a);
 }
 
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
-                               int Kp, int pitch0, int64_t t, int P, __nv_bfloat16* H0,
-                               __nv_bfloat16* HT0, cudaStream_t s) {
+                               int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s) {
   dim3 grid((d0 + 63) / 64, P);
-  k_gather_bf16<<<grid, 256, 0, s>>>(X, N, d0, B, Bn, Kp, pitch0, t, H0, HT0);
+  k_gather_bf16<<<grid, 256, 0, s>>>(X, N, d0, B, Bn, pitch0, t, H0);
   return cudaGetLastError();
 }
 
 cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
-                             int Bn, int Kp, int C, int pitch_c, float lr, float* bias_L,
-                             int64_t ld, __nv_bfloat16* dZ, __nv_bfloat16* dZT, float* loss,
-                             int P, cudaStream_t s) {
+                             int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
+                             __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s) {
   dim3 grid(P, (C + kXentThreads - 1) / kXentThreads);
-  k_xent_bf16<<<grid, kXentThreads, 0, s>>>(Z, y, N, t, B, Bn, Kp, C, pitch_c, lr, bias_L, ld, dZ, dZT, loss);
+  k_xent_bf16<<<grid, kXentThreads, 0, s>>>(Z, y, N, t, B, Bn, C, pitch_c, lr, bias_L, ld, dZ, loss);
   return cudaGetLastError();
 }
 
