@@ -158,8 +158,8 @@ def launches_per_round(w) -> int:
             if (t * w.B) % w.N + w.B > w.N:
                 gathers += 1
         C, din = w.dims[-1], w.dims[-2]
-        if C <= 16 and din % 64 == 0 and w.B <= 64:      # small last layer: 2 CUDA-core kernels
-            per_step = (L - 1) + 2 + (L - 1)
+        if C <= 16 and din % 64 == 0 and w.B <= 64:      # small last layer: one cluster kernel
+            per_step = (L - 1) + 1 + (L - 1)
         else:
             per_step = L + (0 if C <= 128 else 1) + L
         n = w.K1 * w.K2 * per_step + gathers

@@ -65,7 +65,6 @@ struct hier_avg {
   std::vector<int64_t> off_H, off_dZ;
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
-  int64_t off_gq = 0;                         // small-head CE gradient
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
   std::vector<int> bwd_ctas, bwd_tiles;       // per layer: stream-K CTAs, input slices
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
@@ -191,7 +190,6 @@ int plan_layout(hier_avg* h) {
     h->fused_xent = h->dims[L] <= 128;
     h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B));
     h->off_part = take(part_bytes);
-    h->off_gq = take(h->head ? int64_t(ha::head_scratch_floats(h->P, h->Bn)) * 4 : 16);
     h->off_cnt = take(max_tiles * 4);
   } else {
     for (int l = 0; l <= L; ++l) h->pitch[l] = h->dims[l];
@@ -363,7 +361,6 @@ int do_step(hier_avg* h) {
         a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[L - 1]);
       }
       a.loss = h->loss();
-      a.gq = h->wsp<float>(h->off_gq);
       const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0));
       rc = h->timed(HA_KERNEL_HEAD, hb, [&] { return ha::launch_head(a, P, s); }, "head");
       if (rc) return rc;

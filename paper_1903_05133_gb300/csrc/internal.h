@@ -85,8 +85,8 @@ cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_
                              int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
                              __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s);
 
-// Small last layer (<= 16 classes) on CUDA cores: a per-learner forward + softmax-CE
-// kernel and a per-feature-slice backward kernel, linked by the scratch `gq`.
+// Small last layer (<= 16 classes) on CUDA cores: one kernel, a thread-block cluster
+// of feature slices per learner (forward, softmax-CE and backward).
 struct HeadArgs {
   int C, in, B, Bn, pitch_in;
   int64_t ld, N, t;
@@ -100,10 +100,8 @@ struct HeadArgs {
   float* bias_prev;
   __nv_bfloat16* dz_prev;     // [P][Bn][pitch_in]
   float* loss;                // [P]
-  float* gq;                  // scratch: bf16-rounded CE gradient [P][Bn][16]
 };
 bool head_supported(int C, int in, int B);
-int head_scratch_floats(int P, int Bn);
 cudaError_t head_configure();   // raises the dynamic shared-memory limit once
 cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s);
 

@@ -1,16 +1,19 @@
 // Last layer of the learner step when it is small (at most 16 classes), on CUDA
 // cores (Algorithm 1 inner loop, Sec. 3.1).  The layer holds only C x d_{L-1}
 // weights, far too few to feed a tensor-core tile; bf16 operands, fp32
-// accumulation in a fixed order.  Two kernels:
-//   k_head_fwd  one CTA per learner.  Z[b][c] = sum_k H[b][k] W_q[c][k] + b_L[c]
-//               (warps own samples, lanes split k, butterfly sum), the CE gradient
-//               g[b][c] = (softmax(Z[b])_c - [c == y_b]) / B into a scratch buffer
-//               (fp32 and bf16-rounded), b_L -= lr * sum_b g, and the loss.
-//   k_head_bwd  one CTA per (128-feature slice, learner), one thread per feature k:
-//               with W before its update, dW[c][k] = sum_b g_q[b][c] H[b][k],
-//               dH[b][k] = sum_c g_q[b][c] W_q[c][k], dZ_{L-1}[b][k] = dH [H > 0]
-//               (bf16 and transposed copies, fp32 sum into b_{L-1}[k]), then
-//               W[c][k] -= lr * dW[c][k].
+// accumulation in a fixed order.  One kernel, one thread-block cluster of S CTAs
+// per learner, CTA s owning the input features [s*F, (s+1)*F):
+//   1. partial logits over its features: Zp_s[b][c] = sum_k H[b][k] W_q[c][k]
+//      (k ascending);
+//   2. after a cluster barrier every CTA reads all S partials through distributed
+//      shared memory and adds them in slice order: Z = sum_s Zp_s + b_L, then the
+//      softmax cross-entropy gradient g[b][c] = (softmax(Z[b])_c - [c == y_b]) / B
+//      (recomputed identically in every CTA); the first CTA updates b_L -= lr sum_b g
+//      and writes the loss;
+//   3. one thread per feature k of its slice: with W before its update,
+//      dW[c][k] = sum_b g_q[b][c] H[b][k], dH[b][k] = sum_c g_q[b][c] W_q[c][k],
+//      dZ_{L-1}[b][k] = dH [H > 0] (bf16, fp32 sum into b_{L-1}[k]), then
+//      W[c][k] -= lr * dW[c][k].
 // (_q = rounded to bf16).  The class count is a template parameter so no work is
 // issued for absent classes.  For a one-layer model the input rows are read from X.
 #include <cstdint>
@@ -22,12 +25,10 @@
 namespace ha {
 namespace {
 
-constexpr int kFwdThreads = 512;
-constexpr int kFwdWarps = kFwdThreads / 32;
-constexpr int kKC = 512;                      // input features staged per chunk
-constexpr int kRowsPerWarp = 4;               // B <= 64 = kFwdWarps * kRowsPerWarp
+constexpr int kHeadThreads = 128;
 constexpr int kHeadMaxC = 16;
-constexpr int kBwdCols = 128;                 // features per backward CTA
+constexpr int kHeadClusterMax = 8;
+constexpr int kHeadPad = 8;                   // bf16 row padding (spreads banks)
 
 __device__ __forceinline__ float bf16r(float x) {
   return __bfloat162float(__float2bfloat16_rn(x));
@@ -38,195 +39,187 @@ __device__ __forceinline__ const __nv_bfloat16* head_row(const HeadArgs& a, int 
   return a.H + (static_cast<int64_t>(j) * a.Bn + b) * a.pitch_in;
 }
 
-// C: compile-time class count (0 = runtime count up to kHeadMaxC).
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+// The float at the same shared-memory offset in CTA `rank` of this cluster.
+__device__ __forceinline__ float ld_cluster(const float* p, int rank) {
+  const uint32_t la = static_cast<uint32_t>(__cvta_generic_to_shared(p));
+  uint32_t ra;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(la), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(ra) : "memory");
+  return v;
+}
+
+// Features per CTA: a multiple of 64, at least 128, and at most 8 CTAs per learner.
+__host__ __device__ inline int head_slice(int in) {
+  const int f = ((in + kHeadClusterMax - 1) / kHeadClusterMax + 63) / 64 * 64;
+  return f < 128 ? 128 : f;
+}
+__host__ __device__ inline int head_smem_bytes(int in, int Bn) {
+  return (Bn + kHeadMaxC) * (head_slice(in) + kHeadPad) * 2 + 3 * 64 * kHeadMaxC * 4 + 64 * 4;
+}
+
 template <int CT>
-__global__ void __launch_bounds__(kFwdThreads, 1) k_head_fwd(const HeadArgs a) {
+__global__ void __launch_bounds__(kHeadThreads) k_head(const HeadArgs a) {
   constexpr int CM = CT > 0 ? CT : kHeadMaxC;
   extern __shared__ __align__(16) uint8_t smem[];
   const int C = CT > 0 ? CT : a.C, B = a.B, in = a.in;
-  __nv_bfloat16* wq = reinterpret_cast<__nv_bfloat16*>(smem);                       // [C][in]
-  __nv_bfloat16* hs = wq + static_cast<size_t>(C) * in;                              // [64][kKC]
-  float* rl = reinterpret_cast<float*>(hs + 64 * kKC);                               // [B]
-  float* gsum = rl + 64;                                                             // [64][CM]
-  float* bls = gsum + 64 * CM;                                                       // [CM]
-  int* ys = reinterpret_cast<int*>(bls + CM);                                        // [64]
-  const int j = blockIdx.x, t = threadIdx.x, warp = t >> 5, lane = t & 31;
-  const float* W = a.W + static_cast<int64_t>(j) * a.ld;
+  const int S = gridDim.x, s = blockIdx.x, j = blockIdx.y, t = threadIdx.x;
+  const int F = head_slice(in), FP = F + kHeadPad;
+  const int k0 = s * F, kc = min(F, in - k0);          // kc > 0, a multiple of 64
+  __nv_bfloat16* hs = reinterpret_cast<__nv_bfloat16*>(smem);   // [Bn][FP]  H slice
+  __nv_bfloat16* wq = hs + a.Bn * FP;                           // [16][FP]  W_q slice
+  float* zp = reinterpret_cast<float*>(wq + kHeadMaxC * FP);    // [64][16]  partial logits
+  float* zz = zp + 64 * kHeadMaxC;                              // [64][16]  logits
+  float* gs = zz + 64 * kHeadMaxC;                              // [64][16]  CE gradient
+  float* rl = gs + 64 * kHeadMaxC;                              // [64]      per-sample loss
+  float* W = a.W + static_cast<int64_t>(j) * a.ld;
   float* bL = a.bias + static_cast<int64_t>(j) * a.ld;
-  if (t < B) ys[t] = a.y[static_cast<int64_t>(j) * a.N + (a.t * B + t) % a.N];
-  if (t < C) bls[t] = bL[t];
 
-  for (int e = t * 4; e < C * in; e += kFwdThreads * 4) {
-    const float4 v = *reinterpret_cast<const float4*>(W + e);
-    reinterpret_cast<__nv_bfloat162*>(wq + e)[0] = __floats2bfloat162_rn(v.x, v.y);
-    reinterpret_cast<__nv_bfloat162*>(wq + e)[1] = __floats2bfloat162_rn(v.z, v.w);
+  // ---- 1. stage the slice and form the partial logits
+  const int vpr = kc / 8;                                       // 16-byte vectors per H row
+  for (int idx = t; idx < B * vpr; idx += kHeadThreads) {
+    const int b = idx / vpr, v = idx - b * vpr;
+    *reinterpret_cast<uint4*>(hs + b * FP + v * 8) =
+        *reinterpret_cast<const uint4*>(head_row(a, j, b) + k0 + v * 8);
   }
-  float acc[kRowsPerWarp][CM];
-#pragma unroll
-  for (int r = 0; r < kRowsPerWarp; ++r)
-#pragma unroll
-    for (int c = 0; c < CM; ++c) acc[r][c] = 0.f;
-  for (int k0 = 0; k0 < in; k0 += kKC) {
-    const int kc = min(kKC, in - k0);
-    const int vpr = kc / 8;
-    if (k0 > 0) __syncthreads();
-    for (int idx = t; idx < B * vpr; idx += kFwdThreads) {
-      const int b = idx / vpr, v = idx - b * vpr;
-      *reinterpret_cast<uint4*>(hs + b * kKC + v * 8) =
-          *reinterpret_cast<const uint4*>(head_row(a, j, b) + k0 + v * 8);
+  const int wpr = kc / 4;                                       // float4s per W row
+  for (int idx = t; idx < C * wpr; idx += kHeadThreads) {
+    const int c = idx / wpr, v = idx - c * wpr;
+    const float4 w = *reinterpret_cast<const float4*>(W + static_cast<int64_t>(c) * in + k0 + v * 4);
+    __nv_bfloat162* d = reinterpret_cast<__nv_bfloat162*>(wq + c * FP + v * 4);
+    d[0] = __floats2bfloat162_rn(w.x, w.y);
+    d[1] = __floats2bfloat162_rn(w.z, w.w);
+  }
+  __syncthreads();
+  for (int pr = t; pr < B * C; pr += kHeadThreads) {
+    const int b = pr / C, c = pr - b * C;
+    const __nv_bfloat162* hp = reinterpret_cast<const __nv_bfloat162*>(hs + b * FP);
+    const __nv_bfloat162* wp = reinterpret_cast<const __nv_bfloat162*>(wq + c * FP);
+    float acc = 0.f;
+    for (int k = 0; k < kc / 2; ++k) {
+      const float2 h = __bfloat1622float2(hp[k]), w = __bfloat1622float2(wp[k]);
+      acc = fmaf(h.y, w.y, fmaf(h.x, w.x, acc));
     }
-    __syncthreads();
-    for (int kk = 2 * lane; kk < kc; kk += 64) {
-      float2 hv[kRowsPerWarp];
+    zp[b * kHeadMaxC + c] = acc;
+  }
+  cluster_sync();
+
+  // ---- 2. full logits (partials added in slice order), bias read before its update
+  for (int pr = t; pr < B * C; pr += kHeadThreads) {
+    const int b = pr / C, c = pr - b * C;
+    float z = 0.f;
+    for (int r = 0; r < S; ++r) z = __fadd_rn(z, ld_cluster(zp + b * kHeadMaxC + c, r));
+    zz[b * kHeadMaxC + c] = __fadd_rn(z, bL[c]);
+  }
+  cluster_sync();   // every CTA is done with the partials and with b_L
+  if (t < B) {
+    const float* z = zz + t * kHeadMaxC;
+    const int yb = a.y[static_cast<int64_t>(j) * a.N + (a.t * B + t) % a.N];
+    float m = -INFINITY;
 #pragma unroll
-      for (int r = 0; r < kRowsPerWarp; ++r) {
-        const int b = warp + r * kFwdWarps;
-        hv[r] = b < B ? __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(hs + b * kKC + kk))
-                      : make_float2(0.f, 0.f);
-      }
+    for (int c = 0; c < CM; ++c)
+      if (CT > 0 || c < C) m = fmaxf(m, z[c]);
+    float e[CM], sum = 0.f;
+#pragma unroll
+    for (int c = 0; c < CM; ++c) {
+      e[c] = (CT > 0 || c < C) ? expf(z[c] - m) : 0.f;
+      sum += e[c];
+    }
+    const float fB = static_cast<float>(B);
+#pragma unroll
+    for (int c = 0; c < CM; ++c)
+      if (CT > 0 || c < C)
+        gs[t * kHeadMaxC + c] = __fdiv_rn(__fsub_rn(__fdiv_rn(e[c], sum), c == yb ? 1.f : 0.f), fB);
+    rl[t] = logf(sum) + m - z[yb];
+  }
+  __syncthreads();
+  if (s == 0) {
+    if (t < C) {
+      float db = 0.f;
+      for (int b = 0; b < B; ++b) db = __fadd_rn(db, gs[b * kHeadMaxC + t]);
+      bL[t] = __fsub_rn(bL[t], __fmul_rn(a.lr, db));
+    } else if (t == 32) {
+      float l = 0.f;
+      for (int b = 0; b < B; ++b) l += rl[b];
+      a.loss[j] = l / B;
+    }
+  }
+
+  // ---- 3. backward of the slice, one thread per feature
+  for (int kk = t; kk < kc; kk += kHeadThreads) {
+    const int k = k0 + kk;
+    float w32[CM], wk[CM], dw[CM];
+#pragma unroll
+    for (int c = 0; c < CM; ++c) {
+      w32[c] = (CT > 0 || c < C) ? W[static_cast<int64_t>(c) * in + k] : 0.f;
+      wk[c] = bf16r(w32[c]);
+      dw[c] = 0.f;
+    }
+    float db = 0.f;
+    for (int b = 0; b < B; ++b) {
+      const float h = __bfloat162float(hs[b * FP + kk]);
+      float dh = 0.f;
 #pragma unroll
       for (int c = 0; c < CM; ++c) {
         if (CT > 0 || c < C) {
-          const float2 wv =
-              __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(wq + c * in + k0 + kk));
-#pragma unroll
-          for (int r = 0; r < kRowsPerWarp; ++r)
-            acc[r][c] = fmaf(hv[r].y, wv.y, fmaf(hv[r].x, wv.x, acc[r][c]));
+          const float g = bf16r(gs[b * kHeadMaxC + c]);
+          dw[c] = fmaf(g, h, dw[c]);
+          dh = fmaf(g, wk[c], dh);
         }
       }
-    }
-  }
-  const float fB = static_cast<float>(B);
-#pragma unroll
-  for (int r = 0; r < kRowsPerWarp; ++r) {
-    const int b = warp + r * kFwdWarps;
-    if (b >= B) continue;                       // warp-uniform
-#pragma unroll
-    for (int c = 0; c < CM; ++c) {
-      if (CT > 0 || c < C) {
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) acc[r][c] += __shfl_xor_sync(0xffffffffu, acc[r][c], off);
+      if (a.has_dx) {
+        const float dz = h > 0.f ? dh : 0.f;
+        db = __fadd_rn(db, dz);
+        a.dz_prev[(static_cast<int64_t>(j) * a.Bn + b) * a.pitch_in + k] = __float2bfloat16_rn(dz);
       }
     }
-    float z = -INFINITY;
 #pragma unroll
     for (int c = 0; c < CM; ++c)
-      if (c == lane && (CT > 0 || c < C)) z = __fadd_rn(acc[r][c], bls[c]);
-    float m = z;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-    const float e = lane < C ? expf(z - m) : 0.f;
-    float s = e;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    const int yb = ys[b];
-    const float zy = __shfl_sync(0xffffffffu, z, yb & 31);
-    if (lane < C) {
-      const float p = __fdiv_rn(e, s);
-      const float g = __fdiv_rn(__fsub_rn(p, lane == yb ? 1.f : 0.f), fB);
-      gsum[b * CM + lane] = g;
-      a.gq[(static_cast<int64_t>(j) * a.Bn + b) * kHeadMaxC + lane] = bf16r(g);
+      if (CT > 0 || c < C) W[static_cast<int64_t>(c) * in + k] = __fsub_rn(w32[c], __fmul_rn(a.lr, dw[c]));
+    if (a.has_dx) {
+      float* bp = a.bias_prev + static_cast<int64_t>(j) * a.ld + k;
+      *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
     }
-    if (lane == 0) rl[b] = logf(s) + m - zy;
-  }
-  __syncthreads();
-  if (t < C) {
-    float db = 0.f;
-    for (int b = 0; b < B; ++b) db = __fadd_rn(db, gsum[b * CM + t]);
-    bL[t] = __fsub_rn(bls[t], __fmul_rn(a.lr, db));
-  }
-  if (t == 0) {
-    float l = 0.f;
-    for (int b = 0; b < B; ++b) l += rl[b];
-    a.loss[j] = l / B;
   }
 }
 
 template <int CT>
-__global__ void __launch_bounds__(kBwdCols) k_head_bwd(const HeadArgs a) {
-  constexpr int CM = CT > 0 ? CT : kHeadMaxC;
-  __shared__ float gq[64 * kHeadMaxC];
-  const int C = CT > 0 ? CT : a.C, B = a.B, in = a.in;
-  const int j = blockIdx.y, t = threadIdx.x, k = blockIdx.x * kBwdCols + t;
-  for (int e = t; e < B * kHeadMaxC; e += kBwdCols)
-    gq[e] = a.gq[static_cast<int64_t>(j) * a.Bn * kHeadMaxC + e];
-  __syncthreads();
-  if (k >= in) return;
-  float* W = a.W + static_cast<int64_t>(j) * a.ld;
-  float w32[CM], wk[CM], dw[CM];
-#pragma unroll
-  for (int c = 0; c < CM; ++c) {
-    w32[c] = (CT > 0 || c < C) ? W[c * in + k] : 0.f;
-    wk[c] = bf16r(w32[c]);
-    dw[c] = 0.f;
-  }
-  float db = 0.f;
-  for (int b0 = 0; b0 < a.Bn; b0 += 8) {
-    float h[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q)
-      h[q] = b0 + q < B ? __bfloat162float(head_row(a, j, b0 + q)[k]) : 0.f;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int b = b0 + q;
-      if (b < B) {
-        float dh = 0.f;
-#pragma unroll
-        for (int c = 0; c < CM; ++c) {
-          if (CT > 0 || c < C) {
-            const float g = gq[b * kHeadMaxC + c];
-            dw[c] = fmaf(g, h[q], dw[c]);
-            dh = fmaf(g, wk[c], dh);
-          }
-        }
-        if (a.has_dx) {
-          const float dz = h[q] > 0.f ? dh : 0.f;
-          db = __fadd_rn(db, dz);
-          a.dz_prev[(static_cast<int64_t>(j) * a.Bn + b) * a.pitch_in + k] = __float2bfloat16_rn(dz);
-        }
-      }
-    }
-  }
-#pragma unroll
-  for (int c = 0; c < CM; ++c)
-    if (CT > 0 || c < C) W[c * in + k] = __fsub_rn(w32[c], __fmul_rn(a.lr, dw[c]));
-  if (a.has_dx) {
-    float* bp = a.bias_prev + static_cast<int64_t>(j) * a.ld + k;
-    *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
-  }
-}
-
-int fwd_smem_bytes(int C, int in) {
-  return C * in * 2 + 64 * kKC * 2 + 64 * 4 + 64 * kHeadMaxC * 4 + kHeadMaxC * 4 + 64 * 4;
-}
-
-template <int CT>
-cudaError_t launch_pair(const HeadArgs& a, int P, cudaStream_t s) {
-  k_head_fwd<CT><<<P, kFwdThreads, fwd_smem_bytes(a.C, a.in), s>>>(a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  dim3 grid((a.in + kBwdCols - 1) / kBwdCols, P);
-  k_head_bwd<CT><<<grid, kBwdCols, 0, s>>>(a);
-  return cudaGetLastError();
+cudaError_t launch_cluster(const HeadArgs& a, int P, cudaStream_t s) {
+  const int S = (a.in + head_slice(a.in) - 1) / head_slice(a.in);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(S, P);
+  cfg.blockDim = dim3(kHeadThreads);
+  cfg.dynamicSmemBytes = head_smem_bytes(a.in, a.Bn);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_head<CT>, a);
 }
 
 }  // namespace
 
-int head_scratch_floats(int P, int Bn) { return P * Bn * kHeadMaxC; }
-
 bool head_supported(int C, int in, int B) {
-  return C <= kHeadMaxC && in % 64 == 0 && B <= 64 && fwd_smem_bytes(C, in) <= 200 * 1024;
+  return C <= kHeadMaxC && in % 64 == 0 && B <= 64 && head_smem_bytes(in, 64) <= 200 * 1024;
 }
 
 cudaError_t head_configure() {
-  cudaError_t e = cudaFuncSetAttribute(k_head_fwd<10>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(k_head<10>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        200 * 1024);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_head_fwd<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  return cudaFuncSetAttribute(k_head<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
 }
 
 cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s) {
-  return a.C == 10 ? launch_pair<10>(a, P, s) : launch_pair<0>(a, P, s);
+  return a.C == 10 ? launch_cluster<10>(a, P, s) : launch_cluster<0>(a, P, s);
 }
 
 }  // namespace ha

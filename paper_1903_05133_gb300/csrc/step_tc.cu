@@ -4,27 +4,19 @@
 // forward Z_l = H_{l-1} W_l^T + b_l, softmax cross-entropy gradient, backward
 // dH_{l-1} = dZ_l W_l (with W_l before its update) and W_l -= lr * dZ_l^T H_{l-1}.
 // The fp32 master weights W_l [P][out][in] are streamed from HBM by TMA and
-// rounded to bf16 in shared memory by the CTA itself; MMAs accumulate in fp32 in
-// tensor memory.  All operands use the K-major 128-byte-swizzle layout.
+// rounded to bf16 by the CTA itself into tensor memory; MMAs accumulate in fp32 in
+// tensor memory.  Activations exist once, batch-major ([Bn][features], 128-byte
+// swizzled tiles): the forward reads them K-major, the backward's dW MMA MN-major.
 //
 // Because the per-learner batch B (<= 64) is far below the MMA's M, every GEMM
 // is issued "swap-AB": the weight tile supplies M = 128 rows and the batch is
-// the N extent.
-//
-// Forward kernel  (grid: out tiles of 128 x P learners)
-//   warp 4: TMA producer - fp32 W tile [128 x 64] + bf16 H tile [Bn x 64] per stage
-//   warps 0-3: round W to bf16 into the swizzled A tile; then the epilogue
-//              (bias, ReLU, bf16 H and H^T of the next layer, or fp32 logits)
-//   warp 5: TMEM allocation + single-thread MMA issue, Z^T[128 x Bn] += W H^T
-// Backward kernel (grid: in tiles of 128 x P learners), one pass over W_l:
-//   per out-chunk of 64 rows: TMA loads fp32 W [64 x 128], dZ [Bn x 64],
-//   dZ^T [64 x 64]; warps 0-3 write W^T (bf16) for the dX MMA; MMA warp issues
-//     dH^T[128 x Bn] += W^T(chunk) dZ^T(chunk)          (accumulated over chunks)
-//     dW^T[128 x 64]  = H^T[128 x B] dZ(chunk)           (double-buffered in TMEM)
-//   warps 0-3 then update the fp32 chunk in shared memory (w - lr * dw, separate
-//   rounded multiply and subtract) and TMA-store it back: W is read once and
-//   written once per step.  Finally dZ_{l-1} = dH * [H_{l-1} > 0] and the bias
-//   b_{l-1} -= lr * sum_b dZ_{l-1}.
+// the N extent.  Both kernels are persistent stream-K kernels (one CTA per SM):
+//   forward:  unit = 128 output features x 64 inputs of one learner;
+//             Z^T[128 x Bn] += W_q H^T, epilogue bias + ReLU (or fused softmax-CE);
+//   backward: unit = 128 input features x 64 output rows of one learner;
+//             dW^T = H^T dZ, the fp32 update of W, and dH^T += W_q^T dZ^T;
+//             epilogue dZ_{l-1} = dH [H_{l-1} > 0], b_{l-1} -= lr sum_b dZ_{l-1}.
+// W is read once by the forward and once (read, written) by the backward.
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -48,7 +40,10 @@ namespace {
 // Warps 0-7 convert the fp32 weight tiles to bf16 and own the accumulator rows:
 // warp w serves TMEM lanes 32*(w%4).., converts K half w/4 of those 32 rows, and
 // the two warps on the same lanes split the batch columns in interleaved 16-column
-// blocks (group w/4 takes blocks 2m + w/4).  Warp 8 issues TMA, warp 9 the MMAs.
+// blocks (group w/4 takes blocks 2m + w/4).  Warp 8 streams the weight tiles,
+// warp 9 issues the MMAs, warp 10 streams the batch tiles and publishes this CTA's
+// split-tile partial.  Every role that waits has a warp of its own: a lane blocked
+// in an mbarrier wait would hold up the other lanes of its warp.
 // The bf16 A tile (128 rows x 64 K) lives in tensor memory, double-buffered, so
 // shared memory holds only the two TMA rings: the fp32 weight tiles (two
 // 128-byte-swizzled 128 x 32 boxes per chunk, released by the converter warps as
@@ -58,7 +53,7 @@ namespace {
 // about 4 us from TMA issue to arrival under full load, so both rings are as deep
 // as shared memory allows.
 constexpr int kFwdConv = 256;
-constexpr int kFwdThreads = kFwdConv + 64;
+constexpr int kFwdThreads = kFwdConv + 96;
 constexpr int kFwdWRingMax = 6, kFwdHRingMax = 8;
 constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile (2 boxes)
 constexpr int kFwdWBox = 128 * 32 * 4;                 // one 128 x 32 fp32 box
@@ -255,39 +250,47 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 8) {
-    // Lane 0 streams the weight tiles, lane 1 the batch tiles: each ring runs as
-    // far ahead as its own consumer allows.
-    if (lane < 2) {
-      const bool wside = lane == 0;
-      const int n = wside ? nw : nh;
-      uint64_t* fullb = wside ? wfull : hfull;
-      uint64_t* emptyb = wside ? wempty : hempty;
-      if (wside) tma_prefetch_desc(&tm_w);
-      else tma_prefetch_desc(&tm_h);
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_w);
       int issued = 0, tau = tile0, c = c0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-        const int s = i % n;
-        if (i >= n && !mbar_wait(&emptyb[s], ((i / n) - 1) & 1, a.err)) break;
-        if (wside) {
-          mbar_arrive_expect_tx(&fullb[s], kFwdWf32);
-          tma_load_3d(wf(s), &tm_w, &fullb[s], c * 64, ot * 128, j);
-          tma_load_3d(wf(s) + kFwdWBox, &tm_w, &fullb[s], c * 64 + 32, ot * 128, j);
-        } else {
-          mbar_arrive_expect_tx(&fullb[s], a.Bn * 128);
-          tma_load_3d(hb(s), &tm_h, &fullb[s], c * 64, h_row0, j);
-        }
+        const int s = i % nw;
+        if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
+        tma_load_3d(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j);
+        tma_load_3d(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j);
         issued = i + 1;
         if (++c == nk) { c = 0; ++tau; }
       }
       // Every load issued must have landed before the CTA may exit.
-      for (int i = issued - n > 0 ? issued - n : 0; i < issued; ++i)
-        mbar_wait(&fullb[i % n], (i / n) & 1, a.err);
-    } else if (lane == 2 && c0 != 0 && n_local > 0) {
-      // The first tile began in an earlier CTA, which finishes it: once the
-      // converter warps have written this CTA's partial, publish it (release
-      // order makes the partial visible before the count).
-      if (mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+      for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
+        mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
+    }
+  } else if (warp == 10) {
+    if (lane == 0) {
+      // Batch tiles.  Also: if the first tile began in an earlier CTA (which
+      // finishes it), publish this CTA's partial once the converter warps have
+      // written it (release order makes the partial visible before the count).
+      tma_prefetch_desc(&tm_h);
+      bool publish = c0 != 0 && n_local > 0;
+      int issued = 0, tau = tile0, c = c0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.o_tiles;
+        const int s = i % nh;
+        if (publish && mbar_test(pready, 0)) {
+          red_release_add(a.counters + tile0, 1);
+          publish = false;
+        }
+        if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&hfull[s], a.Bn * 128);
+        tma_load_3d(hb(s), &tm_h, &hfull[s], c * 64, h_row0, j);
+        issued = i + 1;
+        if (++c == nk) { c = 0; ++tau; }
+      }
+      for (int i = issued - nh > 0 ? issued - nh : 0; i < issued; ++i)
+        mbar_wait(&hfull[i % nh], (i / nh) & 1, a.err);
+      if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
     }
   } else if (warp == 9) {
     if (lane == 0) {
@@ -502,12 +505,14 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 // finished, as in the forward, by the CTA holding its first chunk.  The tile epilogue
 // applies the ReLU mask of H_{l-1}, writes dZ_{l-1} and updates b_{l-1}.
 // Warps 0-3: thread t owns input feature i0 + t (TMEM lane t): it converts its column
-// of the fp32 chunk to the bf16 A tile, applies the update and runs the epilogue.
-// Warp 4: lane 0 loads W chunks and H tiles, lane 1 dZ tiles, lane 2 issues the TMA
-// stores of updated chunks (and releases their slots once read), lane 3 publishes a
-// split tile's partial.  Warp 5: the MMAs.
+// of the fp32 chunk to the bf16 A tile, applies the update in shared memory and runs
+// the tile epilogue.  Warp 4 loads W chunks and H tiles, warp 5 issues the MMAs, warp
+// 6 loads dZ tiles and publishes a split tile's partial, warp 7 TMA-stores updated
+// chunks (bulk stores: per-thread row stores of the same bytes ran at half the speed)
+// and frees their slots once read.  Each waiting role has a warp of its own: a lane
+// blocked in an mbarrier wait holds up the other lanes of its warp.
 constexpr int kBwdConv = 128;
-constexpr int kBwdThreads = kBwdConv + 64;
+constexpr int kBwdThreads = kBwdConv + 128;
 constexpr int kBwdWf32 = 64 * 128 * 4;                 // 32 KB fp32 W chunk [64 o][128 i]
 constexpr int kBwdWRingMax = 5, kBwdZRingMax = 8;
 constexpr int kBwdSmemMax = 227 * 1024;
@@ -516,7 +521,7 @@ constexpr uint32_t kBwdTmemCols = 512;
 constexpr uint32_t kBwdTmemW = 128, kBwdTmemA = 256;
 
 // Layout: W ring | 2 H tiles (2 x [Bn][64] bf16 each) | dZ ring ([Bn][64] bf16) | barriers.
-__host__ __device__ constexpr int bwd_wring(int Bn) { return Bn <= 32 ? 5 : 4; }
+__host__ __device__ constexpr int bwd_wring(int Bn) { return (void)Bn, 5; }
 __host__ __device__ constexpr int bwd_h_off(int Bn) { return bwd_wring(Bn) * kBwdWf32; }
 __host__ __device__ constexpr int bwd_z_off(int Bn) { return bwd_h_off(Bn) + 2 * 2 * Bn * 128; }
 __host__ __device__ constexpr int bwd_zring(int Bn) {
@@ -526,7 +531,7 @@ __host__ __device__ constexpr int bwd_zring(int Bn) {
 }
 __host__ __device__ constexpr int bwd_bar_off(int Bn) { return bwd_z_off(Bn) + bwd_zring(Bn) * Bn * 128; }
 __host__ __device__ constexpr int bwd_smem(int Bn) { return bwd_bar_off(Bn) + 512 + 1024; }
-static_assert(bwd_zring(64) >= 6 && bwd_zring(48) >= 6 && bwd_zring(32) >= 6 && bwd_zring(16) >= 6 &&
+static_assert(bwd_zring(64) >= 4 && bwd_zring(48) >= 6 && bwd_zring(32) >= 8 && bwd_zring(16) >= 8 &&
                   bwd_smem(64) <= kBwdSmemMax && bwd_smem(48) <= kBwdSmemMax &&
                   bwd_smem(32) <= kBwdSmemMax && bwd_smem(16) <= kBwdSmemMax,
               "backward shared-memory plan");
@@ -629,12 +634,21 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
         mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
       for (int k = kt - 2 > 0 ? kt - 2 : 0; k < kt; ++k) mbar_wait(&hfull[k & 1], (k >> 1) & 1, a.err);
-    } else if (lane == 1) {
+    }
+  } else if (warp == 6) {
+    if (lane == 0) {
+      // dZ tiles; also publishes this CTA's partial of a split first tile (see the
+      // forward).
       tma_prefetch_desc(&tm_dz);
+      bool publish = a.has_dx && c0 != 0 && n_local > 0;
       int issued = 0, tau = tile0, c = c0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.s_tiles;
         const int s = i % nz;
+        if (publish && mbar_test(pready, 0)) {
+          red_release_add(a.counters + tile0, 1);
+          publish = false;
+        }
         if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) break;
         mbar_arrive_expect_tx(&zfull[s], tbytes);
         tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j);
@@ -643,22 +657,28 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       }
       for (int i = issued - nz > 0 ? issued - nz : 0; i < issued; ++i)
         mbar_wait(&zfull[i % nz], (i / nz) & 1, a.err);
-    } else if (lane == 2) {
-      // Store each updated chunk; its slot is released once the TMA has read it.
-      int tau = tile0, c = c0;
+      if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+    }
+  } else if (warp == 7) {
+    if (lane == 0) {
+      // Store each updated chunk; its slot is released once the TMA has read it
+      // (two stores in flight).
+      int tau = tile0, c = c0, stored = 0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.s_tiles, i0 = (tau - j * a.s_tiles) * 128;
         const int s = i % nw;
         if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
         tma_store_3d(&tm_w, wf(s), i0, c * 64, j);
         tma_store_commit();
-        tma_store_wait_read_all();
-        mbar_arrive(&wempty[s]);
+        stored = i + 1;
+        if (i > 0) {
+          tma_store_wait_read_1();
+          mbar_arrive(&wempty[(i - 1) % nw]);
+        }
         if (++c == nc) { c = 0; ++tau; }
       }
       tma_store_wait_all();
-    } else if (lane == 3 && a.has_dx && c0 != 0 && n_local > 0) {
-      if (mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+      if (stored > 0) mbar_arrive(&wempty[(stored - 1) % nw]);
     }
   } else if (warp == 5) {
     if (lane == 0) {
