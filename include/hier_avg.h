@@ -184,6 +184,12 @@ int hier_avg_check(hier_avg* h);
 #define HA_KERNEL_KINDS         7
 int hier_avg_profile(hier_avg* h, int enable);
 
+/* The same for a subset: kinds is a bitmask of (1 << HA_KERNEL_*); 0 stops.
+ * Each timed launch costs two event records that separate it from its
+ * neighbours on the stream, so a throughput measurement times only the kinds it
+ * reports.  HA_EINVAL for bits beyond HA_KERNEL_KINDS. */
+int hier_avg_profile_kinds(hier_avg* h, unsigned kinds);
+
 /* Synchronise and read kind's totals since profiling was enabled: summed event
  * time in ms, number of launches, and the algorithmic bytes moved by them. */
 int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* launches,

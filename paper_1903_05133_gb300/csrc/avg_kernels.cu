@@ -15,6 +15,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace ha {
 namespace {
@@ -59,6 +60,7 @@ __device__ __forceinline__ void store_rows(V* p, int64_t ld_v, int n, V m) {
 template <int LOG>
 __global__ void __launch_bounds__(256) k_mean_pow2(float4* __restrict__ w, int64_t ld_v,
                                                    int64_t cols_v) {
+  grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   float4* p = w + static_cast<int64_t>(blockIdx.y) * (int64_t(1) << LOG) * ld_v + c;
@@ -74,6 +76,7 @@ __global__ void __launch_bounds__(256) k_mean_pow2(float4* __restrict__ w, int64
 template <int LOGS, int LOGG>
 __global__ void __launch_bounds__(256) k_local_global_pow2(float4* __restrict__ w,
                                                            int64_t ld_v, int64_t cols_v) {
+  grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   constexpr int S = 1 << LOGS, G = 1 << LOGG;
@@ -126,6 +129,7 @@ __device__ V tree_any(const V* __restrict__ p, int64_t ld_v, int n) {
 template <class V>
 __global__ void __launch_bounds__(256) k_mean_any(V* __restrict__ w, int64_t ld_v,
                                                   int64_t cols_v, int n) {
+  grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   V* p = w + static_cast<int64_t>(blockIdx.y) * n * ld_v + c;
@@ -136,6 +140,7 @@ __global__ void __launch_bounds__(256) k_mean_any(V* __restrict__ w, int64_t ld_
 template <class V>
 __global__ void __launch_bounds__(256) k_local_global_any(V* __restrict__ w, int64_t ld_v,
                                                           int64_t cols_v, int S, int G) {
+  grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   V* p = w + c;
@@ -180,7 +185,7 @@ void launch_mean_pow2(float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
                       cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
             static_cast<unsigned>(groups));
-  k_mean_pow2<LOG><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v);
+  launch_pdl(k_mean_pow2<LOG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v);
 }
 
 bool mean_pow2_dispatch(int log, float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
@@ -200,7 +205,7 @@ bool mean_pow2_dispatch(int log, float4* w, int64_t ld_v, int64_t cols_v, int64_
 template <int LOGS, int LOGG>
 void launch_lg(float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
-  k_local_global_pow2<LOGS, LOGG><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v);
+  launch_pdl(k_local_global_pow2<LOGS, LOGG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v);
 }
 
 template <int LOGS>
@@ -231,13 +236,13 @@ void launch_mean_any(V* w, int64_t ld_v, int64_t cols_v, int n, int64_t groups,
                      cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
             static_cast<unsigned>(groups));
-  k_mean_any<V><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v, n);
+  launch_pdl(k_mean_any<V>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, n);
 }
 
 template <class V>
 void launch_lg_any(V* w, int64_t ld_v, int64_t cols_v, int S, int G, cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
-  k_local_global_any<V><<<grid, kThreads, 0, s>>>(w, ld_v, cols_v, S, G);
+  launch_pdl(k_local_global_any<V>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, S, G);
 }
 
 }  // namespace

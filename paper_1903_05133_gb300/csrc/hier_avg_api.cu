@@ -82,7 +82,7 @@ struct hier_avg {
   CUtensorMap tm_x;                           // X [P][N][d_0] as the first layer's batch tile
   int64_t t = 0;
   // profiling
-  bool prof = false;
+  unsigned prof = 0;                          // kinds timed: bit (1 << HA_KERNEL_*)
   std::vector<ProfRec> recs;
   std::vector<cudaEvent_t> pool;
   size_t pool_used = 0;
@@ -118,14 +118,15 @@ struct hier_avg {
   template <class F>
   int timed(int kind, double bytes, F&& launch, const char* what) {
     cudaEvent_t a = nullptr, b = nullptr;
-    if (prof) {
+    const bool on = (prof >> kind) & 1u;
+    if (on) {
       a = ev();
       b = ev();
       if (a && b) cudaEventRecord(a, stream);
     }
     const cudaError_t e = launch();
     if (e != cudaSuccess) return cuda(e, what);
-    if (prof && a && b) {
+    if (on && a && b) {
       cudaEventRecord(b, stream);
       recs.push_back({kind, a, b, bytes});
     }
@@ -693,13 +694,18 @@ int hier_avg_check(hier_avg* h) {
   return HA_OK;
 }
 
-int hier_avg_profile(hier_avg* h, int enable) {
+int hier_avg_profile_kinds(hier_avg* h, unsigned kinds) {
   if (!h) return HA_EINVAL;
+  if (kinds >> HA_KERNEL_KINDS) return h->fail(HA_EINVAL, "profile: unknown kernel kind bit");
   if (h->bound) cudaStreamSynchronize(h->stream);
   h->recs.clear();
   h->pool_used = 0;
-  h->prof = enable != 0;
+  h->prof = kinds;
   return HA_OK;
+}
+
+int hier_avg_profile(hier_avg* h, int enable) {
+  return hier_avg_profile_kinds(h, enable ? (1u << HA_KERNEL_KINDS) - 1 : 0u);
 }
 
 int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* launches,

@@ -89,6 +89,15 @@ __device__ __forceinline__ bool spin_acquire_eq(const int* p, int want, int* err
   }
 }
 
+// ------------------------------------------------ programmatic dependent launch
+// A kernel launched with programmatic stream serialization is launched while the
+// previous kernel of the stream drains and may run its prologue on SMs that kernel
+// has released; it must call grid_dep_wait() before touching any global memory
+// that kernel reads or writes.  (The dependents are released when this grid
+// completes: releasing them earlier measured slower, since they then take SM
+// resources the rest of this grid needs.)  A no-op for an ordinary launch.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- fences
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");

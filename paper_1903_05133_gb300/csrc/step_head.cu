@@ -21,6 +21,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace ha {
 namespace {
@@ -66,6 +67,7 @@ template <int CT>
 __global__ void __launch_bounds__(kHeadThreads) k_head(const HeadArgs a) {
   constexpr int CM = CT > 0 ? CT : kHeadMaxC;
   extern __shared__ __align__(16) uint8_t smem[];
+  grid_dep_wait();
   const int C = CT > 0 ? CT : a.C, B = a.B, in = a.in;
   const int S = gridDim.x, s = blockIdx.x, j = blockIdx.y, t = threadIdx.x;
   const int F = head_slice(in), FP = F + kHeadPad;
@@ -190,19 +192,8 @@ __global__ void __launch_bounds__(kHeadThreads) k_head(const HeadArgs a) {
 template <int CT>
 cudaError_t launch_cluster(const HeadArgs& a, int P, cudaStream_t s) {
   const int S = (a.in + head_slice(a.in) - 1) / head_slice(a.in);
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(S, P);
-  cfg.blockDim = dim3(kHeadThreads);
-  cfg.dynamicSmemBytes = head_smem_bytes(a.in, a.Bn);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = S;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_head<CT>, a);
+  return launch_pdl(k_head<CT>, dim3(S, P), dim3(kHeadThreads), head_smem_bytes(a.in, a.Bn), s,
+                    false, S, a);
 }
 
 }  // namespace

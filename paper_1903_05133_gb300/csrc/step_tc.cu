@@ -248,6 +248,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  grid_dep_wait();                       // the previous kernel's results are visible
 
   if (warp == 8) {
     if (lane == 0) {
@@ -443,7 +444,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         const int o = ot * 128 + r;
         tbias = o < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
       }
-      const int sw = i % nw, sh = i % nh, bb = i & 1;
+      const int sw = i % nw, bb = i & 1;
       if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
       if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
       tc_fence_after();
@@ -606,6 +607,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  grid_dep_wait();                       // the previous kernel's results are visible
 
   if (warp == 4) {
     if (lane == 0) {
@@ -892,6 +894,7 @@ __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __rest
                                                     int64_t N, int d0, int B, int Bn,
                                                     int pitch0, int64_t t,
                                                     __nv_bfloat16* __restrict__ H0) {
+  grid_dep_wait();
   const int j = blockIdx.y, k0 = blockIdx.x * 64;
   const int nvec = B * 8;                       // 16-byte vectors in the [B][64] slice
   for (int idx = threadIdx.x; idx < nvec; idx += blockDim.x) {
@@ -920,6 +923,7 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
                                                            __nv_bfloat16* dZ, float* loss) {
   __shared__ float row_max[64], row_sum[64], row_loss[64];
   __shared__ int row_y[64];
+  grid_dep_wait();
   const int j = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float* Zj = Z + static_cast<int64_t>(j) * B * C;
   for (int b = warp; b < B; b += kXentThreads / 32) {
@@ -978,49 +982,30 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
   (void)P;
   // Cooperative: the finisher of a split tile waits for the other contributors,
   // so every CTA of the grid must be resident at once (the launch fails otherwise).
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.ctas);
-  cfg.blockDim = dim3(kFwdThreads);
-  cfg.dynamicSmemBytes = fwd_smem(a.mode, a.Bn);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_tc_forward, w_fwd, h_in, a);
+  return launch_pdl(k_tc_forward, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s, true,
+                    1, w_fwd, h_in, a);
 }
 
 cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
                                const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s) {
   (void)P;
   // Cooperative for the same reason as the forward (split dX tiles).
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.ctas);
-  cfg.blockDim = dim3(kBwdThreads);
-  cfg.dynamicSmemBytes = bwd_smem(a.Bn);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_tc_backward, w_bwd, h_in, dz, a);
+  return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, true, 1,
+                    w_bwd, h_in, dz, a);
 }
 
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
                                int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s) {
   dim3 grid((d0 + 63) / 64, P);
-  k_gather_bf16<<<grid, 256, 0, s>>>(X, N, d0, B, Bn, pitch0, t, H0);
-  return cudaGetLastError();
+  return launch_pdl(k_gather_bf16, grid, dim3(256), 0, s, false, 1, X, N, d0, B, Bn, pitch0, t, H0);
 }
 
 cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
                              int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
                              __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s) {
   dim3 grid(P, (C + kXentThreads - 1) / kXentThreads);
-  k_xent_bf16<<<grid, kXentThreads, 0, s>>>(Z, y, N, t, B, Bn, C, pitch_c, lr, bias_L, ld, dZ, loss);
-  return cudaGetLastError();
+  return launch_pdl(k_xent_bf16, grid, dim3(kXentThreads), 0, s, false, 1, Z, y, N, t, B, Bn, C,
+                    pitch_c, lr, bias_L, ld, dZ, loss);
 }
 
 }  // namespace ha

@@ -171,8 +171,16 @@ class HierAvg:
     def check(self) -> None:
         check(self._lib.hier_avg_check(self.h), "check", self.h)
 
-    def profile(self, enable: bool) -> None:
-        check(self._lib.hier_avg_profile(self.h, 1 if enable else 0), "profile", self.h)
+    def profile(self, enable) -> None:
+        """Start (and clear) kernel timing: True for every kind, an iterable of kind
+        names for a subset; False stops it."""
+        if isinstance(enable, bool) or enable is None:
+            check(self._lib.hier_avg_profile(self.h, 1 if enable else 0), "profile", self.h)
+            return
+        mask = 0
+        for k in enable:
+            mask |= 1 << KERNEL_KINDS[k]
+        check(self._lib.hier_avg_profile_kinds(self.h, mask), "profile", self.h)
 
     def profile_read(self, kind: str) -> Tuple[float, int, float]:
         ms, n, by = c_double(), c_int64(), c_double()
