@@ -68,6 +68,7 @@ struct hier_avg {
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
   std::vector<int> bwd_ctas, bwd_tiles;       // per layer: stream-K CTAs, input slices
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
+  bool w_stream = true;                       // parameters exceed L2: stream W evict-first
   bool head = false;                          // d_L <= 16: fused last-layer kernel
   // binding
   bool bound = false;
@@ -224,6 +225,13 @@ int make_map(hier_avg* h, CUtensorMap* m, CUtensorMapDataType dt, void* base, ui
 
 int build_maps(hier_avg* h) {
   const int L = h->L;
+  // When all learners' parameters fit in L2, the backward re-reads what the
+  // forward just read and the next step what the backward wrote, so W keeps the
+  // normal L2 policy; otherwise it is marked evict-first so that it does not push
+  // the small, re-read activation tiles out of L2.
+  int l2 = 0;
+  if (cudaDeviceGetAttribute(&l2, cudaDevAttrL2CacheSize, h->device) != cudaSuccess) l2 = 0;
+  h->w_stream = static_cast<double>(h->P) * h->ld * 4 > static_cast<double>(l2);
   h->tm_wf.resize(L);
   h->tm_wb.resize(L);
   h->tm_h.resize(L);
@@ -314,6 +322,7 @@ int do_step(hier_avg* h) {
       a.part = h->wsp<float>(h->off_part);
       a.counters = h->wsp<int>(h->off_cnt);
       a.x_direct = (l == 0 && x_direct) ? 1 : 0;
+      a.w_stream = h->w_stream ? 1 : 0;
       a.x_row0 = static_cast<int>(r0);
       if (l + 1 < L) {
         a.mode = 0;
@@ -391,6 +400,7 @@ int do_step(hier_avg* h) {
       // the forward read them there too.
       const bool from_x = l == 0 && x_direct;
       a.h_row0 = from_x ? static_cast<int>(r0) : 0;
+      a.w_stream = h->w_stream ? 1 : 0;
       a.ctas = h->bwd_ctas[l];
       a.s_tiles = h->bwd_tiles[l];
       a.n_tiles = h->bwd_tiles[l] * P;

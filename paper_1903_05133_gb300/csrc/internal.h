@@ -78,6 +78,7 @@ struct TcFwdArgs {
   int* counters;
   // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)
   int x_direct, x_row0;
+  int w_stream;               // load W with the L2 evict-first policy
   // mode 2: labels and outputs of the fused cross-entropy
   const int32_t* y;
   int64_t N, t;
@@ -95,6 +96,7 @@ struct TcBwdArgs {
   __nv_bfloat16* dz_prev;     // dZ_{l-1} [P][Bn][pitch_in]
   int pitch_in;
   int h_row0;                 // first batch row of H_{l-1} in its tensor map (X rows for l = 0)
+  int w_stream;               // load and store W with the L2 evict-first policy
   // persistent stream-K schedule over n_tiles = P x ceil(in/128) tiles x ceil(out/64)
   // chunks, same partial/counter protocol as the forward
   int ctas, n_tiles, s_tiles;

@@ -253,14 +253,15 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   if (warp == 8) {
     if (lane == 0) {
       tma_prefetch_desc(&tm_w);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
       int issued = 0, tau = tile0, c = c0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
         const int s = i % nw;
         if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) break;
         mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
-        tma_load_3d(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j);
-        tma_load_3d(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j);
+        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j, stream);
+        tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j, stream);
         issued = i + 1;
         if (++c == nk) { c = 0; ++tau; }
       }
@@ -614,6 +615,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       // W chunks, and each tile's H tile (two 64-feature boxes) ahead of its first chunk
       tma_prefetch_desc(&tm_w);
       tma_prefetch_desc(&tm_h);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
       int issued = 0, tau = tile0, c = c0, kt = 0;
       bool ok = true;
       for (int i = 0; i < n_local && ok; ++i) {
@@ -629,7 +631,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         const int s = i % nw;
         if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
         mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
-        tma_load_3d(wf(s), &tm_w, &wfull[s], i0, c * 64, j);
+        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], i0, c * 64, j, stream);
         issued = i + 1;
         if (++c == nc) { c = 0; ++tau; }
       }
@@ -665,12 +667,13 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     if (lane == 0) {
       // Store each updated chunk; its slot is released once the TMA has read it
       // (two stores in flight).
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
       int tau = tile0, c = c0, stored = 0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.s_tiles, i0 = (tau - j * a.s_tiles) * 128;
         const int s = i % nw;
         if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
-        tma_store_3d(&tm_w, wf(s), i0, c * 64, j);
+        tma_store_3d_hint(&tm_w, wf(s), i0, c * 64, j, stream);
         tma_store_commit();
         stored = i + 1;
         if (i > 0) {
