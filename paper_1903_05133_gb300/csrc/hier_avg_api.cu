@@ -66,6 +66,7 @@ struct hier_avg {
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
+  std::vector<int> fwd_cq;                    // per layer: cluster split factor (1 = stream-K)
   std::vector<int> bwd_ctas, bwd_tiles;       // per layer: stream-K CTAs, input slices
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
   bool w_stream = true;                       // parameters exceed L2: stream W evict-first
@@ -176,6 +177,7 @@ int plan_layout(hier_avg* h) {
     // 64-input chunks; backward tile = 128 inputs x 64-output chunks.
     h->fwd_ctas.assign(L, 1);
     h->fwd_tiles.assign(L, 1);
+    h->fwd_cq.assign(L, 1);
     h->bwd_ctas.assign(L, 1);
     h->bwd_tiles.assign(L, 1);
     int64_t part_bytes = 16, max_tiles = 1;
@@ -184,6 +186,15 @@ int plan_layout(hier_avg* h) {
       const int64_t ftiles = (out + 127) / 128, btiles = (in + 127) / 128;
       h->fwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, ftiles * P * ((in + 63) / 64)));
       h->fwd_tiles[l] = static_cast<int>(ftiles);
+      // Few tiles: a cluster of cq CTAs per tile, reduced through distributed shared
+      // memory (the stream-K fix-up through global memory costs a few microseconds of
+      // latency at the end, which is a large share of a short layer).
+      const int64_t nk = (in + 63) / 64;
+      const int64_t cq = std::min<int64_t>(std::min<int64_t>(8, nk), kTargetCtas / (ftiles * P));
+      if (cq >= 2) {
+        h->fwd_cq[l] = static_cast<int>(cq);
+        h->fwd_ctas[l] = static_cast<int>(ftiles * P * cq);
+      }
       h->bwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, btiles * P * ((out + 63) / 64)));
       h->bwd_tiles[l] = static_cast<int>(btiles);
       part_bytes = std::max(part_bytes, int64_t(std::max(h->fwd_ctas[l], h->bwd_ctas[l])) * 128 * h->Bn * 4);
@@ -317,6 +328,7 @@ int do_step(hier_avg* h) {
       a.ld = h->ld;
       a.bias = h->params + h->boff[l];
       a.ctas = h->fwd_ctas[l];
+      a.cq = h->fwd_cq[l];
       a.o_tiles = h->fwd_tiles[l];
       a.n_tiles = h->fwd_tiles[l] * P;
       a.part = h->wsp<float>(h->off_part);

@@ -74,6 +74,7 @@ struct TcFwdArgs {
   // part [ctas][128][Bn] and bumps counters[tile] (reset to 0 by the finisher), and
   // the finisher adds the partials in CTA order.
   int ctas, n_tiles, o_tiles;
+  int cq;                     // > 1: cluster split-K, ctas = n_tiles * cq (no part/counters)
   float* part;
   int* counters;
   // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)

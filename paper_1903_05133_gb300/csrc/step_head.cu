@@ -96,7 +96,6 @@ __host__ __device__ inline int head_smem_bytes(int in, int Bn) {
 
 template <int CT>
 __global__ void __launch_bounds__(kHeadThreads) k_head(const HeadArgs a) {
-  constexpr int CM = CT > 0 ? CT : kHeadMaxC;
   extern __shared__ __align__(16) uint8_t smem[];
   grid_dep_wait();
   const int C = CT > 0 ? CT : a.C, B = a.B, Bn = a.Bn, in = a.in;

@@ -37,6 +37,11 @@ namespace {
 // boundaries.  A tile whose chunks are spread over several CTAs is finished by
 // the CTA that holds its first chunk (see tile_end) with the partials of the
 // others added in CTA order (deterministic).
+// Small layers (at most 76 tiles, so at least two CTAs per tile) run in cluster
+// split-K mode instead: tile t gets a cluster of cq CTAs, rank k taking chunks
+// [k*nk/cq, (k+1)*nk/cq); at the end ranks 1.. leave their partial in shared
+// memory and rank 0 adds them in rank order through distributed shared memory and
+// runs the epilogue.  No global partials, no waiting on other clusters.
 // Warps 0-7 convert the fp32 weight tiles to bf16 and own the accumulator rows:
 // warp w serves TMEM lanes 32*(w%4).., converts K half w/4 of those 32 rows, and
 // the two warps on the same lanes split the batch columns in interleaved 16-column
@@ -197,7 +202,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   const int g = blockIdx.x, G = gridDim.x;
   const int nk = (a.in + 63) / 64;
   const int U = a.n_tiles * nk;
-  const int u0 = unit_begin(g, U, G), u1 = unit_begin(g + 1, U, G);
+  const int cq = a.cq > 1 ? a.cq : 1, part = g % cq;       // cluster split-K rank
+  const int u0 = cq > 1 ? (g / cq) * nk + part * nk / cq : unit_begin(g, U, G);
+  const int u1 = cq > 1 ? (g / cq) * nk + (part + 1) * nk / cq : unit_begin(g + 1, U, G);
   const int n_local = u1 - u0;
   const int nw = fwd_wring(a.mode, a.Bn), nh = fwd_hring(a.mode, a.Bn);
   const int hbytes = a.Bn * 128;
@@ -269,13 +276,17 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
         mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
     }
+    if (cq > 1) {
+      cluster_sync_all();   // the two barriers of the cluster reduction (see below)
+      cluster_sync_all();
+    }
   } else if (warp == 10) {
     if (lane == 0) {
       // Batch tiles.  Also: if the first tile began in an earlier CTA (which
       // finishes it), publish this CTA's partial once the converter warps have
       // written it (release order makes the partial visible before the count).
       tma_prefetch_desc(&tm_h);
-      bool publish = c0 != 0 && n_local > 0;
+      bool publish = cq == 1 && c0 != 0 && n_local > 0;
       int issued = 0, tau = tile0, c = c0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.o_tiles;
@@ -293,6 +304,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       for (int i = issued - nh > 0 ? issued - nh : 0; i < issued; ++i)
         mbar_wait(&hfull[i % nh], (i / nh) & 1, a.err);
       if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
     }
   } else if (warp == 9) {
     if (lane == 0) {
@@ -322,6 +337,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       }
       tc_commit(done);
       mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
     }
   } else {
     // ---- warps 0-7: fp32 -> bf16 A tile (and H_0^T for the first layer), the
@@ -438,6 +457,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     bool ok = true;
     int tau = tile0, c = c0, p = 0;
     float tbias = 0.f;                 // bias of row r of the current tile, loaded early
+    int ep_tau = -1;                   // cluster split-K: this CTA's tile
+    float ep_bias = 0.f;
     for (int i = 0; i < n_local && ok; ++i) {
       const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
       const bool tlast = i == n_local - 1 || c == nk - 1;
@@ -474,7 +495,26 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       if (tlast) {
         while (ok && drained <= qc)
           if (!drain()) ok = false;
-        if (ok) {
+        if (ok && cq > 1) {
+          // cluster split-K: rank 0 keeps its partial in registers, the others
+          // leave theirs in the (now idle) weight ring for rank 0 to read
+          ep_tau = tau;
+          ep_bias = tbias;
+          if (part != 0) {
+            float* red = reinterpret_cast<float*>(smem) + r * a.Bn;
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+              const int cb = (2 * m + gr) * 16;
+              if (cb < a.Bn) {
+#pragma unroll
+                for (int q = 0; q < 16; q += 4)
+                  *reinterpret_cast<float4*>(red + cb + q) =
+                      make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                                  acc[16 * m + q + 3]);
+              }
+            }
+          }
+        } else if (ok) {
           const bool whole = (tau != tile0 || c0 == 0) && c == nk - 1;
           ok = __all_sync(0xffffffffu, tile_end(tau, whole, tbias));
         }
@@ -483,6 +523,33 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       }
       ++p;
       if (++c == nk) { c = 0; p = 0; ++tau; }
+    }
+    if (cq > 1) {
+      // Cluster split-K finish: rank 0 adds the partials of ranks 1.. (left in their
+      // shared memory) in rank order and runs the epilogue.  (Splitting the epilogue
+      // by column blocks across the ranks measured slower.)
+      cluster_sync_all();   // the partials of ranks 1.. are in their shared memory
+      if (part == 0 && __all_sync(0xffffffffu, ok && ep_tau >= 0)) {
+        for (int rk = 1; rk < cq; ++rk) {
+          const float* red = reinterpret_cast<const float*>(smem) + r * a.Bn;
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int cb = (2 * m + gr) * 16;
+            if (cb < a.Bn) {
+#pragma unroll
+              for (int q = 0; q < 16; q += 4) {
+                const float4 v = ld_cluster_f4(red + cb + q, rk);
+                acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v.x);
+                acc[16 * m + q + 1] = __fadd_rn(acc[16 * m + q + 1], v.y);
+                acc[16 * m + q + 2] = __fadd_rn(acc[16 * m + q + 2], v.z);
+                acc[16 * m + q + 3] = __fadd_rn(acc[16 * m + q + 3], v.w);
+              }
+            }
+          }
+        }
+        tile_end(ep_tau, true, ep_bias);
+      }
+      cluster_sync_all();   // rank 0 has read them: every CTA may exit
     }
   }
   tc_fence_before();
@@ -985,8 +1052,9 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
   (void)P;
   // Cooperative: the finisher of a split tile waits for the other contributors,
   // so every CTA of the grid must be resident at once (the launch fails otherwise).
-  return launch_pdl(k_tc_forward, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s, true,
-                    1, w_fwd, h_in, a);
+  // (Cluster split-K needs no cooperative launch: no cluster waits on another.)
+  return launch_pdl(k_tc_forward, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s,
+                    a.cq <= 1, a.cq > 1 ? a.cq : 1, w_fwd, h_in, a);
 }
 
 cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
