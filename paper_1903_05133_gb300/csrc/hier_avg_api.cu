@@ -301,6 +301,33 @@ double bytes_backward(const hier_avg* h, int l) {
   return P * (in * out * 8.0 + B * in * act + B * out * act + dx);
 }
 
+// Arguments of the small last layer (input H_{L-1}, or X rows for a one-layer model).
+ha::HeadArgs head_args(hier_avg* h) {
+  const int L = h->L;
+  ha::HeadArgs a{};
+  a.C = h->dims[L];
+  a.in = h->dims[L - 1];
+  a.B = h->B;
+  a.Bn = h->Bn;
+  a.pitch_in = h->pitch[L - 1];
+  a.ld = h->ld;
+  a.N = h->N;
+  a.t = h->t;
+  a.lr = h->lr;
+  a.W = h->params + h->woff[L - 1];
+  a.bias = h->params + h->boff[L - 1];
+  a.x_rows = L == 1;
+  a.H = L == 1 ? static_cast<const __nv_bfloat16*>(h->X) : h->wsp<__nv_bfloat16>(h->off_H[L - 1]);
+  a.y = h->y;
+  a.has_dx = L > 1;
+  if (L > 1) {
+    a.bias_prev = h->params + h->boff[L - 2];
+    a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[L - 1]);
+  }
+  a.loss = h->loss();
+  return a;
+}
+
 int do_step(hier_avg* h) {
   const int L = h->L, P = h->P, B = h->B;
   cudaStream_t s = h->stream;
@@ -362,27 +389,7 @@ int do_step(hier_avg* h) {
     }
     const int C = h->dims[L];
     if (h->head) {
-      ha::HeadArgs a{};
-      a.C = C;
-      a.in = h->dims[L - 1];
-      a.B = B;
-      a.Bn = h->Bn;
-      a.pitch_in = h->pitch[L - 1];
-      a.ld = h->ld;
-      a.N = h->N;
-      a.t = h->t;
-      a.lr = h->lr;
-      a.W = h->params + h->woff[L - 1];
-      a.bias = h->params + h->boff[L - 1];
-      a.x_rows = L == 1;
-      a.H = L == 1 ? static_cast<const __nv_bfloat16*>(h->X) : h->wsp<__nv_bfloat16>(h->off_H[L - 1]);
-      a.y = h->y;
-      a.has_dx = L > 1;
-      if (L > 1) {
-        a.bias_prev = h->params + h->boff[L - 2];
-        a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[L - 1]);
-      }
-      a.loss = h->loss();
+      const ha::HeadArgs a = head_args(h);
       const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0));
       rc = h->timed(HA_KERNEL_HEAD, hb, [&] { return ha::launch_head(a, P, s); }, "head");
       if (rc) return rc;

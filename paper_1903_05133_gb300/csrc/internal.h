@@ -60,6 +60,22 @@ cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, 
 // Bn = B rounded up to 16 (the MMA N extent, B <= 64), pitch(d) = d rounded up to
 // 64.  The backward reads H and dZ as stored (MN-major operands), so no transposed
 // copies exist.
+// Small last layer (<= 16 classes) on CUDA cores: one kernel, a thread-block cluster
+// of feature slices per learner (forward, softmax-CE and backward).
+struct HeadArgs {
+  int C, in, B, Bn, pitch_in;
+  int64_t ld, N, t;
+  float lr;
+  float* W;                   // learner 0's W_L [C][in] (fp32 master)
+  float* bias;                // learner 0's b_L
+  const __nv_bfloat16* H;     // H_{L-1} [P][Bn][pitch_in], or X [P][N][in] when x_rows
+  int x_rows;
+  const int32_t* y;
+  int has_dx;                 // write dZ_{L-1} and update b_{L-1}
+  float* bias_prev;
+  __nv_bfloat16* dz_prev;     // [P][Bn][pitch_in]
+  float* loss;                // [P]
+};
 struct TcFwdArgs {
   int in, out, B, Bn;
   int64_t ld;                 // parameter row length (floats)
@@ -121,22 +137,6 @@ cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_
                              int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
                              __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s);
 
-// Small last layer (<= 16 classes) on CUDA cores: one kernel, a thread-block cluster
-// of feature slices per learner (forward, softmax-CE and backward).
-struct HeadArgs {
-  int C, in, B, Bn, pitch_in;
-  int64_t ld, N, t;
-  float lr;
-  float* W;                   // learner 0's W_L [C][in] (fp32 master)
-  float* bias;                // learner 0's b_L
-  const __nv_bfloat16* H;     // H_{L-1} [P][Bn][pitch_in], or X [P][N][in] when x_rows
-  int x_rows;
-  const int32_t* y;
-  int has_dx;                 // write dZ_{L-1} and update b_{L-1}
-  float* bias_prev;
-  __nv_bfloat16* dz_prev;     // [P][Bn][pitch_in]
-  float* loss;                // [P]
-};
 bool head_supported(int C, int in, int B);
 cudaError_t head_configure();   // raises the dynamic shared-memory limit once
 cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s);
