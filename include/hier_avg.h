@@ -190,6 +190,12 @@ int hier_avg_profile(hier_avg* h, int enable);
  * reports.  HA_EINVAL for bits beyond HA_KERNEL_KINDS. */
 int hier_avg_profile_kinds(hier_avg* h, unsigned kinds);
 
+/* Time only every n-th launch of each enabled kind (n >= 1, default 1; counted from
+ * the last hier_avg_profile / hier_avg_profile_kinds), so that a throughput
+ * measurement perturbs few launches.  hier_avg_profile_read then reports the
+ * sampled launches.  HA_EINVAL for n < 1. */
+int hier_avg_profile_every(hier_avg* h, int every);
+
 /* Synchronise and read kind's totals since profiling was enabled: summed event
  * time in ms, number of launches, and the algorithmic bytes moved by them. */
 int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* launches,

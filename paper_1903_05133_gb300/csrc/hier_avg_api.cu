@@ -85,6 +85,8 @@ struct hier_avg {
   int64_t t = 0;
   // profiling
   unsigned prof = 0;                          // kinds timed: bit (1 << HA_KERNEL_*)
+  int prof_every = 1;                         // time every n-th launch of those kinds
+  int64_t prof_seen[HA_KERNEL_KINDS] = {};    // launches of each kind since enabled
   std::vector<ProfRec> recs;
   std::vector<cudaEvent_t> pool;
   size_t pool_used = 0;
@@ -120,7 +122,8 @@ struct hier_avg {
   template <class F>
   int timed(int kind, double bytes, F&& launch, const char* what) {
     cudaEvent_t a = nullptr, b = nullptr;
-    const bool on = (prof >> kind) & 1u;
+    bool on = (prof >> kind) & 1u;
+    if (on) on = prof_seen[kind]++ % prof_every == 0;
     if (on) {
       a = ev();
       b = ev();
@@ -723,11 +726,18 @@ int hier_avg_check(hier_avg* h) {
   return HA_OK;
 }
 
+int hier_avg_profile_every(hier_avg* h, int every) {
+  if (!h || every < 1) return HA_EINVAL;
+  h->prof_every = every;
+  return HA_OK;
+}
+
 int hier_avg_profile_kinds(hier_avg* h, unsigned kinds) {
   if (!h) return HA_EINVAL;
   if (kinds >> HA_KERNEL_KINDS) return h->fail(HA_EINVAL, "profile: unknown kernel kind bit");
   if (h->bound) cudaStreamSynchronize(h->stream);
   h->recs.clear();
+  for (auto& n : h->prof_seen) n = 0;
   h->pool_used = 0;
   h->prof = kinds;
   return HA_OK;

@@ -182,6 +182,10 @@ class HierAvg:
             mask |= 1 << KERNEL_KINDS[k]
         check(self._lib.hier_avg_profile_kinds(self.h, mask), "profile", self.h)
 
+    def profile_every(self, every: int) -> None:
+        """Time only every n-th launch of each enabled kind."""
+        check(self._lib.hier_avg_profile_every(self.h, int(every)), "profile_every", self.h)
+
     def profile_read(self, kind: str) -> Tuple[float, int, float]:
         ms, n, by = c_double(), c_int64(), c_double()
         check(self._lib.hier_avg_profile_read(self.h, KERNEL_KINDS[kind], ctypes.byref(ms),
