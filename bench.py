@@ -58,6 +58,23 @@ def dist_env():
     return ws, rank, local
 
 
+def job_seconds(seconds: float, ws: int, device=None) -> float:
+    """The job's time: the maximum over the ranks of each rank's timed seconds
+    (every rank runs an independent replica; the slowest one ends the job)."""
+    if ws <= 1:
+        return seconds
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([seconds], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(ws: int, units_per_round: int, rounds: int, seconds: float) -> float:
+    """Whole-job throughput: the units all replicas processed over the job's time."""
+    return ws * units_per_round * rounds / seconds
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -293,13 +310,9 @@ def run_ours(args):
     clocks = sampler.stop(uuid)
     ha.check()
     round_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    T = sum(round_ms) / 1000.0
-    if ws > 1:
-        t = torch.tensor([T], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        T = float(t.item())
+    T = job_seconds(sum(round_ms) / 1000.0, ws, dev)
     per_round = w.samples_per_round
-    value = ws * per_round * args.steps / T
+    value = replica_throughput(ws, per_round, args.steps, T)
 
     dom_live = ha.profile_read(dom)          # the dominant kernel, timed inside the timed rounds
     ha.profile(False)
@@ -369,14 +382,10 @@ def run_ours(args):
         for _ in range(args.steps):
             ha.round_host(Xh, yh, loss)
         torch.cuda.synchronize()
-        Te = time.perf_counter() - t0
-        if ws > 1:
-            t = torch.tensor([Te], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            Te = float(t.item())
+        Te = job_seconds(time.perf_counter() - t0, ws, dev)
         rows = w.B * w.K1 * w.K2
         es = 2 if w.precision == "bf16" else 4
-        line["e2e"] = {"value": ws * per_round * args.steps / Te, "unit": UNIT,
+        line["e2e"] = {"value": replica_throughput(ws, per_round, args.steps, Te), "unit": UNIT,
                        "h2d_bytes_per_step": w.P * rows * (w.dims[0] * es + 4),
                        "d2h_bytes_per_step": w.P * 4,
                        "api": "hier_avg_round_host (pinned host X, y; loss read back)"}
