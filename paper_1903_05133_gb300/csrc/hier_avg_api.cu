@@ -65,6 +65,7 @@ struct hier_avg {
   std::vector<int64_t> off_H, off_dZ;
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
+  int64_t off_dyn = 0;                        // update kernel's work-item counters
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
   std::vector<int> fwd_cq;                    // per layer: cluster split factor (1 = stream-K)
   std::vector<int> bwd_ctas, bwd_tiles;       // per layer: stream-K CTAs, input slices
@@ -207,6 +208,7 @@ int plan_layout(hier_avg* h) {
     h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B));
     h->off_part = take(part_bytes);
     h->off_cnt = take(max_tiles * 4);
+    h->off_dyn = take(16);
   } else {
     for (int l = 0; l <= L; ++l) h->pitch[l] = h->dims[l];
     for (int l = 0; l < L; ++l) h->off_H[l] = take(P * B * h->dims[l] * 4);
@@ -430,9 +432,22 @@ int do_step(hier_avg* h) {
       a.counters = h->wsp<int>(h->off_cnt);
       a.err = h->err_word();
       const CUtensorMap& hin = from_x ? h->tm_x : h->tm_h[l];
-      rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
-        return ha::launch_tc_backward(h->tm_wb[l], hin, h->tm_dz[l + 1], a, P, s);
-      }, "backward");
+      // The first layer's backward (no dX) hands its independent units out dynamically
+      // when there are many of them per SM (work items of 8 chunks); a short layer keeps
+      // the even static split, which work items that coarse would unbalance.
+      const int64_t units = int64_t(a.n_tiles) * ((a.out + 63) / 64);
+      if (a.has_dx || units < int64_t(kTargetCtas) * 64) {
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+          return ha::launch_tc_backward(h->tm_wb[l], hin, h->tm_dz[l + 1], a, P, s);
+        }, "backward");
+      } else {
+        // no dX: independent units, handed out dynamically
+        a.dyn = h->wsp<int>(h->off_dyn);
+        a.ctas = kTargetCtas;
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+          return ha::launch_tc_update(h->tm_wb[l], hin, h->tm_dz[l + 1], a, s);
+        }, "backward");
+      }
       if (rc) return rc;
     }
   } else {

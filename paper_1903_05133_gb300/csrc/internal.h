@@ -119,6 +119,7 @@ struct TcBwdArgs {
   int ctas, n_tiles, s_tiles;
   float* part;
   int* counters;
+  int* dyn;                   // update-only kernel: [0] work items claimed, [1] CTAs done
   int* err;
 };
 int tc_fwd_smem_bytes();
@@ -128,6 +129,10 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s);
 cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
                                const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s);
+// The first layer's backward (no dX): dW, update and store only, units claimed
+// dynamically (a.dyn zero on entry; reset by the kernel on exit).
+cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
+                             const CUtensorMap& dz, const TcBwdArgs& a, cudaStream_t s);
 // Mini-batch fetch for the bf16 path: rows (t*B + b) mod N of X -> H_0.
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
                                int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s);

@@ -957,6 +957,282 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   }
 }
 
+// ------------------------------------------------------------------ update only
+// The first layer's backward has no dX: every unit (tile, chunk) is independent
+// (dW^T of the chunk, the fp32 update, the store), so the units are handed out
+// dynamically and faster SMs simply take more of them (a static split left SMs idle
+// for up to a third of the kernel waiting for slow ones).  Work item = a run of up to
+// kRun chunks of one tile, claimed by warp 4 from a global counter and announced to
+// the other roles through a small queue in shared memory; the last CTA to finish
+// resets the counters.  Roles as in k_tc_backward, without the dX path.
+constexpr int kRun = 8;                 // chunks per work item
+constexpr int kQueue = 8;               // queued work items
+__host__ __device__ constexpr int upd_smem(int Bn) { return bwd_smem(Bn) + 512; }
+static_assert(upd_smem(64) <= kBwdSmemMax && upd_smem(48) <= kBwdSmemMax &&
+                  upd_smem(32) <= kBwdSmemMax && upd_smem(16) <= kBwdSmemMax,
+              "update kernel shared-memory plan");
+
+__global__ void __launch_bounds__(kBwdThreads, 1)
+    k_tc_update(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
+                const __grid_constant__ CUtensorMap tm_dz, const TcBwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nc = (a.out + 63) / 64;
+  const int rpt = (nc + kRun - 1) / kRun;                  // work items per tile
+  const int n_items = a.n_tiles * rpt;
+  const int nw = bwd_wring(a.Bn), nz = bwd_zring(a.Bn);
+  const int tbytes = a.Bn * 128;
+  uint8_t* h_base = smem + bwd_h_off(a.Bn);
+  uint8_t* z_base = smem + bwd_z_off(a.Bn);
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + bwd_bar_off(a.Bn));
+  uint64_t* wempty = wfull + kBwdWRingMax;   // chunk stored back (TMA has read it)
+  uint64_t* upd = wempty + kBwdWRingMax;     // chunk updated in shared memory
+  uint64_t* zfull = upd + kBwdWRingMax;
+  uint64_t* zempty = zfull + kBwdZRingMax;   // dZ tile consumed by the MMA
+  uint64_t* hfull = zempty + kBwdZRingMax;   // [2]
+  uint64_t* hempty = hfull + 2;              // [2] the item's last MMA is done
+  uint64_t* dwdone = hempty + 2;             // [2]
+  uint64_t* dwfree = dwdone + 2;             // [2]
+  uint64_t* done = dwfree + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* qfull = reinterpret_cast<uint64_t*>(smem + bwd_bar_off(a.Bn) + 512);
+  uint64_t* qempty = qfull + kQueue;         // read by the 7 consuming warps
+  int* items = reinterpret_cast<int*>(qempty + kQueue);
+  auto wf = [&](int s) { return smem + s * kBwdWf32; };
+  auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
+  auto zb = [&](int s) { return z_base + s * tbytes; };
+  constexpr int kConsumers = 3 + kBwdConv / 32;             // dZ, MMA, store + converter warps
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kBwdWRingMax; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], 1);
+      mbar_init(&upd[s], kBwdConv / 32);
+    }
+    for (int s = 0; s < kBwdZRingMax; ++s) {
+      mbar_init(&zfull[s], 1);
+      mbar_init(&zempty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&hfull[b], 1);
+      mbar_init(&hempty[b], 1);
+      mbar_init(&dwdone[b], 1);
+      mbar_init(&dwfree[b], kBwdConv / 32);
+    }
+    for (int q = 0; q < kQueue; ++q) {
+      mbar_init(&qfull[q], 1);
+      mbar_init(&qempty[q], kConsumers);
+    }
+    mbar_init(done, 1);
+    fence_barrier_init();
+  }
+  if (warp == 5) {
+    tmem_alloc(tmem_slot, kBwdTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  grid_dep_wait();                       // the previous kernel's results are visible
+
+  // Consumers: the k-th queued work item (-1: no more), read by every lane of the
+  // warp; lane 0 then frees the slot for this warp.
+  auto take = [&](int k) -> int {
+    const int q = k % kQueue;
+    if (!wait_warp(&qfull[q], (k / kQueue) & 1, a.err)) return -1;
+    const int it = items[q];
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&qempty[q]);
+    return it;
+  };
+  // Chunks [c_lo, c_hi) of tile `tile` for work item `it`.
+  auto decode = [&](int it, int& tile, int& c_lo, int& c_hi) {
+    tile = it / rpt;
+    c_lo = (it - tile * rpt) * kRun;
+    c_hi = c_lo + kRun < nc ? c_lo + kRun : nc;
+  };
+
+  if (warp == 4) {
+    if (lane == 0) {
+      // claim, announce, and load: W chunks and each item's H tile
+      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_h);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      int i = 0, kt = 0, issued = 0;
+      bool ok = true;
+      int next = atomicAdd(a.dyn, 1);
+      for (int k = 0; ok; ++k) {
+        const int it = next < n_items ? next : -1;
+        const int q = k % kQueue;
+        if (k >= kQueue && !mbar_wait(&qempty[q], ((k / kQueue) - 1) & 1, a.err)) break;
+        items[q] = it;
+        mbar_arrive(&qfull[q]);
+        if (it < 0) break;
+        next = atomicAdd(a.dyn, 1);           // the next claim, hidden behind these loads
+        int tile, c_lo, c_hi;
+        decode(it, tile, c_lo, c_hi);
+        const int j = tile / a.s_tiles, i0 = (tile - j * a.s_tiles) * 128;
+        const int hbuf = kt & 1;
+        if (kt >= 2 && !mbar_wait(&hempty[hbuf], ((kt >> 1) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&hfull[hbuf], 2 * tbytes);
+        tma_load_3d(hb(hbuf), &tm_h, &hfull[hbuf], i0, a.h_row0, j);
+        tma_load_3d(hb(hbuf) + tbytes, &tm_h, &hfull[hbuf], i0 + 64, a.h_row0, j);
+        ++kt;
+        for (int c = c_lo; c < c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
+          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], i0, c * 64, j, stream);
+          issued = i + 1;
+        }
+      }
+      for (int u = issued - nw > 0 ? issued - nw : 0; u < issued; ++u)
+        mbar_wait(&wfull[u % nw], (u / nw) & 1, a.err);
+      for (int u = kt - 2 > 0 ? kt - 2 : 0; u < kt; ++u) mbar_wait(&hfull[u & 1], (u >> 1) & 1, a.err);
+    }
+  } else if (warp == 6) {
+    int i = 0, issued = 0;
+    if (lane == 0) tma_prefetch_desc(&tm_dz);
+    for (int k = 0;; ++k) {
+      const int it = take(k);
+      if (it < 0) break;
+      if (lane == 0) {
+        int tile, c_lo, c_hi;
+        decode(it, tile, c_lo, c_hi);
+        const int j = tile / a.s_tiles;
+        for (int c = c_lo; c < c_hi; ++c, ++i) {
+          const int s = i % nz;
+          if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) break;
+          mbar_arrive_expect_tx(&zfull[s], tbytes);
+          tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j);
+          issued = i + 1;
+        }
+      }
+      __syncwarp();
+    }
+    if (lane == 0)
+      for (int u = issued - nz > 0 ? issued - nz : 0; u < issued; ++u)
+        mbar_wait(&zfull[u % nz], (u / nz) & 1, a.err);
+  } else if (warp == 7) {
+    const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+    int i = 0;
+    for (int k = 0;; ++k) {
+      const int it = take(k);
+      if (it < 0) break;
+      if (lane == 0) {
+        int tile, c_lo, c_hi;
+        decode(it, tile, c_lo, c_hi);
+        const int j = tile / a.s_tiles, i0 = (tile - j * a.s_tiles) * 128;
+        for (int c = c_lo; c < c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
+          tma_store_3d_hint(&tm_w, wf(s), i0, c * 64, j, stream);
+          tma_store_commit();
+          if (i > 0) {
+            tma_store_wait_read_1();
+            mbar_arrive(&wempty[(i - 1) % nw]);
+          }
+        }
+      }
+      __syncwarp();
+    }
+    if (lane == 0) {
+      tma_store_wait_all();
+      if (i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
+    }
+  } else if (warp == 5) {
+    const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
+    const int kb = a.Bn / 16;
+    int i = 0, kt = -1;
+    bool ok = true;
+    for (int k = 0; ok; ++k) {
+      const int it = take(k);
+      if (it < 0) break;
+      ++kt;
+      if (lane == 0) {
+        int tile, c_lo, c_hi;
+        decode(it, tile, c_lo, c_hi);
+        if (!mbar_wait(&hfull[kt & 1], (kt >> 1) & 1, a.err)) ok = false;
+        const uint32_t hs = smem_u32(hb(kt & 1));
+        for (int c = c_lo; c < c_hi && ok; ++c, ++i) {
+          const int sz = i % nz, b = i & 1;
+          if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) { ok = false; break; }
+          if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t zs = smem_u32(zb(sz));
+          for (int kk = 0; kk < kb; ++kk)
+            tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
+                        umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+          tc_commit(&dwdone[b]);
+          tc_commit(&zempty[sz]);
+        }
+        tc_commit(&hempty[kt & 1]);          // the H tile is free once these MMAs are
+      }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
+      tc_commit(done);
+      mbar_wait(done, 0, a.err);
+    }
+  } else {
+    // ---- warps 0-3: thread t owns input feature i0 + t of the current chunk
+    const int t = threadIdx.x;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    int i = 0;
+    bool ok = true;
+    for (int k = 0; ok; ++k) {
+      const int it = take(k);
+      if (it < 0) break;
+      int tile, c_lo, c_hi;
+      decode(it, tile, c_lo, c_hi);
+      for (int c = c_lo; c < c_hi; ++c, ++i) {
+        const int sw = i % nw, b = i & 1;
+        if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+        float* w = reinterpret_cast<float*>(wf(sw));
+        float wv[64];
+#pragma unroll
+        for (int o = 0; o < 64; ++o) wv[o] = w[o * 128 + t];
+        if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int qb = 0; qb < 4; ++qb) {
+          float d[16];
+          tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&dwfree[b]);
+#pragma unroll
+        for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&upd[sw]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kBwdTmemCols);
+  }
+  if (threadIdx.x == 0) {
+    // the last CTA out resets the counters for the next launch (every claim of every
+    // CTA precedes that CTA's increment here)
+    __threadfence();
+    if (atomicAdd(a.dyn + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+      a.dyn[0] = 0;
+      a.dyn[1] = 0;
+    }
+  }
+}
+
 // ------------------------------------------------------------------ gather
 // H_0[j][b][:] = X[j][(t*B + b) mod N][:] for b < B, one CTA per (64-feature slice,
 // learner); rows b >= B stay zero.
@@ -1043,8 +1319,9 @@ cudaError_t tc_configure() {
   cudaError_t e = cudaFuncSetAttribute(k_tc_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        kFwdSmemMax);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              kBwdSmemMax);
+  e = cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_tc_update, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
 }
 
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
@@ -1062,6 +1339,13 @@ cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in
   (void)P;
   // Cooperative for the same reason as the forward (split dX tiles).
   return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, true, 1,
+                    w_bwd, h_in, dz, a);
+}
+
+cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
+                             const CUtensorMap& dz, const TcBwdArgs& a, cudaStream_t s) {
+  // no CTA waits on another: an ordinary (programmatically serialised) launch
+  return launch_pdl(k_tc_update, dim3(a.ctas), dim3(kBwdThreads), upd_smem(a.Bn), s, false, 1,
                     w_bwd, h_in, dz, a);
 }
 
