@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--N", type=int, default=None,
                     help="samples per learner (default: the workload's); for small profiling runs")
+    ap.add_argument("--P", type=int, default=None,
+                    help="learners (default: the workload's; a multiple of S); for small profiling runs")
     return ap.parse_args()
 
 
@@ -261,6 +263,10 @@ def run_ours(args):
     w = configs.SHORT[args.workload]
     if args.N:
         w = w.replace(N=args.N)
+    if args.P:
+        if args.P % w.S:
+            raise SystemExit(f"--P must be a multiple of S = {w.S}")
+        w = w.replace(P=args.P)
     X, y = learner_data(w, device=dev)
     layers = initial_layers(w, device=dev)
     ha = HierAvg(w.P, w.S, w.K1, w.K2, w.lr, w.B, w.dims, w.precision)
@@ -339,7 +345,8 @@ def run_ours(args):
                           "GBps": round(by / (ms / 1e3) / 1e9, 1) if ms > 0 else None}
     avg_ms = prof["local_avg"][0] + prof["global_avg"][0]
     avg_by = prof["local_avg"][2] + prof["global_avg"][2]
-    traffic = ncu_traffic(dom, w.name)
+    # per-launch DRAM bytes scale with P: a run with fewer learners has no captured figure
+    traffic = ncu_traffic(dom, w.name) if not args.P else None
     roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"],
                 "unit": "GB/s", "frac": (achieved / pk["hbm_gbs"]) if achieved else None,
                 "peak_source": pk_src,
