@@ -182,7 +182,15 @@ def launches_per_round(w) -> int:
             per_step = (L - 1) + 1 + (L - 1)
         else:
             per_step = L + (0 if C <= 128 else 1) + L
-        n = w.K1 * w.K2 * per_step + gathers
+        # inside a local block, a step whose successor reads a contiguous batch also runs
+        # that successor's first-layer forward (one launch fewer)
+        fused = 0
+        if L >= 2:
+            for t in steps:
+                nxt = ((t + 1) * w.B) % w.N
+                if t % w.K1 != w.K1 - 1 and nxt + w.B <= w.N:
+                    fused += 1
+        n = w.K1 * w.K2 * per_step + gathers - fused
     else:
         per_step = 1 + L + 1 + L + (L - 1)       # dX is its own launch for layers > 1
         n = w.K1 * w.K2 * per_step
@@ -282,14 +290,16 @@ def run_ours(args):
     # Untimed profiling pass: every kernel kind, to find the dominant kernel and to
     # report the per-kind breakdown.  (An event pair around a launch separates it
     # from its neighbours, so the timed rounds below time only the dominant kind.)
-    kinds = ["gather", "forward", "xent", "backward", "local_avg", "global_avg", "head"]
+    kinds = ["gather", "forward", "xent", "backward", "local_avg", "global_avg", "head",
+             "update_forward"]
     ha.profile(True)
     for _ in range(max(1, min(args.steps, 3))):
         flush.zero_()
         ha.round()
     prof = {k: ha.profile_read(k) for k in kinds}
     ha.profile(False)
-    main_kinds = ["forward", "backward", "local_avg", "global_avg", "xent", "gather", "head"]
+    main_kinds = ["forward", "backward", "local_avg", "global_avg", "xent", "gather", "head",
+                  "update_forward"]
     dom = max(main_kinds, key=lambda k: prof[k][0])
 
     props = torch.cuda.get_device_properties(dev)

@@ -126,7 +126,11 @@ int hier_avg_global_average(hier_avg* h);
 
 /* One global round of Algorithm 1: K2 x (K1 x step, local average), then the
  * global average; the last local average is fused with the global one
- * (bit-identical to doing them in turn). */
+ * (bit-identical to doing them in turn).  Within the round, a step whose successor
+ * starts no local block and reads a contiguous batch also computes that successor's
+ * first-layer output from the weights it has just updated (bf16 path, two or more
+ * layers), so W_1 is read once per step; the results are those of calling
+ * hier_avg_step in turn. */
 int hier_avg_round(hier_avg* h);
 
 /* One round end to end from host memory: copies the rows this round reads from
@@ -181,7 +185,8 @@ int hier_avg_check(hier_avg* h);
 #define HA_KERNEL_LOCAL_AVG     4
 #define HA_KERNEL_GLOBAL_AVG    5   /* fused last local + global average     */
 #define HA_KERNEL_HEAD          6   /* fused last layer (<= 16 classes)      */
-#define HA_KERNEL_KINDS         7
+#define HA_KERNEL_UPDATE_FORWARD 7  /* first-layer update + next forward     */
+#define HA_KERNEL_KINDS         8
 int hier_avg_profile(hier_avg* h, int enable);
 
 /* The same for a subset: kinds is a bitmask of (1 << HA_KERNEL_*); 0 stops.

@@ -299,6 +299,12 @@ double bytes_forward(const hier_avg* h, int l) {
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
   return P * (in * out * 4.0 + out * 4.0 + B * in * act + B * out * (l + 1 == h->L ? 4.0 : act));
 }
+// The first layer's update fused with the next step's first-layer forward: W read and
+// written once, this step's and the next step's batch rows, dZ_1 read, b_1 read, H_1' written.
+double bytes_update_forward(const hier_avg* h) {
+  const double P = h->P, in = h->dims[0], out = h->dims[1], B = h->B;
+  return P * (in * out * 8.0 + out * 4.0 + 2.0 * B * in * 2.0 + 2.0 * B * out * 2.0);
+}
 double bytes_backward(const hier_avg* h, int l) {
   const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
@@ -333,8 +339,13 @@ ha::HeadArgs head_args(hier_avg* h) {
   return a;
 }
 
-int do_step(hier_avg* h) {
+// One step.  h1_ready: H_1 of this step was written by the previous step's
+// update+forward kernel (skip the first layer's forward).  fuse_next: the caller runs
+// the next step right after this one with nothing in between, so this step may
+// compute the next step's H_1; *fused reports whether it did.
+int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr) {
   const int L = h->L, P = h->P, B = h->B;
+  if (fused) *fused = false;
   cudaStream_t s = h->stream;
   int rc;
   if (h->prec == HA_PREC_BF16) {
@@ -351,7 +362,7 @@ int do_step(hier_avg* h) {
       if (rc) return rc;
     }
     const int n_fwd = h->head ? L - 1 : L;
-    for (int l = 0; l < n_fwd; ++l) {
+    for (int l = h1_ready ? 1 : 0; l < n_fwd; ++l) {
       TcFwdArgs a{};
       a.in = h->dims[l];
       a.out = h->dims[l + 1];
@@ -432,6 +443,39 @@ int do_step(hier_avg* h) {
       a.counters = h->wsp<int>(h->off_cnt);
       a.err = h->err_word();
       const CUtensorMap& hin = from_x ? h->tm_x : h->tm_h[l];
+      // The next step's batch, if contiguous in X, lets the first layer's update also
+      // produce the next step's H_1 (the layer must be hidden, i.e. L >= 2).
+      const int64_t r1 = ((h->t + 1) * B) % h->N;
+      if (l == 0 && fuse_next && L >= 2 && r1 + B <= h->N) {
+        TcFwdArgs f{};
+        f.in = h->dims[0];
+        f.out = h->dims[1];
+        f.B = B;
+        f.Bn = h->Bn;
+        f.ld = h->ld;
+        f.bias = h->params + h->boff[0];
+        f.mode = 0;
+        f.h_out = h->wsp<__nv_bfloat16>(h->off_H[1]);
+        f.pitch_out = h->pitch[1];
+        f.ctas = h->fwd_ctas[0];
+        f.cq = h->fwd_cq[0];
+        f.o_tiles = h->fwd_tiles[0];
+        f.n_tiles = h->fwd_tiles[0] * P;
+        f.part = h->wsp<float>(h->off_part);
+        f.counters = h->wsp<int>(h->off_cnt);
+        f.x_direct = 1;
+        f.x_row0 = static_cast<int>(r1);
+        f.hc_row0 = a.h_row0;
+        f.w_stream = a.w_stream;
+        f.lr = h->lr;
+        f.err = h->err_word();
+        rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h), [&] {
+          return ha::launch_tc_update_forward(h->tm_wf[0], hin, h->tm_x, h->tm_dz[1], f, s);
+        }, "update+forward");
+        if (rc) return rc;
+        if (fused) *fused = true;
+        continue;
+      }
       // The first layer's backward (no dX) hands its independent units out dynamically
       // when there are many of them per SM (work items of 8 chunks); a short layer keeps
       // the even static split, which work items that coarse would unbalance.
@@ -506,8 +550,9 @@ int do_local_global(hier_avg* h) {
 int do_round(hier_avg* h) {
   int rc;
   for (int b = 0; b < h->K2; ++b) {
+    bool h1_ready = false;
     for (int k = 0; k < h->K1; ++k)
-      if ((rc = do_step(h))) return rc;
+      if ((rc = do_step(h, h1_ready, k + 1 < h->K1, &h1_ready))) return rc;
     if (b + 1 < h->K2 && (rc = do_local(h))) return rc;
   }
   return do_local_global(h);

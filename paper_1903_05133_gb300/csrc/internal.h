@@ -95,6 +95,7 @@ struct TcFwdArgs {
   int* counters;
   // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)
   int x_direct, x_row0;
+  int hc_row0;                // update+forward: rows of this step's batch in its map
   int w_stream;               // load W with the L2 evict-first policy
   // mode 2: labels and outputs of the fused cross-entropy
   const int32_t* y;
@@ -133,6 +134,12 @@ cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in
 // dynamically (a.dyn zero on entry; reset by the kernel on exit).
 cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
                              const CUtensorMap& dz, const TcBwdArgs& a, cudaStream_t s);
+// The first layer's backward (dW, update, store) fused with the next step's first-layer
+// forward (H_1' = relu(X' W_1'^T + b_1), schedule and arithmetic of launch_tc_forward):
+// h_cur holds this step's batch rows (a.hc_row0 ..), x_next the next step's (a.x_row0 ..).
+cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_cur,
+                                     const CUtensorMap& x_next, const CUtensorMap& dz,
+                                     const TcFwdArgs& a, cudaStream_t s);
 // Mini-batch fetch for the bf16 path: rows (t*B + b) mod N of X -> H_0.
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
                                int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s);

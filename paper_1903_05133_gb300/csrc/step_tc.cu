@@ -1233,6 +1233,486 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   }
 }
 
+// ------------------------------------------------------------------ update + next forward
+// The first layer's input is the data, so the forward of the NEXT step's first layer,
+// Z_1' = X' W_1'^T (X' = the next batch, W_1' = W_1 after this step's update), can be
+// computed by the kernel that produces W_1': this step's first-layer backward.  Then
+// W_1 is read once per step instead of twice (update + next forward: 8 bytes per
+// weight instead of 12).  The kernel keeps the forward's units and schedule exactly
+// (tile = learner j x 128 outputs, chunk = 64 inputs; stream-K or cluster split-K with
+// the same split, the same 4 MMAs per chunk and the same every-kSegChunks promotion),
+// so Z_1' is bit-identical to what k_tc_forward computes from the stored W_1'.  Per
+// chunk:
+//   dW[o][i]  = sum_b dZ_1[b][o] X[b][i]      M = 128 outputs, N = 64 inputs, K = Bn
+//                                             (dZ tile and X tile both MN-major)
+//   W[o][i]  -= lr dW[o][i]                   fp32, in the shared-memory W tile, which is
+//                                             then TMA-stored back
+//   Z'^T     += W'_q X'^T                      A = W' rounded to bf16, written to TMEM by
+//                                             the thread that owns output row o
+// and the tile epilogue writes H_1' = relu(Z' + b_1) (b_1 already updated by the layer
+// above).  Warps 0-7 own the accumulator rows as in the forward (row 32*(w%4) + lane,
+// input half w/4) and do the update, the bf16 conversion and the drains; warp 8 loads
+// W tiles, warp 9 issues the MMAs (the dW MMAs of chunk i before the forward MMAs of
+// chunk i-1, so the update of one chunk overlaps the dW of the next), warp 10 loads
+// the batch tiles (X and X' rows of the chunk) and dZ tiles and publishes a split
+// tile's partial, warp 11 stores updated W tiles and frees their slots.
+constexpr int kUfConv = 256;
+constexpr int kUfThreads = kUfConv + 128;
+// TMEM columns: Z'^T accumulators at 0 and 64, bf16 A tiles at 128 and 160, dW
+// accumulators at 256 and 320.
+constexpr uint32_t kUfTmemCols = 512, kUfTmemA = 128, kUfTmemDW = 256;
+
+// Layout: W ring | 2 dZ tiles ([Bn][128] bf16, two boxes each) | batch ring (X box, X'
+// box per chunk) | barriers.
+__host__ __device__ constexpr int uf_wring(int Bn) { return Bn <= 32 ? 5 : 4; }
+__host__ __device__ constexpr int uf_z_off(int Bn) { return uf_wring(Bn) * kFwdWf32; }
+__host__ __device__ constexpr int uf_h_off(int Bn) { return uf_z_off(Bn) + 2 * 2 * Bn * 128; }
+__host__ __device__ constexpr int uf_hring(int Bn) {
+  return (kFwdSmemMax - 1024 - 512 - uf_h_off(Bn)) / (2 * Bn * 128) < kFwdHRingMax
+             ? (kFwdSmemMax - 1024 - 512 - uf_h_off(Bn)) / (2 * Bn * 128)
+             : kFwdHRingMax;
+}
+__host__ __device__ constexpr int uf_bar_off(int Bn) { return uf_h_off(Bn) + uf_hring(Bn) * 2 * Bn * 128; }
+__host__ __device__ constexpr int uf_smem(int Bn) { return uf_bar_off(Bn) + 512 + 1024; }
+// (the cluster split-K partial [128][Bn] fp32 is staged in the batch ring: hring >= 2)
+static_assert(uf_hring(64) >= 4 && uf_hring(48) >= 6 && uf_hring(32) >= 6 && uf_hring(16) == 8 &&
+                  uf_smem(64) <= kFwdSmemMax && uf_smem(48) <= kFwdSmemMax &&
+                  uf_smem(32) <= kFwdSmemMax && uf_smem(16) <= kFwdSmemMax,
+              "update+forward shared-memory plan");
+
+__global__ void __launch_bounds__(kUfThreads, 1)
+    k_tc_update_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_hc,
+                        const __grid_constant__ CUtensorMap tm_hn, const __grid_constant__ CUtensorMap tm_dz,
+                        const TcFwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = blockIdx.x, G = gridDim.x;
+  const int nk = (a.in + 63) / 64;
+  const int U = a.n_tiles * nk;
+  const int cq = a.cq > 1 ? a.cq : 1, part = g % cq;
+  const int u0 = cq > 1 ? (g / cq) * nk + part * nk / cq : unit_begin(g, U, G);
+  const int u1 = cq > 1 ? (g / cq) * nk + (part + 1) * nk / cq : unit_begin(g + 1, U, G);
+  const int n_local = u1 - u0;
+  const int nw = uf_wring(a.Bn), nh = uf_hring(a.Bn);
+  const int tbytes = a.Bn * 128;                            // one [Bn][64] bf16 box
+  const int tile0 = u0 / nk, c0 = u0 - tile0 * nk;
+  uint8_t* z_base = smem + uf_z_off(a.Bn);
+  uint8_t* h_base = smem + uf_h_off(a.Bn);
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + uf_bar_off(a.Bn));
+  uint64_t* wempty = wfull + kFwdWRingMax;   // W tile stored back (the TMA has read it)
+  uint64_t* upd = wempty + kFwdWRingMax;     // W tile updated in shared memory
+  uint64_t* hfull = upd + kFwdWRingMax;
+  uint64_t* hempty = hfull + kFwdHRingMax;   // X and X' boxes consumed by both MMAs
+  uint64_t* zfull = hempty + kFwdHRingMax;   // [2]
+  uint64_t* zempty = zfull + 2;              // [2] dZ tile consumed by the tile's dW MMAs
+  uint64_t* dwdone = zempty + 2;             // [2] dW of the chunk complete
+  uint64_t* dwfree = dwdone + 2;             // [2] dW read by the update
+  uint64_t* conv = dwfree + 2;               // [2] A tile written to TMEM
+  uint64_t* afree = conv + 2;                // [2] A tile consumed by the forward MMA
+  uint64_t* accf = afree + 2;                // [2] accumulator segment complete
+  uint64_t* accr = accf + 2;                 // [2] accumulator segment drained
+  uint64_t* gbar = accr + 2;
+  uint64_t* done = gbar + 1;
+  uint64_t* pready = done + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
+  auto wf = [&](int s) { return smem + s * kFwdWf32; };
+  auto zb = [&](int s) { return z_base + s * 2 * tbytes; };
+  auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kFwdWRingMax; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], 1);
+      mbar_init(&upd[s], kUfConv / 32);
+    }
+    for (int s = 0; s < kFwdHRingMax; ++s) {
+      mbar_init(&hfull[s], 1);
+      mbar_init(&hempty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&zfull[b], 1);
+      mbar_init(&zempty[b], 1);
+      mbar_init(&dwdone[b], 1);
+      mbar_init(&dwfree[b], kUfConv / 32);
+      mbar_init(&conv[b], kUfConv / 32);
+      mbar_init(&afree[b], 1);
+      mbar_init(&accf[b], 1);
+      mbar_init(&accr[b], kUfConv);
+    }
+    mbar_init(gbar, kUfConv);
+    mbar_init(done, 1);
+    mbar_init(pready, kUfConv / 32);
+    fence_barrier_init();
+  }
+  if (warp == 9) {
+    tmem_alloc(tmem_slot, kUfTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  grid_dep_wait();                       // dZ_1 and b_1 of the layer above are visible
+
+  if (warp == 8) {
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_w);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      int issued = 0, tau = tile0, c = c0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+        const int s = i % nw;
+        if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
+        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j, stream);
+        tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j, stream);
+        issued = i + 1;
+        if (++c == nk) { c = 0; ++tau; }
+      }
+      for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
+        mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
+    }
+  } else if (warp == 10) {
+    if (lane == 0) {
+      // dZ tile of each tile visited, the X and X' boxes of each chunk; publishes
+      // this CTA's partial of a split first tile (see the forward).
+      tma_prefetch_desc(&tm_hc);
+      tma_prefetch_desc(&tm_hn);
+      tma_prefetch_desc(&tm_dz);
+      bool publish = cq == 1 && c0 != 0 && n_local > 0;
+      int issued = 0, zissued = 0, tau = tile0, c = c0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+        if (i == 0 || c == 0) {
+          const int v = zissued, zs = v & 1;
+          if (v >= 2 && !mbar_wait(&zempty[zs], ((v >> 1) - 1) & 1, a.err)) break;
+          mbar_arrive_expect_tx(&zfull[zs], 2 * tbytes);
+          tma_load_3d(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j);
+          tma_load_3d(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j);
+          zissued = v + 1;
+        }
+        if (publish && mbar_test(pready, 0)) {
+          red_release_add(a.counters + tile0, 1);
+          publish = false;
+        }
+        const int s = i % nh;
+        if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&hfull[s], 2 * tbytes);
+        tma_load_3d(hb(s), &tm_hc, &hfull[s], c * 64, a.hc_row0, j);
+        tma_load_3d(hb(s) + tbytes, &tm_hn, &hfull[s], c * 64, a.x_row0, j);
+        issued = i + 1;
+        if (++c == nk) { c = 0; ++tau; }
+      }
+      for (int i = issued - nh > 0 ? issued - nh : 0; i < issued; ++i)
+        mbar_wait(&hfull[i % nh], (i / nh) & 1, a.err);
+      for (int v = zissued - 2 > 0 ? zissued - 2 : 0; v < zissued; ++v)
+        mbar_wait(&zfull[v & 1], (v >> 1) & 1, a.err);
+      if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
+    }
+  } else if (warp == 11) {
+    if (lane == 0) {
+      // Store each updated W tile; its slot is released once the TMA has read it
+      // (two stores in flight).
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      int tau = tile0, c = c0, stored = 0;
+      for (int i = 0; i < n_local; ++i) {
+        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+        const int s = i % nw;
+        if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
+        tma_store_3d_hint(&tm_w, wf(s), c * 64, ot * 128, j, stream);
+        tma_store_3d_hint(&tm_w, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
+        tma_store_commit();
+        stored = i + 1;
+        if (i > 0) {
+          tma_store_wait_read_1();
+          mbar_arrive(&wempty[(i - 1) % nw]);
+        }
+        if (++c == nk) { c = 0; ++tau; }
+      }
+      tma_store_wait_all();
+      if (stored > 0) mbar_arrive(&wempty[(stored - 1) % nw]);
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
+    }
+  } else if (warp == 9) {
+    if (lane == 0) {
+      const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
+      const uint32_t idesc_fw = umma_idesc_bf16(128, a.Bn);
+      const int kb = a.Bn / 16;
+      // Forward MMAs of chunk k into accumulator segment qq (first/last: of the segment).
+      auto fwd = [&](int k, bool first, bool last, int qq) -> bool {
+        const int ab = qq & 1, bb = k & 1, sh = k % nh;
+        if (first && qq >= 2 && !mbar_wait(&accr[ab], ((qq >> 1) - 1) & 1, a.err)) return false;
+        if (!mbar_wait(&conv[bb], (k >> 1) & 1, a.err)) return false;
+        tc_fence_after();
+        const uint32_t at = tmem + kUfTmemA + 32 * bb;
+        const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh) + tbytes));
+        const uint32_t d = tmem + 64 * ab;
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk)
+          tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc_fw, (!first || kk > 0) ? 1u : 0u);
+        tc_commit(&hempty[sh]);
+        tc_commit(&afree[bb]);
+        if (last) tc_commit(&accf[ab]);
+        return true;
+      };
+      int c = c0, p = 0, q = -1, zv = -1;
+      int pend = -1, pend_q = 0;
+      bool pend_first = false, pend_last = false, ok = true;
+      for (int i = 0; i < n_local; ++i) {
+        const bool tlast = i == n_local - 1 || c == nk - 1;
+        const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+        if (first) ++q;
+        const int sh = i % nh, bb = i & 1;
+        if (p == 0) {
+          ++zv;
+          if (!mbar_wait(&zfull[zv & 1], (zv >> 1) & 1, a.err)) { ok = false; break; }
+        }
+        if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
+        if (i >= 2 && !mbar_wait(&dwfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t zs = smem_u32(zb(zv & 1)), hs = smem_u32(hb(sh));
+        for (int kk = 0; kk < kb; ++kk)
+          tc_mma_bf16(tmem + kUfTmemDW + 64 * bb, umma_desc_sw128_mn(zs + kk * 2048, tbytes),
+                      umma_desc_sw128_mn(hs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+        tc_commit(&dwdone[bb]);
+        if (tlast) tc_commit(&zempty[zv & 1]);
+        if (pend >= 0 && !fwd(pend, pend_first, pend_last, pend_q)) { ok = false; break; }
+        pend = i;
+        pend_first = first;
+        pend_last = last;
+        pend_q = q;
+        ++p;
+        if (++c == nk) { c = 0; p = 0; }
+      }
+      if (ok && pend >= 0) fwd(pend, pend_first, pend_last, pend_q);
+      tc_commit(done);
+      mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
+    }
+  } else {
+    // ---- warps 0-7: the update, the bf16 A tile, the drains and the tile epilogues
+    const int t = threadIdx.x;
+    const int r = t & 127, gr = t >> 7;                    // accumulator row, column group
+    const int row = 32 * (warp & 3) + lane, half = warp >> 2;   // (row == r)
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+    GroupSync gsync{gbar, 0, a.err};
+    float acc[32];
+#pragma unroll
+    for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+    int qc = -1, drained = 0;
+    auto drain = [&]() -> bool {
+      const int ab = drained & 1;
+      if (!wait_warp(&accf[ab], (drained >> 1) & 1, a.err)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int m = 0; m < 2; ++m) {
+        const int cb = (2 * m + gr) * 16;
+        if (cb < a.Bn) {
+          float v[16];
+          tmem_ld16(tbase + 64 * ab + cb, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 16; ++q) acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v[q]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&accr[ab]);
+      ++drained;
+      return true;
+    };
+    // As the forward's tile_end, hidden layer only: H_1'[j][b][o] = relu(Z' + b_1).
+    auto tile_end = [&](int tau, bool whole, float bias) -> bool {
+      const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+      if (!whole) {
+        if (tau * nk < u0) {
+          float* mine = a.part + (static_cast<int64_t>(g) * 128 + r) * a.Bn;
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int cb = (2 * m + gr) * 16;
+            if (cb < a.Bn) {
+#pragma unroll
+              for (int q = 0; q < 16; q += 4)
+                __stcg(reinterpret_cast<float4*>(mine + cb + q),
+                       make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                                   acc[16 * m + q + 3]));
+            }
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(pready);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+          return true;
+        }
+        const int g_last = cta_of((tau + 1) * nk - 1, U, G);
+        if (t == 0) {
+          const bool ok = spin_acquire_eq(a.counters + tau, g_last - g, a.err);
+          if (ok) a.counters[tau] = 0;
+        }
+        if (!gsync()) return false;
+        for (int gg = g + 1; gg <= g_last; ++gg) {
+          const float* src = a.part + (static_cast<int64_t>(gg) * 128 + r) * a.Bn;
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int cb = (2 * m + gr) * 16;
+            if (cb < a.Bn) {
+#pragma unroll
+              for (int q = 0; q < 16; q += 4) {
+                const float4 v = __ldcg(reinterpret_cast<const float4*>(src + cb + q));
+                acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v.x);
+                acc[16 * m + q + 1] = __fadd_rn(acc[16 * m + q + 1], v.y);
+                acc[16 * m + q + 2] = __fadd_rn(acc[16 * m + q + 2], v.z);
+                acc[16 * m + q + 3] = __fadd_rn(acc[16 * m + q + 3], v.w);
+              }
+            }
+          }
+        }
+      }
+      const int o = ot * 128 + r;
+      if (o < a.out) {
+#pragma unroll
+        for (int m = 0; m < 2; ++m) {
+          const int cb = (2 * m + gr) * 16;
+          if (cb >= a.Bn) break;
+#pragma unroll
+          for (int q = 0; q < 16; ++q)
+            if (cb + q < a.B)
+              a.h_out[(static_cast<int64_t>(j) * a.Bn + cb + q) * a.pitch_out + o] =
+                  __float2bfloat16_rn(fmaxf(__fadd_rn(acc[16 * m + q], bias), 0.f));
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+      return true;
+    };
+    bool ok = true;
+    int tau = tile0, c = c0, p = 0;
+    float tbias = 0.f;
+    int ep_tau = -1;
+    float ep_bias = 0.f;
+    for (int i = 0; i < n_local && ok; ++i) {
+      const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+      const bool tlast = i == n_local - 1 || c == nk - 1;
+      if (p == 0) {
+        const int o = ot * 128 + r;
+        tbias = o < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
+      }
+      const int sw = i % nw, bb = i & 1;
+      if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+      if (!wait_warp(&dwdone[bb], (i >> 1) & 1, a.err)) { ok = false; break; }
+      tc_fence_after();
+      float d[32];
+      tmem_ld16(tbase + kUfTmemDW + 64 * bb + 32 * half, d);
+      tmem_ld16(tbase + kUfTmemDW + 64 * bb + 32 * half + 16, d + 16);
+      tmem_ld_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&dwfree[bb]);
+      // W[o][32*half + 4q ..] sits in 16-byte chunk q ^ (o % 8) of row o of box `half`
+      uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
+      uint32_t pk[16];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4* pw = reinterpret_cast<float4*>(src + ((q ^ (row & 7)) << 4));
+        float4 x = *pw;
+        x.x = __fsub_rn(x.x, __fmul_rn(a.lr, d[4 * q]));
+        x.y = __fsub_rn(x.y, __fmul_rn(a.lr, d[4 * q + 1]));
+        x.z = __fsub_rn(x.z, __fmul_rn(a.lr, d[4 * q + 2]));
+        x.w = __fsub_rn(x.w, __fmul_rn(a.lr, d[4 * q + 3]));
+        *pw = x;
+        pk[2 * q] = pack_bf16x2(x.x, x.y);
+        pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&upd[sw]);
+      if (i >= 2 && !wait_warp(&afree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+      tc_fence_after();
+      tmem_st16(tbase + kUfTmemA + 32 * bb + 16 * half, pk);
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&conv[bb]);
+      if (p % kSegChunks == 0) ++qc;
+      if (tlast) {
+        while (ok && drained <= qc)
+          if (!drain()) ok = false;
+        if (ok && cq > 1) {
+          ep_tau = tau;
+          ep_bias = tbias;
+          if (part != 0) {
+            // the batch ring is idle once the last segment is drained
+            float* red = reinterpret_cast<float*>(h_base) + r * a.Bn;
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+              const int cb = (2 * m + gr) * 16;
+              if (cb < a.Bn) {
+#pragma unroll
+                for (int q = 0; q < 16; q += 4)
+                  *reinterpret_cast<float4*>(red + cb + q) =
+                      make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                                  acc[16 * m + q + 3]);
+              }
+            }
+          }
+        } else if (ok) {
+          const bool whole = (tau != tile0 || c0 == 0) && c == nk - 1;
+          ok = __all_sync(0xffffffffu, tile_end(tau, whole, tbias));
+        }
+      } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
+        if (!drain()) ok = false;
+      }
+      ++p;
+      if (++c == nk) { c = 0; p = 0; ++tau; }
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      if (part == 0 && __all_sync(0xffffffffu, ok && ep_tau >= 0)) {
+        for (int rk = 1; rk < cq; ++rk) {
+          const float* red = reinterpret_cast<const float*>(h_base) + r * a.Bn;
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            const int cb = (2 * m + gr) * 16;
+            if (cb < a.Bn) {
+#pragma unroll
+              for (int q = 0; q < 16; q += 4) {
+                const float4 v = ld_cluster_f4(red + cb + q, rk);
+                acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v.x);
+                acc[16 * m + q + 1] = __fadd_rn(acc[16 * m + q + 1], v.y);
+                acc[16 * m + q + 2] = __fadd_rn(acc[16 * m + q + 2], v.z);
+                acc[16 * m + q + 3] = __fadd_rn(acc[16 * m + q + 3], v.w);
+              }
+            }
+          }
+        }
+        tile_end(ep_tau, true, ep_bias);
+      }
+      cluster_sync_all();
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kUfTmemCols);
+  }
+}
+
 // ------------------------------------------------------------------ gather
 // H_0[j][b][:] = X[j][(t*B + b) mod N][:] for b < B, one CTA per (64-feature slice,
 // learner); rows b >= B stay zero.
@@ -1321,7 +1801,10 @@ cudaError_t tc_configure() {
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_tc_update, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  e = cudaFuncSetAttribute(k_tc_update, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_tc_update_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kFwdSmemMax);
 }
 
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
@@ -1347,6 +1830,14 @@ cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
   // no CTA waits on another: an ordinary (programmatically serialised) launch
   return launch_pdl(k_tc_update, dim3(a.ctas), dim3(kBwdThreads), upd_smem(a.Bn), s, false, 1,
                     w_bwd, h_in, dz, a);
+}
+
+cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_cur,
+                                     const CUtensorMap& x_next, const CUtensorMap& dz,
+                                     const TcFwdArgs& a, cudaStream_t s) {
+  // cooperative in stream-K mode, as the forward
+  return launch_pdl(k_tc_update_forward, dim3(a.ctas), dim3(kUfThreads), uf_smem(a.Bn), s,
+                    a.cq <= 1, a.cq > 1 ? a.cq : 1, w_fwd, h_cur, x_next, dz, a);
 }
 
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,

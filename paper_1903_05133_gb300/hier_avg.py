@@ -17,7 +17,7 @@ from ._lib import c_double, c_int, c_int64, c_void_p, check
 
 PREC = {"fp32": 0, "bf16": 1}
 KERNEL_KINDS = {"gather": 0, "forward": 1, "xent": 2, "backward": 3, "local_avg": 4,
-                "global_avg": 5, "head": 6}
+                "global_avg": 5, "head": 6, "update_forward": 7}
 
 
 def _stream(stream) -> c_void_p:

@@ -88,7 +88,8 @@ def test_calls_before_bind_fail_cleanly(lib):
     assert lib.hier_avg_profile(h, 1) == 0
     assert lib.hier_avg_profile_every(h, 0) == -1
     assert lib.hier_avg_profile_every(h, 7) == 0
-    assert lib.hier_avg_profile_kinds(h, 1 << 7) == -1          # no such kernel kind
+    assert lib.hier_avg_profile_kinds(h, 1 << 8) == -1          # no such kernel kind
+    assert lib.hier_avg_profile_kinds(h, 1 << 7) == 0
     assert lib.hier_avg_profile_kinds(h, (1 << 1) | (1 << 3)) == 0
     assert lib.hier_avg_profile_read(h, 99, None, None, None) == -1
     lib.hier_avg_destroy(h)

@@ -226,6 +226,44 @@ def test_literal_sequence_equals_round():
     assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
 
 
+# Inside round(), a step whose successor starts no local block and reads a contiguous
+# batch also computes that successor's first-layer output (update+forward kernel, same
+# schedule and arithmetic as the forward).  Cases: ragged 192-wide layer in cluster
+# split-K mode; the 16-learner MLP (cluster split-K, cq = 2); 128 tiles in stream-K mode
+# with K1 = 3, so the middle step both consumes and produces a fused H_1.
+FUSE_STREAMK = configs.Workload("mlp_bf16_streamk", P=16, S=4, K1=3, K2=2, rounds=1,
+                                dims=(512, 1024, 10), precision="bf16", N=200, B=32, lr=0.05,
+                                sigma_mu=0.1, init="he")
+
+
+def _fused_steps(w):
+    return sum(1 for t in range(w.K1 * w.K2)
+               if t % w.K1 != w.K1 - 1 and ((t + 1) * w.B) % w.N + w.B <= w.N)
+
+
+@pytest.mark.parametrize("w", [SMALL_BF16, configs.MLP512_P16.replace(N=512), FUSE_STREAMK],
+                         ids=lambda w: w.name)
+def test_fused_next_forward_equals_steps(w):
+    ha1, X, y = setup(w, perturb=(0.01, 0.01))
+    ha2, _, _ = setup(w, perturb=(0.01, 0.01))
+    ha1.profile(["update_forward", "forward"])
+    ha1.round()
+    _, n_fused, _ = ha1.profile_read("update_forward")
+    _, n_fwd, _ = ha1.profile_read("forward")
+    ha1.profile(False)
+    assert n_fused == _fused_steps(w) > 0
+    assert n_fwd == w.K1 * w.K2 - n_fused      # one layer before the head kernel
+    for b in range(w.K2):
+        for k in range(w.K1):
+            ha2.step()
+        ha2.local_average()
+    ha2.global_average()
+    ha1.check()
+    ha2.check()
+    assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
+    assert torch.equal(ha1.losses(), ha2.losses())
+
+
 def _force(ha, *oracles):
     """Load the GPU's current learner state into the oracles (teacher forcing)."""
     state = oracle_params(ha, ha.params)
