@@ -167,36 +167,6 @@ def ncu_traffic(kind: str, workload: str):
     return e.get("dram_bytes_per_launch")
 
 
-def launches_per_round(w) -> int:
-    """Kernel launches of one round (every launch is one of this library's kernels)."""
-    L = len(w.dims) - 1
-    if w.precision == "bf16":
-        steps = range(w.K1 * w.K2)
-        gathers = 0   # the first layer reads X directly unless a batch wraps around N
-        n = 0
-        for t in steps:
-            if (t * w.B) % w.N + w.B > w.N:
-                gathers += 1
-        C, din = w.dims[-1], w.dims[-2]
-        if C <= 16 and din % 64 == 0 and w.B <= 64:      # small last layer: one cluster kernel
-            per_step = (L - 1) + 1 + (L - 1)
-        else:
-            per_step = L + (0 if C <= 128 else 1) + L
-        # inside a local block, a step whose successor reads a contiguous batch also runs
-        # that successor's first-layer forward (one launch fewer)
-        fused = 0
-        if L >= 2:
-            for t in steps:
-                nxt = ((t + 1) * w.B) % w.N
-                if t % w.K1 != w.K1 - 1 and nxt + w.B <= w.N:
-                    fused += 1
-        n = w.K1 * w.K2 * per_step + gathers - fused
-    else:
-        per_step = 1 + L + 1 + L + (L - 1)       # dX is its own launch for layers > 1
-        n = w.K1 * w.K2 * per_step
-    return n + (w.K2 - 1) * (1 if w.S > 1 else 0) + 1
-
-
 # ----------------------------------------------------------------------------- oracle
 def oracle_block_time(w, X, y, layers, n_blocks: int = 1):
     """Time the CPU oracle on one local block (K1 local steps of every learner +
@@ -315,12 +285,14 @@ def run_ours(args):
     if ws > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    launches0 = ha.launches()
     for k in range(args.steps):
         flush.zero_()                      # L2 flushed between timed rounds (not timed)
         starts[k].record()
         ha.round()
         ends[k].record()
     torch.cuda.synchronize()
+    gpu_launches = ha.launches() - launches0   # the library's own count of its kernel launches
     if ws > 1:
         dist.barrier()
     clocks = sampler.stop(uuid)
@@ -382,7 +354,7 @@ def run_ours(args):
             "kernels": kernels,
             "kernels_timing": "untimed profiling pass before the timed rounds, events around every launch",
             "ms_per_step_without_kernel_events": statistics.median(plain_ms),
-            "gpu_launches": launches_per_round(w) * args.steps,
+            "gpu_launches": gpu_launches,
             "clocks": clocks}
 
     # ---- end to end through the C ABI from pinned host memory

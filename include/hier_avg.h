@@ -195,6 +195,10 @@ int hier_avg_profile(hier_avg* h, int enable);
  * reports.  HA_EINVAL for bits beyond HA_KERNEL_KINDS. */
 int hier_avg_profile_kinds(hier_avg* h, unsigned kinds);
 
+/* Kernels this handle has launched since it was created (every launch of the step,
+ * averaging and round calls, one per kernel).  HA_EINVAL for NULL arguments. */
+int hier_avg_launches(const hier_avg* h, int64_t* launches);
+
 /* Time only every n-th launch of each enabled kind (n >= 1, default 1; counted from
  * the last hier_avg_profile / hier_avg_profile_kinds), so that a throughput
  * measurement perturbs few launches.  hier_avg_profile_read then reports the

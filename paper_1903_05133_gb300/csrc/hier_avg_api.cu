@@ -84,6 +84,7 @@ struct hier_avg {
   std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_dz;
   CUtensorMap tm_x;                           // X [P][N][d_0] as the first layer's batch tile
   int64_t t = 0;
+  int64_t launches = 0;                       // kernels launched since bind
   // profiling
   unsigned prof = 0;                          // kinds timed: bit (1 << HA_KERNEL_*)
   int prof_every = 1;                         // time every n-th launch of those kinds
@@ -125,6 +126,7 @@ struct hier_avg {
     cudaEvent_t a = nullptr, b = nullptr;
     bool on = (prof >> kind) & 1u;
     if (on) on = prof_seen[kind]++ % prof_every == 0;
+    ++launches;
     if (on) {
       a = ev();
       b = ev();
@@ -519,6 +521,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     for (int l = L - 1; l >= 0; --l) {
       rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
         cudaError_t e = cudaSuccess;
+        if (l > 0) ++h->launches;   // dX is its own launch
         if (l > 0)
           e = ha::launch_dx_f32(h->wsp<float>(h->off_dZ[l + 1]), h->params + h->woff[l], h->ld,
                                 h->wsp<float>(h->off_H[l]), h->dims[l], h->dims[l + 1], B,
@@ -783,6 +786,12 @@ int hier_avg_check(hier_avg* h) {
     cudaMemsetAsync(h->err_word(), 0, 4, h->stream);
     return h->fail(HA_ETIMEOUT, "a bounded device wait expired (error word %d)", word);
   }
+  return HA_OK;
+}
+
+int hier_avg_launches(const hier_avg* h, int64_t* launches) {
+  if (!h || !launches) return HA_EINVAL;
+  *launches = h->launches;
   return HA_OK;
 }
 

@@ -182,6 +182,12 @@ class HierAvg:
             mask |= 1 << KERNEL_KINDS[k]
         check(self._lib.hier_avg_profile_kinds(self.h, mask), "profile", self.h)
 
+    def launches(self) -> int:
+        """Kernels this handle has launched since it was created."""
+        n = c_int64()
+        check(self._lib.hier_avg_launches(self.h, ctypes.byref(n)), "launches", self.h)
+        return n.value
+
     def profile_every(self, every: int) -> None:
         """Time only every n-th launch of each enabled kind."""
         check(self._lib.hier_avg_profile_every(self.h, int(every)), "profile_every", self.h)

@@ -92,6 +92,10 @@ def test_calls_before_bind_fail_cleanly(lib):
     assert lib.hier_avg_profile_kinds(h, 1 << 7) == 0
     assert lib.hier_avg_profile_kinds(h, (1 << 1) | (1 << 3)) == 0
     assert lib.hier_avg_profile_read(h, 99, None, None, None) == -1
+    n = ctypes.c_int64(-1)
+    assert lib.hier_avg_launches(h, ctypes.byref(n)) == 0 and n.value == 0   # nothing ran
+    assert lib.hier_avg_launches(h, None) == -1
+    assert lib.hier_avg_launches(None, ctypes.byref(n)) == -1
     lib.hier_avg_destroy(h)
     lib.hier_avg_destroy(None)
 

@@ -234,6 +234,11 @@ def test_literal_sequence_equals_round():
 FUSE_STREAMK = configs.Workload("mlp_bf16_streamk", P=16, S=4, K1=3, K2=2, rounds=1,
                                 dims=(512, 1024, 10), precision="bf16", N=200, B=32, lr=0.05,
                                 sigma_mu=0.1, init="he")
+# Three layers: the first layer's update computes the next H_1, the last layer keeps its
+# own kernel (it does not follow the first).
+FUSE_THREE = configs.Workload("mlp3_bf16_fused", P=4, S=2, K1=3, K2=2, rounds=1,
+                              dims=(256, 320, 192, 10), precision="bf16", N=160, B=32, lr=0.05,
+                              sigma_mu=0.1, init="he")
 
 
 def _fused_steps(w):
@@ -241,23 +246,32 @@ def _fused_steps(w):
                if t % w.K1 != w.K1 - 1 and ((t + 1) * w.B) % w.N + w.B <= w.N)
 
 
-@pytest.mark.parametrize("w", [SMALL_BF16, configs.MLP512_P16.replace(N=512), FUSE_STREAMK],
-                         ids=lambda w: w.name)
+@pytest.mark.parametrize("w", [SMALL_BF16, configs.MLP512_P16.replace(N=512), FUSE_STREAMK,
+                               FUSE_THREE], ids=lambda w: w.name)
 def test_fused_next_forward_equals_steps(w):
     ha1, X, y = setup(w, perturb=(0.01, 0.01))
     ha2, _, _ = setup(w, perturb=(0.01, 0.01))
     ha1.profile(["update_forward", "forward"])
+    n0 = ha1.launches()
     ha1.round()
+    n_round = ha1.launches() - n0
     _, n_fused, _ = ha1.profile_read("update_forward")
     _, n_fwd, _ = ha1.profile_read("forward")
     ha1.profile(False)
+    steps, L = w.K1 * w.K2, len(w.dims) - 1
     assert n_fused == _fused_steps(w) > 0
-    assert n_fwd == w.K1 * w.K2 - n_fused      # one layer before the head kernel
+    # forward launches: every layer before the head kernel, less the fused first layers
+    assert n_fwd == steps * (L - 1) - n_fused
+    n1 = ha2.launches()
     for b in range(w.K2):
         for k in range(w.K1):
             ha2.step()
         ha2.local_average()
     ha2.global_average()
+    # the literal sequence launches every kernel; round() saves the fused forwards and
+    # fuses the last local average into the global one
+    saved = n_fused + 1
+    assert ha2.launches() - n1 == n_round + saved
     ha1.check()
     ha2.check()
     assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
