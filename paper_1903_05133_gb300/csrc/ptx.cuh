@@ -148,6 +148,12 @@ __device__ __forceinline__ uint64_t l2_stream_policy(bool evict_first) {
     asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// For small, often re-read tiles next to a streamed W: kept in L2 ahead of other lines.
+__device__ __forceinline__ uint64_t l2_keep_policy() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
 __device__ __forceinline__ void tma_load_3d_hint(void* smem_dst, const void* tmap, uint64_t* bar,
                                                  int c0, int c1, int c2, uint64_t policy) {
   asm volatile(

@@ -1386,14 +1386,17 @@ __global__ void __launch_bounds__(kUfThreads, 1)
       tma_prefetch_desc(&tm_dz);
       bool publish = cq == 1 && c0 != 0 && n_local > 0;
       int issued = 0, zissued = 0, tau = tile0, c = c0;
+      // (the batch and dZ tiles are re-read for every output tile: kept in L2 ahead of
+      // the streamed W)
+      const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
         if (i == 0 || c == 0) {
           const int v = zissued, zs = v & 1;
           if (v >= 2 && !mbar_wait(&zempty[zs], ((v >> 1) - 1) & 1, a.err)) break;
           mbar_arrive_expect_tx(&zfull[zs], 2 * tbytes);
-          tma_load_3d(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j);
-          tma_load_3d(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j);
+          tma_load_3d_hint(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j, keep);
+          tma_load_3d_hint(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j, keep);
           zissued = v + 1;
         }
         if (publish && mbar_test(pready, 0)) {
@@ -1403,8 +1406,8 @@ __global__ void __launch_bounds__(kUfThreads, 1)
         const int s = i % nh;
         if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) break;
         mbar_arrive_expect_tx(&hfull[s], 2 * tbytes);
-        tma_load_3d(hb(s), &tm_hc, &hfull[s], c * 64, a.hc_row0, j);
-        tma_load_3d(hb(s) + tbytes, &tm_hn, &hfull[s], c * 64, a.x_row0, j);
+        tma_load_3d_hint(hb(s), &tm_hc, &hfull[s], c * 64, a.hc_row0, j, keep);
+        tma_load_3d_hint(hb(s) + tbytes, &tm_hn, &hfull[s], c * 64, a.x_row0, j, keep);
         issued = i + 1;
         if (++c == nk) { c = 0; ++tau; }
       }
