@@ -1254,19 +1254,23 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
 // input half w/4) and do the update, the bf16 conversion and the drains; warp 8 loads
 // W tiles, warp 9 issues the MMAs (the dW MMAs of chunk i before the forward MMAs of
 // chunk i-1, so the update of one chunk overlaps the dW of the next), warp 10 loads
-// the batch tiles (X and X' rows of the chunk) and dZ tiles and publishes a split
-// tile's partial, warp 11 stores updated W tiles and frees their slots.
+// the batch tiles (X and X' rows of the chunk) and publishes a split tile's partial,
+// warp 11 stores updated W tiles and frees their slots, warp 12 loads the dZ tile of
+// each tile visited.  A CTA visits few tiles (one in cluster mode, a handful in
+// stream-K mode), so the dZ tile has one buffer and the shared memory goes to a
+// five-deep weight ring.
 constexpr int kUfConv = 256;
-constexpr int kUfThreads = kUfConv + 128;
+constexpr int kUfThreads = kUfConv + 160;
+constexpr int kUfZBufs = 1;     // dZ tile buffers
 // TMEM columns: Z'^T accumulators at 0 and 64, bf16 A tiles at 128 and 160, dW
 // accumulators at 256 and 320.
 constexpr uint32_t kUfTmemCols = 512, kUfTmemA = 128, kUfTmemDW = 256;
 
-// Layout: W ring | 2 dZ tiles ([Bn][128] bf16, two boxes each) | batch ring (X box, X'
+// Layout: W ring | dZ tile(s) ([Bn][128] bf16, two boxes each) | batch ring (X box, X'
 // box per chunk) | barriers.
-__host__ __device__ constexpr int uf_wring(int Bn) { return Bn <= 32 ? 5 : 4; }
+__host__ __device__ constexpr int uf_wring(int Bn) { return (void)Bn, 5; }
 __host__ __device__ constexpr int uf_z_off(int Bn) { return uf_wring(Bn) * kFwdWf32; }
-__host__ __device__ constexpr int uf_h_off(int Bn) { return uf_z_off(Bn) + 2 * 2 * Bn * 128; }
+__host__ __device__ constexpr int uf_h_off(int Bn) { return uf_z_off(Bn) + kUfZBufs * 2 * Bn * 128; }
 __host__ __device__ constexpr int uf_hring(int Bn) {
   return (kFwdSmemMax - 1024 - 512 - uf_h_off(Bn)) / (2 * Bn * 128) < kFwdHRingMax
              ? (kFwdSmemMax - 1024 - 512 - uf_h_off(Bn)) / (2 * Bn * 128)
@@ -1275,7 +1279,7 @@ __host__ __device__ constexpr int uf_hring(int Bn) {
 __host__ __device__ constexpr int uf_bar_off(int Bn) { return uf_h_off(Bn) + uf_hring(Bn) * 2 * Bn * 128; }
 __host__ __device__ constexpr int uf_smem(int Bn) { return uf_bar_off(Bn) + 512 + 1024; }
 // (the cluster split-K partial [128][Bn] fp32 is staged in the batch ring: hring >= 2)
-static_assert(uf_hring(64) >= 4 && uf_hring(48) >= 6 && uf_hring(32) >= 6 && uf_hring(16) == 8 &&
+static_assert(uf_hring(64) >= 3 && uf_hring(48) >= 4 && uf_hring(32) >= 6 && uf_hring(16) == 8 &&
                   uf_smem(64) <= kFwdSmemMax && uf_smem(48) <= kFwdSmemMax &&
                   uf_smem(32) <= kFwdSmemMax && uf_smem(16) <= kFwdSmemMax,
               "update+forward shared-memory plan");
@@ -1304,8 +1308,8 @@ __global__ void __launch_bounds__(kUfThreads, 1)
   uint64_t* upd = wempty + kFwdWRingMax;     // W tile updated in shared memory
   uint64_t* hfull = upd + kFwdWRingMax;
   uint64_t* hempty = hfull + kFwdHRingMax;   // X and X' boxes consumed by both MMAs
-  uint64_t* zfull = hempty + kFwdHRingMax;   // [2]
-  uint64_t* zempty = zfull + 2;              // [2] dZ tile consumed by the tile's dW MMAs
+  uint64_t* zfull = hempty + kFwdHRingMax;   // [kUfZBufs <= 2]
+  uint64_t* zempty = zfull + 2;              // [..] dZ tile consumed by the tile's dW MMAs
   uint64_t* dwdone = zempty + 2;             // [2] dW of the chunk complete
   uint64_t* dwfree = dwdone + 2;             // [2] dW read by the update
   uint64_t* conv = dwfree + 2;               // [2] A tile written to TMEM
@@ -1379,26 +1383,17 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     }
   } else if (warp == 10) {
     if (lane == 0) {
-      // dZ tile of each tile visited, the X and X' boxes of each chunk; publishes
-      // this CTA's partial of a split first tile (see the forward).
+      // The X and X' boxes of each chunk; publishes this CTA's partial of a split first
+      // tile (see the forward).
       tma_prefetch_desc(&tm_hc);
       tma_prefetch_desc(&tm_hn);
-      tma_prefetch_desc(&tm_dz);
       bool publish = cq == 1 && c0 != 0 && n_local > 0;
-      int issued = 0, zissued = 0, tau = tile0, c = c0;
+      int issued = 0, tau = tile0, c = c0;
       // (the batch and dZ tiles are re-read for every output tile: kept in L2 ahead of
       // the streamed W)
       const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
       for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-        if (i == 0 || c == 0) {
-          const int v = zissued, zs = v & 1;
-          if (v >= 2 && !mbar_wait(&zempty[zs], ((v >> 1) - 1) & 1, a.err)) break;
-          mbar_arrive_expect_tx(&zfull[zs], 2 * tbytes);
-          tma_load_3d_hint(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j, keep);
-          tma_load_3d_hint(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j, keep);
-          zissued = v + 1;
-        }
+        const int j = tau / a.o_tiles;
         if (publish && mbar_test(pready, 0)) {
           red_release_add(a.counters + tile0, 1);
           publish = false;
@@ -1413,9 +1408,30 @@ __global__ void __launch_bounds__(kUfThreads, 1)
       }
       for (int i = issued - nh > 0 ? issued - nh : 0; i < issued; ++i)
         mbar_wait(&hfull[i % nh], (i / nh) & 1, a.err);
-      for (int v = zissued - 2 > 0 ? zissued - 2 : 0; v < zissued; ++v)
-        mbar_wait(&zfull[v & 1], (v >> 1) & 1, a.err);
       if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+    }
+    if (cq > 1) {
+      cluster_sync_all();
+      cluster_sync_all();
+    }
+  } else if (warp == 12) {
+    if (lane == 0 && n_local > 0) {
+      // The dZ tile (128 outputs x Bn) of each tile this CTA visits.
+      tma_prefetch_desc(&tm_dz);
+      const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
+      const int n_visits = (u1 - 1) / nk - tile0 + 1;
+      int zissued = 0;
+      for (int v = 0; v < n_visits; ++v) {
+        const int tau = tile0 + v, j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+        const int zs = v % kUfZBufs;
+        if (v >= kUfZBufs && !mbar_wait(&zempty[zs], ((v / kUfZBufs) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&zfull[zs], 2 * tbytes);
+        tma_load_3d_hint(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j, keep);
+        tma_load_3d_hint(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j, keep);
+        zissued = v + 1;
+      }
+      for (int v = zissued - kUfZBufs > 0 ? zissued - kUfZBufs : 0; v < zissued; ++v)
+        mbar_wait(&zfull[v % kUfZBufs], (v / kUfZBufs) & 1, a.err);
     }
     if (cq > 1) {
       cluster_sync_all();
@@ -1480,17 +1496,17 @@ __global__ void __launch_bounds__(kUfThreads, 1)
         const int sh = i % nh, bb = i & 1;
         if (p == 0) {
           ++zv;
-          if (!mbar_wait(&zfull[zv & 1], (zv >> 1) & 1, a.err)) { ok = false; break; }
+          if (!mbar_wait(&zfull[zv % kUfZBufs], (zv / kUfZBufs) & 1, a.err)) { ok = false; break; }
         }
         if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
         if (i >= 2 && !mbar_wait(&dwfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t zs = smem_u32(zb(zv & 1)), hs = smem_u32(hb(sh));
+        const uint32_t zs = smem_u32(zb(zv % kUfZBufs)), hs = smem_u32(hb(sh));
         for (int kk = 0; kk < kb; ++kk)
           tc_mma_bf16(tmem + kUfTmemDW + 64 * bb, umma_desc_sw128_mn(zs + kk * 2048, tbytes),
                       umma_desc_sw128_mn(hs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
         tc_commit(&dwdone[bb]);
-        if (tlast) tc_commit(&zempty[zv & 1]);
+        if (tlast) tc_commit(&zempty[zv % kUfZBufs]);
         if (pend >= 0 && !fwd(pend, pend_first, pend_last, pend_q)) { ok = false; break; }
         pend = i;
         pend_first = first;
