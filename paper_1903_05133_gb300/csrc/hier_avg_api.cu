@@ -344,8 +344,11 @@ ha::HeadArgs head_args(hier_avg* h) {
 // One step.  h1_ready: H_1 of this step was written by the previous step's
 // update+forward kernel (skip the first layer's forward).  fuse_next: the caller runs
 // the next step right after this one with nothing in between, so this step may
-// compute the next step's H_1; *fused reports whether it did.
-int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr) {
+// compute the next step's H_1; *fused reports whether it did.  shared: the caller has
+// just averaged each local cluster, so its S learners hold identical parameters and
+// the forwards read one copy per cluster (the same values: results are unchanged).
+int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
+            bool shared = false) {
   const int L = h->L, P = h->P, B = h->B;
   if (fused) *fused = false;
   cudaStream_t s = h->stream;
@@ -380,6 +383,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.counters = h->wsp<int>(h->off_cnt);
       a.x_direct = (l == 0 && x_direct) ? 1 : 0;
       a.w_stream = h->w_stream ? 1 : 0;
+      a.share = shared ? h->S : 1;
       a.x_row0 = static_cast<int>(r0);
       if (l + 1 < L) {
         a.mode = 0;
@@ -555,7 +559,8 @@ int do_round(hier_avg* h) {
   for (int b = 0; b < h->K2; ++b) {
     bool h1_ready = false;
     for (int k = 0; k < h->K1; ++k)
-      if ((rc = do_step(h, h1_ready, k + 1 < h->K1, &h1_ready))) return rc;
+      // the block's first step follows a local average (except the round's first block)
+      if ((rc = do_step(h, h1_ready, k + 1 < h->K1, &h1_ready, b > 0 && k == 0))) return rc;
     if (b + 1 < h->K2 && (rc = do_local(h))) return rc;
   }
   return do_local_global(h);

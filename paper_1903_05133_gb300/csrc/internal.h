@@ -97,6 +97,8 @@ struct TcFwdArgs {
   int x_direct, x_row0;
   int hc_row0;                // update+forward: rows of this step's batch in its map
   int w_stream;               // load W with the L2 evict-first policy
+  int share;                  // > 1: learners [g*share, (g+1)*share) hold identical W (right
+                              // after an average): all read learner g*share's copy
   // mode 2: labels and outputs of the fused cross-entropy
   const int32_t* y;
   int64_t N, t;

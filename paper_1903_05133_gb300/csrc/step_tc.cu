@@ -264,11 +264,13 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       int issued = 0, tau = tile0, c = c0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+        // learners whose rows are identical (a.share > 1) read one copy: the group's first
+        const int jw = a.share > 1 ? (j / a.share) * a.share : j;
         const int s = i % nw;
         if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) break;
         mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
-        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j, stream);
-        tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j, stream);
+        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, jw, stream);
+        tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, jw, stream);
         issued = i + 1;
         if (++c == nk) { c = 0; ++tau; }
       }
