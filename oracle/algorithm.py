@@ -12,6 +12,15 @@ The global step counter t counts local SGD steps from 0 and continues across
 rounds.  Reading of "randomly sample a mini-batch": the per-learner data are i.i.d.
 draws, so learner j at step t takes rows (t*B + s) mod N, s = 0..B-1, of its own
 data set.
+
+Sec. 3.1 takes the global interval K1 * beta with beta an integer for the analysis
+and leaves it free in practice (the ImageNet run of Sec. 4 uses 43 local steps per
+global average with K1 = 20).  Reading of a free global interval of G local steps:
+within a round, every K1-th step is followed by a local average (counting from the
+round's start, as Algorithm 1's loops do), and the round's G-th step by the global
+average, preceded by a local average exactly when K1 divides G.  G = K1 * beta is
+Algorithm 1 itself.  The step size gamma_n of round n (Theorem 3.3's diminishing
+schedules) is ``lr`` at the time of the round's steps.
 """
 from __future__ import annotations
 
@@ -30,9 +39,13 @@ def batch_rows(t: int, B: int, N: int) -> np.ndarray:
 
 class HierAvgOracle:
     def __init__(self, P: int, S: int, K1: int, K2: int, lr: float, problem,
-                 params: List[np.ndarray], mode: str = "fp32"):
+                 params: List[np.ndarray], mode: str = "fp32", global_steps: int = 0):
         if min(P, S, K1, K2) < 1 or P % S != 0:
             raise ValueError("need P, S, K1, K2 >= 1 and S | P")
+        if global_steps < 0:
+            raise ValueError("global_steps must be >= 0 (0: K1 * K2)")
+        # local SGD steps per global round
+        self.G = global_steps if global_steps > 0 else K1 * K2
         for p in params:
             if p.shape[0] != P:
                 raise ValueError("every parameter array must have leading axis P")
@@ -60,8 +73,10 @@ class HierAvgOracle:
             global_average(p)
 
     def round(self) -> None:
-        for _b in range(self.K2):
-            for _k in range(self.K1):
-                self.step()
-            self.local_average()
+        """One global round: G local steps, a local average after every K1-th of them,
+        then the global average (Algorithm 1 when G = K1 * K2)."""
+        for r in range(1, self.G + 1):
+            self.step()
+            if r % self.K1 == 0:
+                self.local_average()
         self.global_average()

@@ -147,6 +147,68 @@ def test_quadratic_closed_form(P, S, K1, K2):
         assert np.allclose(o.params[0], wt, rtol=0, atol=1e-12)
 
 
+@pytest.mark.parametrize("P,S,K1,G", [(8, 4, 20, 43), (8, 2, 3, 7), (4, 2, 5, 5), (6, 3, 4, 2),
+                                      (8, 1, 3, 8), (12, 4, 2, 9)])
+def test_quadratic_free_global_interval(P, S, K1, G):
+    # Free global interval of G local steps (Sec. 3.1; Sec. 4's ImageNet run: K1 = 20,
+    # G = 43) and a diminishing step size gamma_n = gamma_0 / (n + 1) (Theorem 3.3).
+    # With f_j(w) = 0.5 ||w - c_j||^2 and q = G // K1 local averages inside the round
+    # (r = 1 - gamma_n): after the b-th, cluster C holds cbar_C + r^(b K1) (w~ - cbar_C);
+    # before the global average learner j holds c_j + r^(G - q K1) (w_C - c_j), where
+    # w_C is its cluster's value after the q-th average (w~ if q = 0); and the round
+    # maps w~ - cbar to r^G (w~ - cbar).
+    D, gamma0 = 4, 0.25
+    rng = np.random.default_rng(P + S + K1 + G)
+    c = rng.standard_normal((P, D))
+    w0 = rng.standard_normal(D)
+    o = HierAvgOracle(P, S, K1, 1, gamma0, QuadraticProblem(c),
+                      [np.broadcast_to(w0, (P, D)).copy()], "f64", global_steps=G)
+    assert o.G == G
+    q, rem = divmod(G, K1)
+    wt = w0.copy()
+    cbar = c.mean(axis=0)
+    cl = np.repeat(c.reshape(P // S, S, D).mean(axis=1), S, axis=0)   # cbar of j's cluster
+    for n in range(3):
+        o.lr = gamma0 / (n + 1)
+        r = 1.0 - o.lr
+        for step in range(1, G + 1):
+            o.step()
+            if step % K1 == 0:
+                o.local_average()
+                b = step // K1
+                assert np.allclose(o.params[0], cl + r ** (b * K1) * (wt - cl), rtol=0, atol=1e-12)
+        wc = cl + r ** (q * K1) * (wt - cl) if q > 0 else np.broadcast_to(wt, (P, D))
+        assert np.allclose(o.params[0], c + r ** rem * (wc - c), rtol=0, atol=1e-12)
+        o.global_average()
+        wt = cbar + r ** G * (wt - cbar)
+        assert np.allclose(o.params[0], wt, rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("K1,G", [(20, 43), (3, 7), (4, 2)])
+def test_round_with_free_interval_follows_its_definition(K1, G):
+    # round() = G steps with a local average after every K1-th and the global average
+    # at the end; checked against the same sequence of calls on a second oracle (MLP).
+    P, S, dims, N, B = 4, 2, (12, 8, 5), 40, 4
+    X, y, params = _mlp_setup(P, dims, N, B, seed=5)
+    o1 = HierAvgOracle(P, S, K1, 1, 0.05, MLPProblem(X, y, B, 2, "fp32"), params, "fp32",
+                       global_steps=G)
+    o2 = HierAvgOracle(P, S, K1, 1, 0.05, MLPProblem(X, y, B, 2, "fp32"), params, "fp32")
+    o1.round()
+    for step in range(1, G + 1):
+        o2.step()
+        if step % K1 == 0:
+            o2.local_average()
+    o2.global_average()
+    assert o1.t == o2.t == G
+    for a, b in zip(o1.params, o2.params):
+        assert np.array_equal(a, b)
+
+
+def test_default_global_interval_is_k1_times_k2():
+    o = HierAvgOracle(4, 2, 3, 5, 0.1, None, [np.zeros((4, 2))])
+    assert o.G == 15
+
+
 def test_batch_rows_cycle():
     # mini-batch of step t: rows (t*B + s) mod N
     assert list(batch_rows(0, 4, 10)) == [0, 1, 2, 3]
@@ -154,6 +216,8 @@ def test_batch_rows_cycle():
 
 
 def test_rejects_bad_config():
+    with pytest.raises(ValueError):
+        HierAvgOracle(4, 2, 1, 1, 0.1, None, [np.zeros((4, 2))], global_steps=-1)
     with pytest.raises(ValueError):
         HierAvgOracle(6, 4, 1, 1, 0.1, None, [np.zeros((6, 2))])
     with pytest.raises(ValueError):
