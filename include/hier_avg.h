@@ -133,6 +133,18 @@ int hier_avg_global_average(hier_avg* h);
  * hier_avg_step in turn. */
 int hier_avg_round(hier_avg* h);
 
+/* Global averaging interval in local steps: hier_avg_round then runs `steps` local
+ * steps, a local average after every K1-th of them, and the global average after the
+ * last, preceded by a local average exactly when K1 divides `steps`.  Sec. 3.1 takes
+ * the interval K1 * beta with beta an integer for the analysis and leaves it free in
+ * practice (Sec. 4's ImageNet run: K1 = 20, 43 steps).  0 restores K1 * K2 (the
+ * default).  HA_EINVAL for steps < 0 or a NULL handle. */
+int hier_avg_set_global_steps(hier_avg* h, int steps);
+
+/* Step size of the following local steps (the gamma_n of round n; Theorem 3.3's
+ * diminishing schedules set it between rounds).  HA_EINVAL if lr is not finite. */
+int hier_avg_set_lr(hier_avg* h, float lr);
+
 /* One round end to end from host memory: copies the rows this round reads from
  * X_host [P, N, d_0] / y_host [P, N] (pinned memory recommended) into the bound
  * device data set, runs hier_avg_round, and copies the per-learner loss of the

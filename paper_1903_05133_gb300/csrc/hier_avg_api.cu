@@ -55,6 +55,7 @@ struct hier_avg {
   // configuration (Sec. 2 notation)
   int P = 0, S = 0, K1 = 0, K2 = 0, B = 0, L = 0, prec = 0;
   float lr = 0.f;
+  int G = 0;                                  // local steps per global round (0: K1 * K2)
   std::vector<int> dims;
   // parameter row layout
   int64_t D = 0, ld = 0;
@@ -554,16 +555,29 @@ int do_local_global(hier_avg* h) {
   }, "local+global average");
 }
 
+int do_global(hier_avg* h) {
+  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, [&] {
+    return ha::launch_group_mean(h->params, h->P, h->P, h->ld, h->ld, h->stream);
+  }, "global average");
+}
+
+int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
+
+// One global round (Algorithm 1, Sec. 3.1): G local steps, a local average after every
+// K1-th, the global average after the G-th (fused with the local average that closes
+// the round when K1 divides G).  G = K1 * K2 unless set: Sec. 3.1 leaves beta = G / K1
+// free in practice.
 int do_round(hier_avg* h) {
   int rc;
-  for (int b = 0; b < h->K2; ++b) {
-    bool h1_ready = false;
-    for (int k = 0; k < h->K1; ++k)
-      // the block's first step follows a local average (except the round's first block)
-      if ((rc = do_step(h, h1_ready, k + 1 < h->K1, &h1_ready, b > 0 && k == 0))) return rc;
-    if (b + 1 < h->K2 && (rc = do_local(h))) return rc;
+  const int G = round_steps(h);
+  bool h1_ready = false;
+  for (int r = 1; r <= G; ++r) {
+    const bool block_end = r % h->K1 == 0;              // a local average follows step r
+    const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
+    if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local))) return rc;
+    if (r < G && block_end && (rc = do_local(h))) return rc;
   }
-  return do_local_global(h);
+  return G % h->K1 == 0 ? do_local_global(h) : do_global(h);
 }
 
 }  // namespace
@@ -719,9 +733,7 @@ int hier_avg_local_average(hier_avg* h) {
 
 int hier_avg_global_average(hier_avg* h) {
   if (int rc = check_bound(h)) return rc;
-  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, [&] {
-    return ha::launch_group_mean(h->params, h->P, h->P, h->ld, h->ld, h->stream);
-  }, "global average");
+  return do_global(h);
 }
 
 int hier_avg_round(hier_avg* h) {
@@ -734,7 +746,7 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
   if (!X_host || !y_host || !loss_host) return h->fail(HA_EINVAL, "round_host: NULL host buffer");
   const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
   const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
-  const int64_t rows = static_cast<int64_t>(h->B) * h->K1 * h->K2;
+  const int64_t rows = static_cast<int64_t>(h->B) * round_steps(h);
   int64_t r0 = (h->t * h->B) % h->N, left = rows < h->N ? rows : h->N;
   if (rows >= h->N) r0 = 0;
   while (left > 0) {   // at most two contiguous row ranges per learner (wrap-around)
@@ -757,6 +769,18 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
                                        h->stream), "round_host: loss copy"))
     return rc;
   return hier_avg_check(h);
+}
+
+int hier_avg_set_global_steps(hier_avg* h, int steps) {
+  if (!h || steps < 0) return HA_EINVAL;
+  h->G = steps;
+  return HA_OK;
+}
+
+int hier_avg_set_lr(hier_avg* h, float lr) {
+  if (!h || !std::isfinite(lr)) return HA_EINVAL;
+  h->lr = lr;
+  return HA_OK;
 }
 
 int hier_avg_get_step(const hier_avg* h, int64_t* t) {

@@ -182,6 +182,15 @@ class HierAvg:
             mask |= 1 << KERNEL_KINDS[k]
         check(self._lib.hier_avg_profile_kinds(self.h, mask), "profile", self.h)
 
+    def set_global_steps(self, steps: int) -> None:
+        """Local steps per global average (0: K1 * K2); see hier_avg_set_global_steps."""
+        check(self._lib.hier_avg_set_global_steps(self.h, int(steps)), "set_global_steps", self.h)
+
+    def set_lr(self, lr: float) -> None:
+        """Step size of the following local steps (per-round schedules)."""
+        check(self._lib.hier_avg_set_lr(self.h, float(lr)), "set_lr", self.h)
+        self.lr = float(lr)
+
     def launches(self) -> int:
         """Kernels this handle has launched since it was created."""
         n = c_int64()

@@ -92,6 +92,11 @@ def test_calls_before_bind_fail_cleanly(lib):
     assert lib.hier_avg_profile_kinds(h, 1 << 7) == 0
     assert lib.hier_avg_profile_kinds(h, (1 << 1) | (1 << 3)) == 0
     assert lib.hier_avg_profile_read(h, 99, None, None, None) == -1
+    assert lib.hier_avg_set_global_steps(h, -1) == -1
+    assert lib.hier_avg_set_global_steps(h, 43) == 0 and lib.hier_avg_set_global_steps(h, 0) == 0
+    assert lib.hier_avg_set_global_steps(None, 5) == -1
+    assert lib.hier_avg_set_lr(h, float("nan")) == -1 and lib.hier_avg_set_lr(h, float("inf")) == -1
+    assert lib.hier_avg_set_lr(h, 0.01) == 0
     n = ctypes.c_int64(-1)
     assert lib.hier_avg_launches(h, ctypes.byref(n)) == 0 and n.value == 0   # nothing ran
     assert lib.hier_avg_launches(h, None) == -1

@@ -278,6 +278,57 @@ def test_fused_next_forward_equals_steps(w):
     assert torch.equal(ha1.losses(), ha2.losses())
 
 
+# Free global interval (Sec. 3.1: beta = G / K1 need not be an integer; Sec. 4's ImageNet
+# run uses K1 = 20 and G = 43) with a diminishing step size gamma_n = gamma_0 / (n + 1)
+# (Theorem 3.3), two rounds each, against the oracle.
+FREE_G = [(SMALL_FP32, 5), (SMALL_BF16, 3), (FUSE_THREE, 7), (SMALL_BF16.replace(K1=3), 7)]
+
+
+@pytest.mark.parametrize("w,G", FREE_G, ids=lambda v: getattr(v, "name", str(v)))
+def test_free_global_interval_against_oracle(w, G):
+    ha, X, y = setup(w)
+    ha.set_global_steps(G)
+    start = oracle_params(ha, ha.params)
+    o = make_oracle(w, ha, X, y, start)
+    o.G = G
+    o_ref = (make_oracle(w, ha, X, y, start, mode="bf16_acc32") if w.precision == "bf16" else None)
+    if o_ref is not None:
+        o_ref.G = G
+    for n in range(2):
+        lr = w.lr / (n + 1)
+        ha.set_lr(lr)
+        for oo in (o, o_ref):
+            if oo is not None:
+                oo.lr = lr
+                oo.round()
+        ha.round()
+    ha.check()
+    compare(ha, o, o_ref=o_ref)
+    p = ha.params.cpu().numpy().view(np.uint32)
+    assert np.all(p == p[0])                      # the round ends with the global average
+    assert ha.get_step() == 2 * G
+
+
+@pytest.mark.parametrize("w,G", [(SMALL_BF16.replace(K1=3), 7), (FUSE_THREE, 6)],
+                         ids=lambda v: getattr(v, "name", str(v)))
+def test_free_global_interval_literal_sequence(w, G):
+    # round() with G steps equals the calls it stands for, bit for bit: a local average
+    # after every K1-th step, the global average after the G-th (preceded by a local
+    # average exactly when K1 divides G)
+    ha1, X, y = setup(w, perturb=(0.01, 0.01))
+    ha2, _, _ = setup(w, perturb=(0.01, 0.01))
+    ha1.set_global_steps(G)
+    ha1.round()
+    for r in range(1, G + 1):
+        ha2.step()
+        if r % w.K1 == 0:
+            ha2.local_average()
+    ha2.global_average()
+    ha1.check()
+    ha2.check()
+    assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
+
+
 def _force(ha, *oracles):
     """Load the GPU's current learner state into the oracles (teacher forcing)."""
     state = oracle_params(ha, ha.params)
