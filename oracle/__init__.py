@@ -21,10 +21,10 @@ contain unknown constants (L, M, M_G) and are not computed here.
 from .averaging import tree_sum, group_mean, local_average, global_average
 from .learner import (bf16_round, softmax_xent_grad, mlp_forward_backward, sgd_update,
                       MLPProblem, QuadraticProblem)
-from .algorithm import HierAvgOracle, batch_rows
+from .algorithm import HierAvgOracle, batch_rows, batch_rows_from
 
 __all__ = [
     "tree_sum", "group_mean", "local_average", "global_average",
     "bf16_round", "softmax_xent_grad", "mlp_forward_backward", "sgd_update",
-    "MLPProblem", "QuadraticProblem", "HierAvgOracle", "batch_rows",
+    "MLPProblem", "QuadraticProblem", "HierAvgOracle", "batch_rows", "batch_rows_from",
 ]

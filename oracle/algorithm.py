@@ -19,8 +19,11 @@ global average with K1 = 20).  Reading of a free global interval of G local step
 within a round, every K1-th step is followed by a local average (counting from the
 round's start, as Algorithm 1's loops do), and the round's G-th step by the global
 average, preceded by a local average exactly when K1 divides G.  G = K1 * beta is
-Algorithm 1 itself.  The step size gamma_n of round n (Theorem 3.3's diminishing
-schedules) is ``lr`` at the time of the round's steps.
+Algorithm 1 itself.  The step size gamma_n and batch size B_n of round n (Theorem
+3.3's diminishing step sizes and growing batches) are ``lr`` and ``B`` at the time of
+the round's steps.  With a batch size that changes, each learner reads its data
+sequentially: the batch of a step starts where the previous one ended, at row
+(sum of the earlier steps' batch sizes) mod N, which is t * B for a constant B.
 """
 from __future__ import annotations
 
@@ -33,8 +36,13 @@ from .learner import sgd_update
 
 
 def batch_rows(t: int, B: int, N: int) -> np.ndarray:
-    """Row indices of the mini-batch at local step t."""
-    return (t * B + np.arange(B)) % N
+    """Row indices of the mini-batch at local step t (constant batch size B)."""
+    return batch_rows_from(t * B, B, N)
+
+
+def batch_rows_from(start: int, B: int, N: int) -> np.ndarray:
+    """Row indices of a mini-batch of B rows that starts at row `start` (mod N)."""
+    return (start + np.arange(B)) % N
 
 
 class HierAvgOracle:
@@ -54,15 +62,20 @@ class HierAvgOracle:
         dt = np.float64 if mode == "f64" else np.float32
         self.params = [np.array(p, dtype=dt, copy=True) for p in params]
         self.t = 0
+        self.B = getattr(problem, "B", 0)       # batch size of the following steps
+        self.cursor = 0                         # rows read so far (per learner)
 
     def step(self) -> None:
         """One local SGD step on every learner (Algorithm 1, innermost loop)."""
+        X = getattr(self.problem, "X", None)
+        rows = None if X is None else batch_rows_from(self.cursor, self.B, X.shape[1])
         for j in range(self.P):
             pj = [p[j] for p in self.params]
-            grads = self.problem.gradients(j, self.t, pj)
+            grads = self.problem.gradients(j, rows, pj)
             for p, g in zip(self.params, grads):
                 p[j] = sgd_update(p[j], g, self.lr, self.mode)
         self.t += 1
+        self.cursor += self.B
 
     def local_average(self) -> None:
         for p in self.params:

@@ -137,16 +137,15 @@ class MLPProblem:
     """Learner j's mini-batch gradient of the MLP objective on its own data.
 
     X [P, N, d_0] (float values; bf16 data passed as its exact fp32 values),
-    y [P, N] integer labels.  The rows of step t are chosen by ``batch_rows``."""
+    y [P, N] integer labels; B is the default batch size.  A step's rows are chosen by
+    the caller (``batch_rows_from``)."""
 
     def __init__(self, X: np.ndarray, y: np.ndarray, B: int, n_layers: int, mode: str):
         self.X, self.y, self.B, self.L, self.mode = X, y, B, n_layers, mode
         self.last_loss = np.zeros(X.shape[0])
         self.last_preacts: dict = {}
 
-    def gradients(self, j: int, t: int, params_j: List[np.ndarray]) -> List[np.ndarray]:
-        from .algorithm import batch_rows
-        rows = batch_rows(t, self.B, self.X.shape[1])
+    def gradients(self, j: int, rows: np.ndarray, params_j: List[np.ndarray]) -> List[np.ndarray]:
         Ws, bs = params_j[0::2], params_j[1::2]
         pre: list = []
         loss, gW, gb = mlp_forward_backward(Ws, bs, self.X[j, rows], self.y[j, rows], self.mode,
@@ -167,5 +166,5 @@ class QuadraticProblem:
         self.c = np.asarray(c, dtype=np.float64)
         self.mode = "f64"
 
-    def gradients(self, j: int, t: int, params_j: List[np.ndarray]) -> List[np.ndarray]:
+    def gradients(self, j: int, rows, params_j: List[np.ndarray]) -> List[np.ndarray]:
         return [params_j[0] - self.c[j]]

@@ -6,7 +6,7 @@ import numpy as np
 import pytest
 import torch
 
-from oracle import HierAvgOracle, MLPProblem, QuadraticProblem, batch_rows
+from oracle import HierAvgOracle, MLPProblem, QuadraticProblem, batch_rows, batch_rows_from
 from oracle import learner as ln
 
 
@@ -53,6 +53,32 @@ def test_sync_sgd_special_case(P, S):
             assert np.allclose(got[j], w, rtol=1e-12, atol=1e-13)
 
 
+def test_sync_sgd_with_growing_batch():
+    # Theorem 3.3's growing batch: round n uses B_n rows per learner, read where the
+    # previous step's batch ended.  With K1 = 1, S = P the round is one step of
+    # minibatch SGD on the P * B_n rows (torch autograd, independent of the oracle),
+    # including the wrap past the end of the data.
+    P, dims, N, lr = 4, (6, 5, 3), 20, 0.1
+    X, y, params = _mlp_setup(P, dims, N, 4, seed=11)
+    o = HierAvgOracle(P, P, 1, 1, lr, MLPProblem(X, y, 4, 2, "f64"), params, "f64")
+    start, cur = 0, [p.copy() for p in params]
+    for Bn in (2, 3, 5, 8, 7):
+        o.B = Bn
+        o.round()
+        want = _torch_big_batch_step(cur, X, y, batch_rows_from(start, Bn, N), lr, dims)
+        start += Bn
+        for got, w in zip(o.params, want):
+            for j in range(P):
+                assert np.allclose(got[j], w, rtol=1e-12, atol=1e-13)
+        cur = [p.copy() for p in o.params]
+    assert o.cursor == 25 and o.t == 5
+
+
+def test_batch_rows_from_continues_a_cursor():
+    assert list(batch_rows_from(18, 4, 20)) == [18, 19, 0, 1]
+    assert list(batch_rows_from(8, 4, 10)) == list(batch_rows(2, 4, 10))
+
+
 def _kavg(params, problem, P, K, lr, rounds):
     """K-AVG written independently: K local steps per learner, then the mean over
     learners (numpy mean, not the oracle's tree)."""
@@ -61,7 +87,8 @@ def _kavg(params, problem, P, K, lr, rounds):
     for _ in range(rounds):
         for _k in range(K):
             for j in range(P):
-                g = problem.gradients(j, t, [p[j] for p in ps])
+                g = problem.gradients(j, batch_rows(t, problem.B, problem.X.shape[1]),
+                                      [p[j] for p in ps])
                 for p, gg in zip(ps, g):
                     p[j] = p[j] - lr * gg
             t += 1
