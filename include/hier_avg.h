@@ -145,6 +145,13 @@ int hier_avg_set_global_steps(hier_avg* h, int steps);
  * diminishing schedules set it between rounds).  HA_EINVAL if lr is not finite. */
 int hier_avg_set_lr(hier_avg* h, float lr);
 
+/* Mini-batch size of the following local steps (the B_n of round n; Theorem 3.3's
+ * growing batches), 1 <= B <= the B given at create (which sizes the buffers).  Each
+ * learner reads its data sequentially: a step's batch starts where the previous one
+ * ended, at row (rows read so far) mod N, which is t * B for a constant B.
+ * HA_EINVAL outside that range; HA_ECUDA if clearing device buffers fails. */
+int hier_avg_set_batch(hier_avg* h, int B);
+
 /* One round end to end from host memory: copies the rows this round reads from
  * X_host [P, N, d_0] / y_host [P, N] (pinned memory recommended) into the bound
  * device data set, runs hier_avg_round, and copies the per-learner loss of the
@@ -175,7 +182,8 @@ int hier_avg_step_static(hier_avg* h, float* params_dev, const void* X_dev,
                          const int32_t* y_dev, int64_t N, void* stream);
 
 /* Step counter t (local SGD steps taken); setting it resumes a run whose
- * parameters were saved, since the mini-batch is a function of t only. */
+ * parameters were saved: it also sets the rows read so far to t * B (the current
+ * batch size), which is where a run with a constant batch size stands. */
 int hier_avg_get_step(const hier_avg* h, int64_t* t);
 int hier_avg_set_step(hier_avg* h, int64_t t);
 

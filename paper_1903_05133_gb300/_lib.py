@@ -43,6 +43,7 @@ SIGNATURES = {
     "hier_avg_launches": (c_int, [c_void_p, c_void_p]),
     "hier_avg_set_global_steps": (c_int, [c_void_p, c_int]),
     "hier_avg_set_lr": (c_int, [c_void_p, ctypes.c_float]),
+    "hier_avg_set_batch": (c_int, [c_void_p, c_int]),
     "hier_avg_profile_every": (c_int, [c_void_p, c_int]),
     "hier_avg_profile_read": (c_int, [c_void_p, c_int, P_double, P_int64, P_double]),
     "hier_avg_strerror": (c_char_p, [c_int]),

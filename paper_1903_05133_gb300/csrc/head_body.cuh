@@ -28,7 +28,7 @@ constexpr int kGA = kHeadMaxC + 8;            // g_q   [b][c] row stride (bf16)
 constexpr int kGT = 64 + 8;                   // g_q^T [c][b] row stride (bf16)
 
 __device__ __forceinline__ const __nv_bfloat16* head_row(const HeadArgs& a, int j, int b) {
-  if (a.x_rows) return a.H + (static_cast<int64_t>(j) * a.N + (a.t * a.B + b) % a.N) * a.in;
+  if (a.x_rows) return a.H + (static_cast<int64_t>(j) * a.N + (a.row0 + b) % a.N) * a.in;
   return a.H + (static_cast<int64_t>(j) * a.Bn + b) * a.pitch_in;
 }
 
@@ -124,7 +124,7 @@ __device__ __forceinline__ void head_body(const HeadArgs& a, uint8_t* smem, int 
     d[1] = __floats2bfloat162_rn(w.z, w.w);
   }
   if (t < kHeadMaxC) bls[t] = t < C ? bL[t] : 0.f;
-  if (t >= 64 && t < 64 + B) ys[t - 64] = a.y[static_cast<int64_t>(j) * a.N + (a.t * B + t - 64) % a.N];
+  if (t >= 64 && t < 64 + B) ys[t - 64] = a.y[static_cast<int64_t>(j) * a.N + (a.row0 + t - 64) % a.N];
   sync();
   for (int tile = warp; tile < (Bn / 16) * 2; tile += kHeadThreads / 32) {
     const int mt = tile >> 1, nt = tile & 1;                    // 16 samples x 8 classes

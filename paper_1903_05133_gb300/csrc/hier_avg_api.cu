@@ -85,6 +85,8 @@ struct hier_avg {
   std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_dz;
   CUtensorMap tm_x;                           // X [P][N][d_0] as the first layer's batch tile
   int64_t t = 0;
+  int64_t cursor = 0;                         // rows each learner has read (next batch: mod N)
+  int Bstep = 0;                              // batch size of the following steps (<= B)
   int64_t launches = 0;                       // kernels launched since bind
   // profiling
   unsigned prof = 0;                          // kinds timed: bit (1 << HA_KERNEL_*)
@@ -298,18 +300,18 @@ int check_bound(hier_avg* h) {
 
 // Algorithmic bytes of the big kernels (fp32 master read + write, activations).
 double bytes_forward(const hier_avg* h, int l) {
-  const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
+  const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->Bstep;
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
   return P * (in * out * 4.0 + out * 4.0 + B * in * act + B * out * (l + 1 == h->L ? 4.0 : act));
 }
 // The first layer's update fused with the next step's first-layer forward: W read and
 // written once, this step's and the next step's batch rows, dZ_1 read, b_1 read, H_1' written.
 double bytes_update_forward(const hier_avg* h) {
-  const double P = h->P, in = h->dims[0], out = h->dims[1], B = h->B;
+  const double P = h->P, in = h->dims[0], out = h->dims[1], B = h->Bstep;
   return P * (in * out * 8.0 + out * 4.0 + 2.0 * B * in * 2.0 + 2.0 * B * out * 2.0);
 }
 double bytes_backward(const hier_avg* h, int l) {
-  const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->B;
+  const double P = h->P, in = h->dims[l], out = h->dims[l + 1], B = h->Bstep;
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
   const double dx = l > 0 ? (B * in * act + in * 8.0) : 0.0;
   return P * (in * out * 8.0 + B * in * act + B * out * act + dx);
@@ -321,12 +323,12 @@ ha::HeadArgs head_args(hier_avg* h) {
   ha::HeadArgs a{};
   a.C = h->dims[L];
   a.in = h->dims[L - 1];
-  a.B = h->B;
+  a.B = h->Bstep;
   a.Bn = h->Bn;
   a.pitch_in = h->pitch[L - 1];
   a.ld = h->ld;
   a.N = h->N;
-  a.t = h->t;
+  a.row0 = h->cursor % h->N;
   a.lr = h->lr;
   a.W = h->params + h->woff[L - 1];
   a.bias = h->params + h->boff[L - 1];
@@ -350,7 +352,7 @@ ha::HeadArgs head_args(hier_avg* h) {
 // the forwards read one copy per cluster (the same values: results are unchanged).
 int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
             bool shared = false) {
-  const int L = h->L, P = h->P, B = h->B;
+  const int L = h->L, P = h->P, B = h->Bstep;
   if (fused) *fused = false;
   cudaStream_t s = h->stream;
   int rc;
@@ -358,12 +360,12 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     const int d0 = h->dims[0];
     // The first layer reads its batch tile straight from X unless the batch wraps
     // around the end of the data set; then the rows are gathered first.
-    const int64_t r0 = (h->t * B) % h->N;
+    const int64_t r0 = h->cursor % h->N;   // this step's batch: rows r0 .. (mod N)
     const bool x_direct = r0 + B <= h->N;
     if (!x_direct) {
       rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, [&] {
         return ha::launch_gather_bf16(static_cast<const __nv_bfloat16*>(h->X), h->N, d0, B, h->Bn,
-                                      h->pitch[0], h->t, P, h->wsp<__nv_bfloat16>(h->off_H[0]), s);
+                                      h->pitch[0], r0, P, h->wsp<__nv_bfloat16>(h->off_H[0]), s);
       }, "gather");
       if (rc) return rc;
     }
@@ -394,7 +396,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         a.mode = 2;
         a.y = h->y;
         a.N = h->N;
-        a.t = h->t;
+        a.row0 = r0;
         a.lr = h->lr;
         a.pitch_out = h->pitch[L];
         a.dz_out = h->wsp<__nv_bfloat16>(h->off_dZ[L]);
@@ -418,7 +420,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       if (rc) return rc;
     } else if (!h->fused_xent) {
       rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
-        return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->Bn, C,
+        return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, r0, B, h->Bn, C,
                                     h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
                                     h->wsp<__nv_bfloat16>(h->off_dZ[L]), h->loss(), P, s);
       }, "xent");
@@ -452,7 +454,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       const CUtensorMap& hin = from_x ? h->tm_x : h->tm_h[l];
       // The next step's batch, if contiguous in X, lets the first layer's update also
       // produce the next step's H_1 (the layer must be hidden, i.e. L >= 2).
-      const int64_t r1 = ((h->t + 1) * B) % h->N;
+      const int64_t r1 = (h->cursor + B) % h->N;
       if (l == 0 && fuse_next && L >= 2 && r1 + B <= h->N) {
         TcFwdArgs f{};
         f.in = h->dims[0];
@@ -504,7 +506,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
   } else {
     const int d0 = h->dims[0];
     rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 4 * 2, [&] {
-      return ha::launch_gather_f32(static_cast<const float*>(h->X), h->N, d0, B, h->t, P,
+      return ha::launch_gather_f32(static_cast<const float*>(h->X), h->N, d0, B, h->cursor % h->N, P,
                                    h->wsp<float>(h->off_H[0]), s);
     }, "gather");
     if (rc) return rc;
@@ -519,7 +521,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       if (rc) return rc;
     }
     rc = h->timed(HA_KERNEL_XENT, double(P) * B * h->dims[L] * 4 * 2, [&] {
-      return ha::launch_xent_f32(h->wsp<float>(h->off_Z), h->y, h->N, h->t, B, h->dims[L],
+      return ha::launch_xent_f32(h->wsp<float>(h->off_Z), h->y, h->N, h->cursor % h->N, B, h->dims[L],
                                  h->wsp<float>(h->off_dZ[L]), h->loss(), P, s);
     }, "xent");
     if (rc) return rc;
@@ -540,6 +542,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     }
   }
   ++h->t;
+  h->cursor += B;
   return HA_OK;
 }
 
@@ -652,6 +655,7 @@ int hier_avg_create(int P, int S, int K1, int K2, float lr, int B, const int* di
   h->K1 = K1;
   h->K2 = K2;
   h->B = B;
+  h->Bstep = B;
   h->lr = lr;
   h->prec = precision;
   h->dims.assign(dims, dims + n_dims);
@@ -710,6 +714,7 @@ int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t w
   h->N = N;
   h->stream = static_cast<cudaStream_t>(stream);
   h->t = 0;
+  h->cursor = 0;
   int rc;
   if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_bytes, h->stream), "bind: memset"))) return rc;
   if (h->prec == HA_PREC_BF16) {
@@ -746,8 +751,8 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
   if (!X_host || !y_host || !loss_host) return h->fail(HA_EINVAL, "round_host: NULL host buffer");
   const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
   const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
-  const int64_t rows = static_cast<int64_t>(h->B) * round_steps(h);
-  int64_t r0 = (h->t * h->B) % h->N, left = rows < h->N ? rows : h->N;
+  const int64_t rows = static_cast<int64_t>(h->Bstep) * round_steps(h);
+  int64_t r0 = h->cursor % h->N, left = rows < h->N ? rows : h->N;
   if (rows >= h->N) r0 = 0;
   while (left > 0) {   // at most two contiguous row ranges per learner (wrap-around)
     const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
@@ -777,6 +782,21 @@ int hier_avg_set_global_steps(hier_avg* h, int steps) {
   return HA_OK;
 }
 
+int hier_avg_set_batch(hier_avg* h, int B) {
+  if (!h || B < 1 || B > h->B) return HA_EINVAL;
+  if (B < h->Bstep && h->bound && h->prec == HA_PREC_BF16) {
+    // The bf16 path keeps Bn-row gradient tiles; rows from B on must add nothing to dW.
+    cudaSetDevice(h->device);
+    for (int l = 1; l <= h->L; ++l)
+      if (int rc = h->cuda(cudaMemsetAsync(h->ws + h->off_dZ[l], 0,
+                                           static_cast<size_t>(h->P) * h->Bn * h->pitch[l] * 2,
+                                           h->stream), "set_batch: clear dZ"))
+        return rc;
+  }
+  h->Bstep = B;
+  return HA_OK;
+}
+
 int hier_avg_set_lr(hier_avg* h, float lr) {
   if (!h || !std::isfinite(lr)) return HA_EINVAL;
   h->lr = lr;
@@ -792,6 +812,7 @@ int hier_avg_get_step(const hier_avg* h, int64_t* t) {
 int hier_avg_set_step(hier_avg* h, int64_t t) {
   if (!h || t < 0) return HA_EINVAL;
   h->t = t;
+  h->cursor = t * h->Bstep;
   return HA_OK;
 }
 

@@ -64,7 +64,8 @@ cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, 
 // of feature slices per learner (forward, softmax-CE and backward).
 struct HeadArgs {
   int C, in, B, Bn, pitch_in;
-  int64_t ld, N, t;
+  int64_t ld, N;
+  int64_t row0;               // first row of this step's batch in each learner's data (< N)
   float lr;
   float* W;                   // learner 0's W_L [C][in] (fp32 master)
   float* bias;                // learner 0's b_L
@@ -101,7 +102,7 @@ struct TcFwdArgs {
                               // after an average): all read learner g*share's copy
   // mode 2: labels and outputs of the fused cross-entropy
   const int32_t* y;
-  int64_t N, t;
+  int64_t N, row0;            // labels: rows row0 + b (mod N)
   float lr;
   __nv_bfloat16* dz_out;      // dZ_L [P][Bn][pitch_out]
   float* loss;                // [P]
@@ -142,12 +143,12 @@ cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
 cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_cur,
                                      const CUtensorMap& x_next, const CUtensorMap& dz,
                                      const TcFwdArgs& a, cudaStream_t s);
-// Mini-batch fetch for the bf16 path: rows (t*B + b) mod N of X -> H_0.
+// Mini-batch fetch for the bf16 path: rows (row0 + b) mod N of X -> H_0.
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
-                               int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s);
+                               int pitch0, int64_t row0, int P, __nv_bfloat16* H0, cudaStream_t s);
 // Softmax cross-entropy gradient of the last layer (bf16 operands out), loss, and
 // the SGD update of the last bias.
-cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t row0, int B,
                              int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
                              __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s);
 
@@ -157,12 +158,12 @@ cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s);
 
 // ----------------------------------------------------------------- fp32 CUDA-core step
 // Buffers: H_l [P][B][d_l] fp32, Z_L [P][B][d_L], dZ_l [P][B][d_l] fp32.
-cudaError_t launch_gather_f32(const float* X, int64_t N, int d0, int B, int64_t t, int P,
+cudaError_t launch_gather_f32(const float* X, int64_t N, int d0, int B, int64_t row0, int P,
                               float* H0, cudaStream_t s);
 cudaError_t launch_fwd_f32(const float* H, const float* W, const float* bias, int64_t ld,
                            int in, int out, int B, int relu, float* out_act, int P,
                            cudaStream_t s);
-cudaError_t launch_xent_f32(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+cudaError_t launch_xent_f32(const float* Z, const int32_t* y, int64_t N, int64_t row0, int B,
                             int C, float* dZ, float* loss, int P, cudaStream_t s);
 cudaError_t launch_dx_f32(const float* dZ, const float* W, int64_t ld, const float* Hprev,
                           int in, int out, int B, float* dZprev, int P, cudaStream_t s);

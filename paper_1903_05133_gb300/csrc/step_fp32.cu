@@ -14,15 +14,15 @@ namespace {
 
 constexpr int T = 16;
 
-// H0[j][b][:] = X[j][(t*B + b) mod N][:]
-__global__ void k_gather_f32(const float* __restrict__ X, int64_t N, int d0, int B, int64_t t,
+// H0[j][b][:] = X[j][(row0 + b) mod N][:]  (row0: the batch's first row)
+__global__ void k_gather_f32(const float* __restrict__ X, int64_t N, int d0, int B, int64_t row0,
                              float* __restrict__ H0) {
   const int j = blockIdx.y;
   const int64_t total = static_cast<int64_t>(B) * d0;
   for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
        idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const int b = static_cast<int>(idx / d0), k = static_cast<int>(idx % d0);
-    const int64_t row = (t * B + b) % N;
+    const int64_t row = (row0 + b) % N;
     H0[(static_cast<int64_t>(j) * B + b) * d0 + k] = X[(static_cast<int64_t>(j) * N + row) * d0 + k];
   }
 }
@@ -56,7 +56,7 @@ __global__ void k_fwd_f32(const float* __restrict__ H, const float* __restrict__
 // One CTA per learner: dZ = (softmax(z_b) - onehot(y_b)) / B, loss = mean CE.
 __global__ void __launch_bounds__(256) k_xent_f32(const float* __restrict__ Z,
                                                  const int32_t* __restrict__ y, int64_t N,
-                                                 int64_t t, int B, int C, float* __restrict__ dZ,
+                                                 int64_t row0, int B, int C, float* __restrict__ dZ,
                                                  float* __restrict__ loss) {
   extern __shared__ float sh[];
   float* row_max = sh;
@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(256) k_xent_f32(const float* __restrict__ Z,
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
     if (lane == 0) {
-      const int yb = y[static_cast<int64_t>(j) * N + (t * B + b) % N];
+      const int yb = y[static_cast<int64_t>(j) * N + (row0 + b) % N];
       row_max[b] = m;
       row_sum[b] = s;
       row_y[b] = yb;
@@ -157,11 +157,11 @@ __global__ void k_dw_update_f32(const float* __restrict__ dZ, const float* __res
 
 }  // namespace
 
-cudaError_t launch_gather_f32(const float* X, int64_t N, int d0, int B, int64_t t, int P,
+cudaError_t launch_gather_f32(const float* X, int64_t N, int d0, int B, int64_t row0, int P,
                               float* H0, cudaStream_t s) {
   const int64_t total = static_cast<int64_t>(B) * d0;
   dim3 grid(static_cast<unsigned>((total + 255) / 256 < 1024 ? (total + 255) / 256 : 1024), P);
-  k_gather_f32<<<grid, 256, 0, s>>>(X, N, d0, B, t, H0);
+  k_gather_f32<<<grid, 256, 0, s>>>(X, N, d0, B, row0, H0);
   return cudaGetLastError();
 }
 
@@ -173,10 +173,10 @@ cudaError_t launch_fwd_f32(const float* H, const float* W, const float* bias, in
   return cudaGetLastError();
 }
 
-cudaError_t launch_xent_f32(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+cudaError_t launch_xent_f32(const float* Z, const int32_t* y, int64_t N, int64_t row0, int B,
                             int C, float* dZ, float* loss, int P, cudaStream_t s) {
   const size_t sh = static_cast<size_t>(4) * B * sizeof(float);
-  k_xent_f32<<<P, 256, sh, s>>>(Z, y, N, t, B, C, dZ, loss);
+  k_xent_f32<<<P, 256, sh, s>>>(Z, y, N, row0, B, C, dZ, loss);
   return cudaGetLastError();
 }
 

@@ -151,7 +151,7 @@ __device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, 
     for (int c = 0; c < C; ++c) m = fmaxf(m, zs[c * ZP + t]);
     float s = 0.f;
     for (int c = 0; c < C; ++c) s += expf(zs[c * ZP + t] - m);
-    const int yb = a.y[static_cast<int64_t>(j) * a.N + (a.t * B + t) % a.N];
+    const int yb = a.y[static_cast<int64_t>(j) * a.N + (a.row0 + t) % a.N];
     stat[t] = m;
     stat[64 + t] = s;
     stat[128 + t] = __int_as_float(yb);
@@ -1735,11 +1735,11 @@ __global__ void __launch_bounds__(kUfThreads, 1)
 }
 
 // ------------------------------------------------------------------ gather
-// H_0[j][b][:] = X[j][(t*B + b) mod N][:] for b < B, one CTA per (64-feature slice,
+// H_0[j][b][:] = X[j][(row0 + b) mod N][:] for b < B, one CTA per (64-feature slice,
 // learner); rows b >= B stay zero.
 __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __restrict__ X,
                                                     int64_t N, int d0, int B, int Bn,
-                                                    int pitch0, int64_t t,
+                                                    int pitch0, int64_t row0,
                                                     __nv_bfloat16* __restrict__ H0) {
   grid_dep_wait();
   const int j = blockIdx.y, k0 = blockIdx.x * 64;
@@ -1748,7 +1748,7 @@ __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __rest
     const int b = idx >> 3, v = idx & 7;
     const int k = k0 + v * 8;
     if (k < d0) {
-      const int64_t row = (t * B + b) % N;
+      const int64_t row = (row0 + b) % N;
       *reinterpret_cast<uint4*>(H0 + (static_cast<int64_t>(j) * Bn + b) * pitch0 + k) =
           *reinterpret_cast<const uint4*>(X + (static_cast<int64_t>(j) * N + row) * d0 + k);
     }
@@ -1764,7 +1764,7 @@ __global__ void __launch_bounds__(256) k_gather_bf16(const __nv_bfloat16* __rest
 constexpr int kXentThreads = 256;
 __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restrict__ Z,
                                                            const int32_t* __restrict__ y,
-                                                           int64_t N, int64_t t, int B, int Bn,
+                                                           int64_t N, int64_t row0, int B, int Bn,
                                                            int C, int pitch_c, float lr,
                                                            float* bias_L, int64_t ld,
                                                            __nv_bfloat16* dZ, float* loss) {
@@ -1784,7 +1784,7 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
     if (lane == 0) {
-      const int yb = y[static_cast<int64_t>(j) * N + (t * B + b) % N];
+      const int yb = y[static_cast<int64_t>(j) * N + (row0 + b) % N];
       row_max[b] = m;
       row_sum[b] = s;
       row_y[b] = yb;
@@ -1862,16 +1862,16 @@ cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap
 }
 
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
-                               int pitch0, int64_t t, int P, __nv_bfloat16* H0, cudaStream_t s) {
+                               int pitch0, int64_t row0, int P, __nv_bfloat16* H0, cudaStream_t s) {
   dim3 grid((d0 + 63) / 64, P);
-  return launch_pdl(k_gather_bf16, grid, dim3(256), 0, s, false, 1, X, N, d0, B, Bn, pitch0, t, H0);
+  return launch_pdl(k_gather_bf16, grid, dim3(256), 0, s, false, 1, X, N, d0, B, Bn, pitch0, row0, H0);
 }
 
-cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t t, int B,
+cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t row0, int B,
                              int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
                              __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s) {
   dim3 grid(P, (C + kXentThreads - 1) / kXentThreads);
-  return launch_pdl(k_xent_bf16, grid, dim3(kXentThreads), 0, s, false, 1, Z, y, N, t, B, Bn, C,
+  return launch_pdl(k_xent_bf16, grid, dim3(kXentThreads), 0, s, false, 1, Z, y, N, row0, B, Bn, C,
                     pitch_c, lr, bias_L, ld, dZ, loss);
 }
 

@@ -191,6 +191,10 @@ class HierAvg:
         check(self._lib.hier_avg_set_lr(self.h, float(lr)), "set_lr", self.h)
         self.lr = float(lr)
 
+    def set_batch(self, B: int) -> None:
+        """Mini-batch size of the following local steps (<= the B given at creation)."""
+        check(self._lib.hier_avg_set_batch(self.h, int(B)), "set_batch", self.h)
+
     def launches(self) -> int:
         """Kernels this handle has launched since it was created."""
         n = c_int64()

@@ -97,6 +97,9 @@ def test_calls_before_bind_fail_cleanly(lib):
     assert lib.hier_avg_set_global_steps(None, 5) == -1
     assert lib.hier_avg_set_lr(h, float("nan")) == -1 and lib.hier_avg_set_lr(h, float("inf")) == -1
     assert lib.hier_avg_set_lr(h, 0.01) == 0
+    assert lib.hier_avg_set_batch(h, 0) == -1 and lib.hier_avg_set_batch(h, 10 ** 6) == -1
+    assert lib.hier_avg_set_batch(None, 1) == -1
+    assert lib.hier_avg_set_batch(h, 1) == 0
     n = ctypes.c_int64(-1)
     assert lib.hier_avg_launches(h, ctypes.byref(n)) == 0 and n.value == 0   # nothing ran
     assert lib.hier_avg_launches(h, None) == -1

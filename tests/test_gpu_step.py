@@ -329,6 +329,51 @@ def test_free_global_interval_literal_sequence(w, G):
     assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
 
 
+# Per-round batch size B_n (Theorem 3.3's growing batches; a shrinking step is included
+# to check that rows beyond the batch add nothing), each learner reading its data
+# sequentially, with a diminishing step size; against the oracle.
+BATCH_SCHED = [(SMALL_FP32, (3, 7, 5)), (SMALL_BF16, (16, 48, 32)), (FUSE_THREE, (8, 32, 24)),
+               (RAGGED_BF16, (12, 20, 7))]
+
+
+@pytest.mark.parametrize("w,sched", BATCH_SCHED, ids=lambda v: getattr(v, "name", str(v)))
+def test_batch_schedule_against_oracle(w, sched):
+    ha, X, y = setup(w)
+    start = oracle_params(ha, ha.params)
+    o = make_oracle(w, ha, X, y, start)
+    o_ref = (make_oracle(w, ha, X, y, start, mode="bf16_acc32") if w.precision == "bf16" else None)
+    for n, Bn in enumerate(sched):
+        ha.set_batch(Bn)
+        ha.set_lr(w.lr / (n + 1))
+        for oo in (o, o_ref):
+            if oo is not None:
+                oo.B, oo.lr = Bn, w.lr / (n + 1)
+                oo.round()
+        ha.round()
+    ha.check()
+    compare(ha, o, o_ref=o_ref)
+    gl = ha.losses().numpy()
+    assert np.allclose(gl, o.problem.last_loss, rtol=2e-3, atol=1e-4)
+
+
+def test_batch_schedule_literal_sequence():
+    w = SMALL_BF16.replace(K1=3)
+    ha1, X, y = setup(w, perturb=(0.01, 0.01))
+    ha2, _, _ = setup(w, perturb=(0.01, 0.01))
+    for Bn in (48, 16, 32):
+        ha1.set_batch(Bn)
+        ha1.round()
+        ha2.set_batch(Bn)
+        for b in range(w.K2):
+            for k in range(w.K1):
+                ha2.step()
+            ha2.local_average()
+        ha2.global_average()
+    ha1.check()
+    ha2.check()
+    assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
+
+
 def _force(ha, *oracles):
     """Load the GPU's current learner state into the oracles (teacher forcing)."""
     state = oracle_params(ha, ha.params)
