@@ -22,7 +22,7 @@ namespace head {
 constexpr int kHeadThreads = 256;
 constexpr int kHeadMaxC = 16;
 constexpr int kHeadClusterMax = 8;
-constexpr int kHeadClusterPref = 4;           // CTAs per learner while slices stay <= 512
+constexpr int kHeadClusterPref = 4;           // CTAs per learner when 8 per learner would not fit in one wave
 constexpr int kHeadPad = 8;                   // bf16 row padding: ldmatrix rows hit distinct banks
 constexpr int kGA = kHeadMaxC + 8;            // g_q   [b][c] row stride (bf16)
 constexpr int kGT = 64 + 8;                   // g_q^T [c][b] row stride (bf16)

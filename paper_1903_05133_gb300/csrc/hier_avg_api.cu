@@ -210,7 +210,7 @@ int plan_layout(hier_avg* h) {
       max_tiles = std::max(max_tiles, std::max(ftiles, btiles) * P);
     }
     h->fused_xent = h->dims[L] <= 128;
-    h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B));
+    h->head = ha::head_supported(h->dims[L], h->dims[L - 1], static_cast<int>(B), h->P);
     h->off_part = take(part_bytes);
     h->off_cnt = take(max_tiles * 4);
     h->off_dyn = take(16);

@@ -152,7 +152,7 @@ cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_
                              int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
                              __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s);
 
-bool head_supported(int C, int in, int B);
+bool head_supported(int C, int in, int B, int P);
 cudaError_t head_configure();   // raises the dynamic shared-memory limit once
 cudaError_t launch_head(const HeadArgs& a, int P, cudaStream_t s);
 

@@ -7,38 +7,44 @@ namespace ha {
 namespace {
 using namespace head;
 
-// Features per CTA: a multiple of 64, at least 128; 4 CTAs per learner (clusters of
-// 8 are harder to place next to a draining kernel) unless that needs slices over 512.
-__host__ __device__ inline int head_slice(int in) {
-  int f = ((in + kHeadClusterPref - 1) / kHeadClusterPref + 63) / 64 * 64;
+// Features per CTA (a multiple of 64) for P learners: 8 CTAs per learner (slices of at
+// least 64) while all P clusters fit in one wave of the GPU's 152 SMs, else 4 (at least
+// 128; more clusters of 8 than fit at once measured slower), or 8 where 4 would need
+// slices over 512.
+constexpr int kHeadWave = 152;
+__host__ __device__ inline int head_slice(int in, int P) {
+  const bool wide = P * kHeadClusterMax <= kHeadWave;
+  const int per = wide ? kHeadClusterMax : kHeadClusterPref;
+  int f = ((in + per - 1) / per + 63) / 64 * 64;
   if (f > 512) f = ((in + kHeadClusterMax - 1) / kHeadClusterMax + 63) / 64 * 64;
-  return f < 128 ? 128 : f;
+  const int fmin = wide ? 64 : 128;
+  return f < fmin ? fmin : f;
 }
-__host__ __device__ inline int head_smem_bytes(int in, int Bn) {
-  return head_body_smem(head_slice(in), Bn);
+__host__ __device__ inline int head_smem_bytes(int in, int P, int Bn) {
+  return head_body_smem(head_slice(in, P), Bn);
 }
 
 template <int CT>
 __global__ void __launch_bounds__(kHeadThreads) k_head(const HeadArgs a) {
   extern __shared__ __align__(16) uint8_t smem[];
   grid_dep_wait();
-  head_body<CT>(a, smem, blockIdx.y, blockIdx.x, gridDim.x, head_slice(a.in), threadIdx.x,
+  head_body<CT>(a, smem, blockIdx.y, blockIdx.x, gridDim.x, head_slice(a.in, gridDim.y), threadIdx.x,
                 [] { __syncthreads(); });
 }
 
 template <int CT>
 cudaError_t launch_cluster(const HeadArgs& a, int P, cudaStream_t s) {
-  const int S = (a.in + head_slice(a.in) - 1) / head_slice(a.in);
-  return launch_pdl(k_head<CT>, dim3(S, P), dim3(kHeadThreads), head_smem_bytes(a.in, a.Bn), s,
+  const int F = head_slice(a.in, P), S = (a.in + F - 1) / F;
+  return launch_pdl(k_head<CT>, dim3(S, P), dim3(kHeadThreads), head_smem_bytes(a.in, P, a.Bn), s,
                     false, S, a);
 }
 
 }  // namespace
 
-bool head_supported(int C, int in, int B) {
+bool head_supported(int C, int in, int B, int P) {
   return C <= kHeadMaxC && in % 64 == 0 && B <= 64 &&
-         (in + head_slice(in) - 1) / head_slice(in) <= kHeadClusterMax &&
-         head_smem_bytes(in, 64) <= 200 * 1024;
+         (in + head_slice(in, P) - 1) / head_slice(in, P) <= kHeadClusterMax &&
+         head_smem_bytes(in, P, 64) <= 200 * 1024;
 }
 
 cudaError_t head_configure() {
