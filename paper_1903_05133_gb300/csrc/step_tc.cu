@@ -751,7 +751,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         }
         if (++c == nc) { c = 0; ++tau; }
       }
-      tma_store_wait_all();
+      tma_store_wait_read_all();   // (before the shared memory is released)
       if (stored > 0) mbar_arrive(&wempty[(stored - 1) % nw]);
     }
   } else if (warp == 5) {
@@ -1141,7 +1141,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       __syncwarp();
     }
     if (lane == 0) {
-      tma_store_wait_all();
+      tma_store_wait_read_all();   // (before the shared memory is released)
       if (i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
     }
   } else if (warp == 5) {
@@ -1459,7 +1459,7 @@ __global__ void __launch_bounds__(kUfThreads, 1)
         }
         if (++c == nk) { c = 0; ++tau; }
       }
-      tma_store_wait_all();
+      tma_store_wait_read_all();   // (before the shared memory is released)
       if (stored > 0) mbar_arrive(&wempty[(stored - 1) % nw]);
     }
     if (cq > 1) {
@@ -1841,9 +1841,10 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
 cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
                                const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s) {
   (void)P;
-  // Cooperative for the same reason as the forward (split dX tiles).
-  return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, true, 1,
-                    w_bwd, h_in, dz, a);
+  // Cooperative for the same reason as the forward (split dX tiles); without dX no CTA
+  // waits on another, and the cooperative attribute costs ~2 us per launch.
+  return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s,
+                    a.has_dx != 0, 1, w_bwd, h_in, dz, a);
 }
 
 cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
