@@ -1441,10 +1441,12 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     }
   } else if (warp == 11) {
     if (lane == 0) {
-      // Store each updated W tile; its slot is released once the TMA has read it
-      // (two stores in flight).
+      // Store each updated W tile; its slot is released once the TMA has read it.  In
+      // cluster mode (a short layer) each slot is released as soon as its own store has
+      // been read; in stream-K mode one store behind, two in flight (releasing at once
+      // let the fast SMs take bandwidth from the slow ones, whose end sets the kernel's).
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
-      int tau = tile0, c = c0, stored = 0;
+      int tau = tile0, c = c0, stored = 0, released = 0;
       for (int i = 0; i < n_local; ++i) {
         const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
         const int s = i % nw;
@@ -1453,14 +1455,19 @@ __global__ void __launch_bounds__(kUfThreads, 1)
         tma_store_3d_hint(&tm_w, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
         tma_store_commit();
         stored = i + 1;
-        if (i > 0) {
+        if (cq > 1) {
+          tma_store_wait_read_all();
+          mbar_arrive(&wempty[s]);
+          released = stored;
+        } else if (i > 0) {
           tma_store_wait_read_1();
           mbar_arrive(&wempty[(i - 1) % nw]);
+          released = i;
         }
         if (++c == nk) { c = 0; ++tau; }
       }
       tma_store_wait_read_all();   // (before the shared memory is released)
-      if (stored > 0) mbar_arrive(&wempty[(stored - 1) % nw]);
+      if (stored > released) mbar_arrive(&wempty[(stored - 1) % nw]);
     }
     if (cq > 1) {
       cluster_sync_all();
