@@ -157,6 +157,12 @@ MANY_CLASSES_BF16 = configs.Workload("mlp_bf16_c300", P=4, S=4, K1=1, K2=2, roun
                                      sigma_mu=0.1, init="he")
 HEAD_C13 = configs.Workload("mlp_bf16_c13", P=4, S=2, K1=1, K2=2, rounds=1, dims=(192, 128, 13),
                             precision="bf16", N=48, B=24, lr=0.05, sigma_mu=0.1, init="he")
+# Head slices of 128 features (20 learners: clusters of 8 CTAs per learner would not fit
+# in one wave, so 4 per learner), a ragged 320-wide layer (last slice 64 wide) and a batch
+# that is not a multiple of 16.
+HEAD_F128 = configs.Workload("mlp_bf16_head_f128", P=20, S=4, K1=3, K2=2, rounds=1,
+                             dims=(256, 320, 10), precision="bf16", N=120, B=24, lr=0.05,
+                             sigma_mu=0.1, init="he")
 SMALL_FP32 = configs.Workload("tiny_mlp_fp32", P=4, S=2, K1=2, K2=2, rounds=1,
                               dims=(100, 37, 10), precision="fp32", N=40, B=7, lr=0.05,
                               sigma_mu=0.1, init="he")
@@ -190,8 +196,8 @@ def test_one_step_from_distinct_learners(w):
 
 
 @pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16,
-                               HEAD_C13, WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16],
-                         ids=lambda w: w.name)
+                               HEAD_C13, WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16,
+                               HEAD_F128], ids=lambda w: w.name)
 def test_full_run_against_oracle(w):
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
