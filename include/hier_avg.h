@@ -37,7 +37,7 @@ extern "C" {
 #define HA_ECUDA        (-3)  /* a CUDA runtime or driver call failed               */
 #define HA_ESTATE       (-4)  /* call out of order (e.g. a step before bind)        */
 #define HA_ETIMEOUT     (-5)  /* a bounded device-side wait expired; see check      */
-#define HA_EUNSUPPORTED (-6)  /* valid request this build does not implement        */
+#define HA_EUNSUPPORTED (-6)  /* valid request the library does not implement       */
 
 #define HA_PREC_FP32 0        /* every product in fp32 on CUDA cores                */
 #define HA_PREC_BF16 1        /* bf16 GEMM operands, fp32 accumulate, fp32 master   */
