@@ -88,6 +88,11 @@ struct hier_avg {
   int64_t cursor = 0;                         // rows each learner has read (next batch: mod N)
   int Bstep = 0;                              // batch size of the following steps (<= B)
   int64_t launches = 0;                       // kernels launched since bind
+  // round_host: the rows of each step are copied on a stream of their own, one step
+  // ahead of the kernels, which wait on copied[step]
+  cudaStream_t copy_stream = nullptr;
+  std::vector<cudaEvent_t> copied;
+  cudaEvent_t round_start = nullptr;
   // profiling
   unsigned prof = 0;                          // kinds timed: bit (1 << HA_KERNEL_*)
   int prof_every = 1;                         // time every n-th launch of those kinds
@@ -350,8 +355,10 @@ ha::HeadArgs head_args(hier_avg* h) {
 // compute the next step's H_1; *fused reports whether it did.  shared: the caller has
 // just averaged each local cluster, so its S learners hold identical parameters and
 // the forwards read one copy per cluster (the same values: results are unchanged).
+// next_rows (round_host): recorded once the next step's rows are on the device; the
+// update+forward kernel, which reads them, waits for it.
 int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
-            bool shared = false) {
+            bool shared = false, cudaEvent_t next_rows = nullptr) {
   const int L = h->L, P = h->P, B = h->Bstep;
   if (fused) *fused = false;
   cudaStream_t s = h->stream;
@@ -478,6 +485,8 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.w_stream = a.w_stream;
         f.lr = h->lr;
         f.err = h->err_word();
+        if (next_rows && (rc = h->cuda(cudaStreamWaitEvent(s, next_rows, 0), "round_host: wait for the rows")))
+          return rc;
         rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h), [&] {
           return ha::launch_tc_update_forward(h->tm_wf[0], hin, h->tm_x, h->tm_dz[1], f, s);
         }, "update+forward");
@@ -570,14 +579,27 @@ int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 // K1-th, the global average after the G-th (fused with the local average that closes
 // the round when K1 divides G).  G = K1 * K2 unless set: Sec. 3.1 leaves beta = G / K1
 // free in practice.
-int do_round(hier_avg* h) {
+// ready (round_host): ready[k] is recorded once the rows of the round's step k (0-based)
+// are on the device.  Step k reads those rows and, in an update+forward kernel, step
+// k + 1's.  The handle's stream waits for ready[0] before step 0 (and for ready[1] just
+// before step 0's update+forward), then at steps k = 1, 3, 7, ... (k + 1 a power of two)
+// for the rows up to step 2k + 1, which cover every step until the next wait: few waits,
+// since each one ends the overlap of consecutive launches.
+int do_round(hier_avg* h, const std::vector<cudaEvent_t>* ready = nullptr) {
   int rc;
   const int G = round_steps(h);
   bool h1_ready = false;
   for (int r = 1; r <= G; ++r) {
+    const int k = r - 1;
+    if (ready && (k == 0 || (k & (k + 1)) == 0) &&
+        (rc = h->cuda(cudaStreamWaitEvent(h->stream, (*ready)[k == 0 ? 0 : std::min(2 * k + 1, G - 1)], 0),
+                      "round_host: wait for the rows")))
+      return rc;
     const bool block_end = r % h->K1 == 0;              // a local average follows step r
     const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
-    if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local))) return rc;
+    if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local,
+                      ready && r == 1 && G > 1 ? (*ready)[1] : nullptr)))
+      return rc;
     if (r < G && block_end && (rc = do_local(h))) return rc;
   }
   return G % h->K1 == 0 ? do_local_global(h) : do_global(h);
@@ -668,6 +690,9 @@ int hier_avg_create(int P, int S, int K1, int K2, float lr, int B, const int* di
 void hier_avg_destroy(hier_avg* h) {
   if (!h) return;
   for (cudaEvent_t e : h->pool) cudaEventDestroy(e);
+  for (cudaEvent_t e : h->copied) cudaEventDestroy(e);
+  if (h->round_start) cudaEventDestroy(h->round_start);
+  if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   delete h;
 }
 
@@ -751,27 +776,48 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
   if (!X_host || !y_host || !loss_host) return h->fail(HA_EINVAL, "round_host: NULL host buffer");
   const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
   const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
-  const int64_t rows = static_cast<int64_t>(h->Bstep) * round_steps(h);
-  int64_t r0 = h->cursor % h->N, left = rows < h->N ? rows : h->N;
-  if (rows >= h->N) r0 = 0;
-  while (left > 0) {   // at most two contiguous row ranges per learner (wrap-around)
-    const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
-    int rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
-                                       h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
-                                       h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice,
-                                       h->stream),
-                     "round_host: X copy");
-    if (rc) return rc;
-    rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
-                                   n * 4, h->P, cudaMemcpyHostToDevice, h->stream),
-                 "round_host: y copy");
-    if (rc) return rc;
-    left -= n;
-    r0 = 0;
+  const int G = round_steps(h);
+  if (!h->copy_stream &&
+      h->cuda(cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking), "round_host: stream"))
+    return HA_ECUDA;
+  if (!h->round_start &&
+      h->cuda(cudaEventCreateWithFlags(&h->round_start, cudaEventDisableTiming), "round_host: event"))
+    return HA_ECUDA;
+  while (static_cast<int>(h->copied.size()) < G) {
+    cudaEvent_t e;
+    if (int rc = h->cuda(cudaEventCreateWithFlags(&e, cudaEventDisableTiming), "round_host: event")) return rc;
+    h->copied.push_back(e);
   }
-  if (int rc = do_round(h)) return rc;
-  if (int rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost,
-                                       h->stream), "round_host: loss copy"))
+  // The copies start once the work already queued on the handle's stream is done; step
+  // k's rows are (row0 + b) mod N, b < B, of every learner: at most two contiguous
+  // ranges, then copied[k] is recorded.
+  int rc;
+  if ((rc = h->cuda(cudaEventRecord(h->round_start, h->stream), "round_host: record")) ||
+      (rc = h->cuda(cudaStreamWaitEvent(h->copy_stream, h->round_start, 0), "round_host: wait")))
+    return rc;
+  for (int k = 0; k < G; ++k) {
+    int64_t r0 = (h->cursor + static_cast<int64_t>(k) * h->Bstep) % h->N;
+    int64_t left = h->Bstep < h->N ? h->Bstep : h->N;
+    while (left > 0) {
+      const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
+      if ((rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
+                                          h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
+                                          h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice,
+                                          h->copy_stream),
+                        "round_host: X copy")))
+        return rc;
+      if ((rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
+                                          n * 4, h->P, cudaMemcpyHostToDevice, h->copy_stream),
+                        "round_host: y copy")))
+        return rc;
+      left -= n;
+      r0 = 0;
+    }
+    if ((rc = h->cuda(cudaEventRecord(h->copied[k], h->copy_stream), "round_host: record"))) return rc;
+  }
+  if ((rc = do_round(h, &h->copied))) return rc;
+  if ((rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost, h->stream),
+                    "round_host: loss copy")))
     return rc;
   return hier_avg_check(h);
 }
