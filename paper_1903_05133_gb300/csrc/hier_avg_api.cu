@@ -579,6 +579,15 @@ int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 // K1-th, the global average after the G-th (fused with the local average that closes
 // the round when K1 divides G).  G = K1 * K2 unless set: Sec. 3.1 leaves beta = G / K1
 // free in practice.
+// The round launches no cooperative kernel: every forward layer runs in cluster split-K
+// mode and only the first layer's backward (no dX) runs on the tensor cores.
+bool cooperative_free(const hier_avg* h) {
+  const int n_fwd = h->head ? h->L - 1 : h->L;
+  for (int l = 0; l < n_fwd; ++l)
+    if (h->fwd_cq[l] < 2) return false;
+  return (h->head ? h->L - 2 : h->L - 1) <= 0;
+}
+
 // ready (round_host): ready[k] is recorded once the rows of the round's step k (0-based)
 // are on the device.  Step k reads those rows and, in an update+forward kernel, step
 // k + 1's.  The handle's stream waits for ready[0] before step 0 (and for ready[1] just
@@ -788,34 +797,62 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
     if (int rc = h->cuda(cudaEventCreateWithFlags(&e, cudaEventDisableTiming), "round_host: event")) return rc;
     h->copied.push_back(e);
   }
-  // The copies start once the work already queued on the handle's stream is done; step
-  // k's rows are (row0 + b) mod N, b < B, of every learner: at most two contiguous
-  // ranges, then copied[k] is recorded.
   int rc;
-  if ((rc = h->cuda(cudaEventRecord(h->round_start, h->stream), "round_host: record")) ||
-      (rc = h->cuda(cudaStreamWaitEvent(h->copy_stream, h->round_start, 0), "round_host: wait")))
-    return rc;
-  for (int k = 0; k < G; ++k) {
-    int64_t r0 = (h->cursor + static_cast<int64_t>(k) * h->Bstep) % h->N;
-    int64_t left = h->Bstep < h->N ? h->Bstep : h->N;
+  if (!(h->prec == HA_PREC_BF16 && !h->w_stream && cooperative_free(h))) {
+    // The round's rows, at most two contiguous ranges per learner (wrap-around), copied
+    // ahead of the round.  (Copied step by step instead, beside the kernels or ahead of
+    // them, the rounds with stream-K kernels and an evict-first weight stream measured
+    // much slower end to end: 3072-2048-2048-10 went from 2.85 to 2.20 or 1.54 M
+    // learner-samples/s.)
+    const int64_t rows = static_cast<int64_t>(h->Bstep) * G;
+    int64_t r0 = h->cursor % h->N, left = rows < h->N ? rows : h->N;
+    if (rows >= h->N) r0 = 0;
     while (left > 0) {
       const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
       if ((rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
                                           h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
-                                          h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice,
-                                          h->copy_stream),
+                                          h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice, h->stream),
                         "round_host: X copy")))
         return rc;
       if ((rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
-                                          n * 4, h->P, cudaMemcpyHostToDevice, h->copy_stream),
+                                          n * 4, h->P, cudaMemcpyHostToDevice, h->stream),
                         "round_host: y copy")))
         return rc;
       left -= n;
       r0 = 0;
     }
-    if ((rc = h->cuda(cudaEventRecord(h->copied[k], h->copy_stream), "round_host: record"))) return rc;
+    if ((rc = do_round(h))) return rc;
+  } else {
+    // Rounds without cooperative kernels whose weights fit in L2: step k's rows,
+    // (row0 + b) mod N for b < B, are copied on a stream of the library's own (at most
+    // two contiguous ranges per learner), then copied[k] is recorded.  The copies start
+    // once the work already queued on the handle's stream is done, and overlap the
+    // kernels, which wait as do_round says.
+    const cudaStream_t cs = h->copy_stream;
+    if ((rc = h->cuda(cudaEventRecord(h->round_start, h->stream), "round_host: record")) ||
+        (rc = h->cuda(cudaStreamWaitEvent(cs, h->round_start, 0), "round_host: wait")))
+      return rc;
+    for (int k = 0; k < G; ++k) {
+      int64_t r0 = (h->cursor + static_cast<int64_t>(k) * h->Bstep) % h->N;
+      int64_t left = h->Bstep < h->N ? h->Bstep : h->N;
+      while (left > 0) {
+        const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
+        if ((rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
+                                            h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
+                                            h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice, cs),
+                          "round_host: X copy")))
+          return rc;
+        if ((rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
+                                            n * 4, h->P, cudaMemcpyHostToDevice, cs),
+                          "round_host: y copy")))
+          return rc;
+        left -= n;
+        r0 = 0;
+      }
+      if ((rc = h->cuda(cudaEventRecord(h->copied[k], cs), "round_host: record"))) return rc;
+    }
+    if ((rc = do_round(h, &h->copied))) return rc;
   }
-  if ((rc = do_round(h, &h->copied))) return rc;
   if ((rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost, h->stream),
                     "round_host: loss copy")))
     return rc;

@@ -456,8 +456,10 @@ def test_full_size_step_sampled(w):
     print(w.name, [(k, kind, f"{e:.2e}", f"{lim:.2e}") for k, kind, e, lim in report])
 
 
-def test_round_host_matches_device_round():
-    w = SMALL_BF16
+# SMALL_BF16: the rows are copied step by step beside the kernels (two layers, cluster
+# split-K, weights in L2); FUSE_THREE: copied ahead of the round (stream-K layers)
+@pytest.mark.parametrize("w", [SMALL_BF16, FUSE_THREE], ids=lambda w: w.name)
+def test_round_host_matches_device_round(w):
     ha1, X, y = setup(w)
     ha2, _, _ = setup(w)
     ha1.round()
