@@ -145,3 +145,63 @@ def test_sgd_update_fp32_is_separate_multiply_subtract():
     want = (p.astype(np.float64) - step.astype(np.float64)).astype(np.float32)
     assert np.array_equal(got, want)
     assert got.dtype == np.float32
+
+
+def _bf16_step_in_torch(Ws, bs, X, y):
+    """One bf16-mode step written independently of the oracle, in torch float64:
+    every GEMM operand is cast explicitly with .to(bfloat16).to(float64), every
+    stored value with .to(float32).to(float64).  Operands: X, W_l and H_{l-1} in
+    the forward; dZ_l and H_{l-1} in dW_l; dZ_l and W_l (before its update) in the
+    dX product.  Bias add, ReLU, softmax cross-entropy and the bias gradient stay
+    in fp32 storage."""
+    f64, f32, b16 = torch.float64, torch.float32, torch.bfloat16
+
+    def bf(t):
+        return t.to(f32).to(b16).to(f64)
+
+    def st(t):
+        return t.to(f32).to(f64)
+
+    Wt = [torch.tensor(w, dtype=f64) for w in Ws]
+    bt = [torch.tensor(b, dtype=f64) for b in bs]
+    yt = torch.tensor(y)
+    B = X.shape[0]
+    Hs = [bf(torch.tensor(X, dtype=f64))]
+    Zs = []
+    for l in range(len(Wt)):
+        z = st(st(Hs[l] @ bf(Wt[l]).T) + bt[l])
+        Zs.append(z)
+        if l < len(Wt) - 1:
+            Hs.append(bf(st(torch.relu(z))))
+    z = Zs[-1].clone().requires_grad_(True)
+    loss = torch.nn.functional.cross_entropy(z, yt, reduction="mean")
+    loss.backward()
+    dz = st(z.grad)
+    gW, gb = [None] * len(Wt), [None] * len(Wt)
+    for l in reversed(range(len(Wt))):
+        gW[l] = st(bf(dz).T @ Hs[l])
+        gb[l] = st(dz.sum(dim=0))
+        if l > 0:
+            dh = st(bf(dz) @ bf(Wt[l]))
+            dz = st(dh * (Hs[l] > 0).to(f64))
+    return loss.item(), [g.numpy() for g in gW], [g.numpy() for g in gb]
+
+
+@pytest.mark.parametrize("dims,B", [((40, 24, 16, 10), 12), ((96, 72, 56, 13), 20)])
+def test_bf16_mode_operand_placement_against_torch(dims, B):
+    # Pins WHICH operands the bf16 mode rounds: a dropped or extra bf16 rounding of
+    # any one GEMM operand moves a gradient by ~2^-9 relative, far above 1e-12.
+    # X is drawn off the bf16 grid so that its rounding is checked too.
+    Ws, bs, X, y = _tiny_net(dims, B, 21)
+    Ws = [w.astype(np.float32).astype(np.float64) for w in Ws]
+    bs = [b.astype(np.float32).astype(np.float64) for b in bs]
+    X = X.astype(np.float32).astype(np.float64)
+    loss, gW, gb = ln.mlp_forward_backward(Ws, bs, X, y, "bf16")
+    loss_t, gW_t, gb_t = _bf16_step_in_torch(Ws, bs, X, y)
+    assert abs(loss - loss_t) <= 1e-12 * max(1.0, abs(loss_t))
+    for l in range(len(Ws)):
+        for a, b in ((gW[l], gW_t[l]), (gb[l], gb_t[l])):
+            assert np.max(np.abs(a - b)) <= 1e-12 * np.max(np.abs(b)), l
+    # the placement matters at this size: the fp32 mode differs from it
+    _, gW32, _ = ln.mlp_forward_backward(Ws, bs, X, y, "fp32")
+    assert all(np.max(np.abs(a - b)) > 1e-6 * np.max(np.abs(b)) for a, b in zip(gW32, gW_t))
