@@ -6,9 +6,12 @@ SGD steps of all P learners + a local average) + the global average, on
 synthetic Gaussian-mixture data already resident in HBM.  The metric is
 learner-samples per second (P * B * K1 * K2 per round).
 
-  python bench.py [--gpus N --steps K --warmup W] [--workload mlp512|mlp2048|mlp4096|softmax]
+  python bench.py [--gpus N --steps K --warmup W] [--workload mlp4096|mlp2048|mlp512|softmax]
   python bench.py --impl reference ...   # the CPU oracle on a bounded sample
   python bench.py --sweep                # averaging-only sweep (P = 128), GB/s table
+
+The default workload is the largest one that fits one GPU: 32 learners of the
+ImageNet-shaped MLP 12288 -> 4096 -> 4096 -> 1000 (about 71M parameters each).
 
 Under torchrun (N > 1) every rank runs an independent replica on its own GPU
 (the learners of one replica never leave their GPU), timing is max over ranks
@@ -42,10 +45,12 @@ def parse():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="mlp512")
+    ap.add_argument("--workload", default="mlp4096")
     ap.add_argument("--sweep", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-sweep-point", action="store_true",
+                    help="skip the averaging-only point (P = 128, D = 64M) in the JSON line")
     ap.add_argument("--N", type=int, default=None,
                     help="samples per learner (default: the workload's); for small profiling runs")
     ap.add_argument("--P", type=int, default=None,
@@ -151,9 +156,11 @@ def src_hash(*names):
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(kind: str, workload: str):
-    """DRAM bytes per launch of a kernel from a committed ncu summary, if the
-    kernel source has not changed since it was captured."""
+def ncu_traffic(kind: str, workload: str, P: int):
+    """DRAM bytes per launch of a kernel from a committed ncu summary, if the kernel
+    source has not changed since it was captured.  A capture taken with fewer
+    learners (``captured_P``) is scaled to P: every learner's weights are streamed
+    once per launch, so the bytes grow in proportion to the learners."""
     p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(p):
         return None
@@ -164,32 +171,22 @@ def ncu_traffic(kind: str, workload: str):
         return None
     if e.get("source_hash") != src_hash(*e.get("sources", [])):
         return None
-    return e.get("dram_bytes_per_launch")
+    by = e.get("dram_bytes_per_launch")
+    cp = e.get("captured_P")
+    return by * P / cp if (by is not None and cp) else by
+
+
+def run_config(w, ws: int) -> dict:
+    """The workload as both arms of the bench name it."""
+    return {"workload": w.name, "P": w.P, "S": w.S, "K1": w.K1, "K2": w.K2, "B": w.B,
+            "dims": list(w.dims), "lr": w.lr, "N": w.N,
+            "parallelism": f"{w.P} simulated learners per GPU" + (f" x {ws} replicas" if ws > 1 else ""),
+            "l2": f"GPU arm: flushed between timed rounds ({L2_FLUSH_BYTES >> 20} MB write, untimed); "
+                  f"parameters {w.P * w.n_params * 4 / 1e9:.2f} GB",
+            "master": "fp32", "gemm_operands": w.precision}
 
 
 # ----------------------------------------------------------------------------- oracle
-def oracle_block_time(w, X, y, layers, n_blocks: int = 1):
-    """Time the CPU oracle on one local block (K1 local steps of every learner +
-    one local average) per call; returns (seconds per block, samples per block)."""
-    import numpy as np
-    import oracle
-    mode = "fp32" if w.precision == "fp32" else "bf16"
-    params = []
-    for Wl, bl in layers:
-        params += [np.broadcast_to(Wl.numpy(), (w.P,) + tuple(Wl.shape)).copy(),
-                   np.broadcast_to(bl.numpy(), (w.P,) + tuple(bl.shape)).copy()]
-    prob = oracle.MLPProblem(X.float().numpy(), y.numpy().astype(np.int64), w.B, len(w.dims) - 1, mode)
-    o = oracle.HierAvgOracle(w.P, w.S, w.K1, w.K2, w.lr, prob, params, mode)
-    times = []
-    for _ in range(n_blocks):
-        t0 = time.perf_counter()
-        for _k in range(w.K1):
-            o.step()
-        o.local_average()
-        times.append(time.perf_counter() - t0)
-    return times, w.P * w.B * w.K1
-
-
 def cpu_cores():
     try:
         return len(os.sched_getaffinity(0))
@@ -197,35 +194,146 @@ def cpu_cores():
         return os.cpu_count()
 
 
+class OracleSample:
+    """The CPU oracle, as it stands, on a bounded sample of a Hier-AVG round.
+
+    A round is P * K1 * K2 learner steps plus K2 local averages of P / S clusters and
+    one global average.  One sample times ``steps`` local SGD steps of one learner
+    (learner 0, on its own data, batches read as in the round) and the local average
+    of one cluster of S learners over a 1 / ``avg_split`` slice of the parameter row.
+    The round's time is extrapolated from them: the learner steps times P * K1 * K2,
+    the cluster average (times avg_split) times K2 * P / S, and the global average
+    as (P - 1) / (S - 1) cluster averages (a tree over P rows instead of S)."""
+
+    def __init__(self, w, X0, y0, layers):
+        import numpy as np
+        import oracle
+        self.w = w
+        self.mode = "fp32" if w.precision == "fp32" else "bf16"
+        params = []
+        for Wl, bl in layers:
+            params += [Wl.numpy()[None].copy(), bl.numpy()[None].copy()]
+        prob = oracle.MLPProblem(X0.float().numpy(), y0.numpy().astype(np.int64), w.B,
+                                 len(w.dims) - 1, self.mode)
+        self.learner = oracle.HierAvgOracle(1, 1, w.K1, w.K2, w.lr, prob, params, self.mode)
+        D = w.n_params
+        self.avg_split = 8 if D * w.S * 4 > (1 << 30) else 1
+        cols = -(-D // self.avg_split)
+        rng = np.random.default_rng(0)
+        self.cluster = rng.standard_normal((w.S, cols), dtype=np.float32)
+        self.steps = 1 if D > 10_000_000 else w.K1
+
+    def run(self):
+        """One sample: (seconds of the learner steps, seconds of the slice average)."""
+        import oracle
+        t0 = time.perf_counter()
+        for _ in range(self.steps):
+            self.learner.step()
+        t1 = time.perf_counter()
+        oracle.local_average(self.cluster, self.w.S)
+        t2 = time.perf_counter()
+        return t1 - t0, t2 - t1
+
+    def round_seconds(self, t_steps: float, t_avg: float) -> float:
+        w = self.w
+        per_step = t_steps / self.steps
+        per_cluster_avg = t_avg * self.avg_split
+        avgs = w.K2 * (w.P // w.S) + (w.P - 1) / max(1, w.S - 1)
+        return w.P * w.K1 * w.K2 * per_step + avgs * per_cluster_avg
+
+    def describe(self) -> str:
+        w = self.w
+        frac = f"1/{self.avg_split} of the {w.n_params}-parameter row" if self.avg_split > 1 \
+            else f"the whole {w.n_params}-parameter row"
+        return (f"extrapolated: {self.steps} local SGD step(s) of one learner (B = {w.B}) and one local "
+                f"average of {w.S} learners over {frac}, scaled to a round ({w.P * w.K1 * w.K2} learner "
+                f"steps, {w.K2 * (w.P // w.S)} cluster averages, one global average counted as "
+                f"(P-1)/(S-1) cluster averages); numpy, {self.mode} operands, float64 products, "
+                f"multi-threaded BLAS")
+
+
+def oracle_inputs_cpu(w, X0=None, y0=None):
+    """Learner 0's data (generated on the CPU unless given) and the shared w0."""
+    from paper_1903_05133_gb300.inputs import initial_layers, learner_data
+    if X0 is None:
+        X0, y0 = learner_data(w, learners=[0])
+    return X0, y0, initial_layers(w)
+
+
 def run_reference(args):
+    """The CPU oracle timed as it stands on the host cores: every bench step is one
+    bounded sample of the workload's round (OracleSample), and the value is the
+    round's learner-samples over the extrapolated round time."""
     ws, rank, _ = dist_env()
     if rank != 0:
         return 0
     from paper_1903_05133_gb300 import configs
-    from paper_1903_05133_gb300.inputs import initial_layers, learner_data
     w = configs.SHORT[args.workload]
-    X, y = learner_data(w)
-    layers = initial_layers(w)
-    times, samples = oracle_block_time(w, X, y, layers, args.warmup + args.steps)
-    timed = times[args.warmup:]
-    T = sum(timed)
-    value = samples * len(timed) / T
-    sample = (f"one local block per step: {w.K1} local SGD steps of all {w.P} learners + one local "
-              f"average ({samples} learner-samples, 1/{w.K2} of a round; the global average is "
-              f"not in the sample)")
+    X0, y0, layers = oracle_inputs_cpu(w)
+    smp = OracleSample(w, X0, y0, layers)
+    runs = [smp.run() for _ in range(args.warmup + args.steps)][args.warmup:]
+    ts = statistics.mean(r[0] for r in runs)
+    ta = statistics.mean(r[1] for r in runs)
+    value = w.samples_per_round / smp.round_seconds(ts, ta)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * T / len(timed),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16-operands/f64-acc",
-            "data": "synthetic", "config": {"workload": w.name, "P": w.P, "S": w.S, "K1": w.K1,
-                                            "K2": w.K2, "B": w.B, "dims": list(w.dims)},
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000 * statistics.mean(a + b for a, b in runs),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16-operands/f64-products" if w.precision == "bf16" else "f32/f64-products",
+            "data": "synthetic (seeded Gaussian mixture, CIFAR-10 / ImageNet shaped)",
+            "config": run_config(w, ws),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
-                             "sample": sample},
+                             "sample": smp.describe() + "; each bench step is one sample"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
 
 
 # ----------------------------------------------------------------------------- ours
+def gemm_report(by: float, fl: float, ms: float, hbm_gbs: float, tc_tflops: float) -> dict:
+    """TFLOP/s of a set of launches against the tensor-core rate, next to the ceiling
+    that the HBM roofline sets for their arithmetic intensity (flops per byte)."""
+    tflops = fl / (ms / 1e3) / 1e12
+    ceiling = min(tc_tflops, (fl / by) * hbm_gbs / 1e3) if by > 0 else tc_tflops
+    return {"TFLOPs": round(tflops, 2), "tensor_frac": round(tflops / tc_tflops, 4),
+            "flop_per_byte": round(fl / by, 2) if by > 0 else None,
+            "hbm_bound_tensor_frac_ceiling": round(ceiling / tc_tflops, 4),
+            "frac_of_hbm_bound_ceiling": round(tflops / ceiling, 4)}
+
+
+def averaging_point(dev, flush, hbm_gbs: float) -> dict:
+    """One point of the averaging-only sweep: P = 128 fp32 learner rows of D = 64M
+    parameters (32.8 GB, far above L2), the local average over clusters of S = 8 and
+    the fused last-local + global average; L2 flushed before every timed launch."""
+    import torch
+    from paper_1903_05133_gb300.hier_avg import local_average_buffer, local_global_average_buffer
+    from paper_1903_05133_gb300.inputs import replica_matrix
+    P, D, S = 128, 64_000_000, 8
+    wm = replica_matrix(P, D, device=dev)
+    out = {"P": P, "D": D, "S": S, "bytes_per_pass": 8.0 * P * D,
+           "timing": "median of 7 launches, CUDA events, L2 flushed before each"}
+    for op, fn in (("local", lambda: local_average_buffer(wm, S)),
+                   ("local_global", lambda: local_global_average_buffer(wm, S))):
+        fn()
+        ms = []
+        for _ in range(7):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            ms.append(a.elapsed_time(b))
+        med = statistics.median(ms)
+        gbs = 8.0 * P * D / (med / 1e3) / 1e9
+        out[op] = {"ms": round(med, 4), "GBps": round(gbs, 1), "frac_of_measured_hbm": round(gbs / hbm_gbs, 4),
+                   "frac_of_8TBps": round(gbs / 8000.0, 4)}
+    del wm
+    torch.cuda.empty_cache()
+    return out
+
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -246,6 +354,7 @@ def run_ours(args):
             raise SystemExit(f"--P must be a multiple of S = {w.S}")
         w = w.replace(P=args.P)
     X, y = learner_data(w, device=dev)
+    X0c, y0c = X[:1].cpu(), y[:1].cpu()          # learner 0's data for the CPU oracle
     layers = initial_layers(w, device=dev)
     ha = HierAvg(w.P, w.S, w.K1, w.K2, w.lr, w.B, w.dims, w.precision)
     params = ha.pack(layers, device=dev)
@@ -270,7 +379,7 @@ def run_ours(args):
     ha.profile(False)
     main_kinds = ["forward", "backward", "local_avg", "global_avg", "xent", "gather", "head",
                   "update_forward"]
-    dom = max(main_kinds, key=lambda k: prof[k][0])
+    dom = max(main_kinds, key=lambda k: prof[k].total_ms)
 
     props = torch.cuda.get_device_properties(dev)
     uuid = str(getattr(props, "uuid", "") or "")
@@ -316,41 +425,57 @@ def run_ours(args):
         torch.cuda.synchronize()
         plain_ms.append(a_ev.elapsed_time(b_ev))
     pk, pk_src = peaks()
-    dom_ms, dom_n, dom_bytes = dom_live
+    hbm = pk["hbm_gbs"]
+    tc = pk.get("bf16_tflops_sustained") or pk["bf16_tflops"]
+    dom_ms, dom_n, dom_bytes, dom_flops = dom_live
     achieved = dom_bytes / (dom_ms / 1e3) / 1e9 if dom_ms > 0 else None
     kernels = {}
+    total_ms = max(1e-9, sum(v.total_ms for v in prof.values()))
     for k in kinds:
-        ms, n, by = prof[k]
-        if n:
-            kernels[k] = {"launches": n, "total_ms": round(ms, 4), "avg_us": round(1e3 * ms / n, 2),
-                          "share": round(ms / max(1e-9, sum(v[0] for v in prof.values())), 4),
-                          "GBps": round(by / (ms / 1e3) / 1e9, 1) if ms > 0 else None}
-    avg_ms = prof["local_avg"][0] + prof["global_avg"][0]
-    avg_by = prof["local_avg"][2] + prof["global_avg"][2]
-    # per-launch DRAM bytes scale with P: a run with fewer learners has no captured figure
-    traffic = ncu_traffic(dom, w.name) if not args.P else None
-    roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"],
-                "unit": "GB/s", "frac": (achieved / pk["hbm_gbs"]) if achieved else None,
-                "peak_source": pk_src,
+        ms, n, by, fl = prof[k]
+        if n and ms > 0:
+            e = {"launches": n, "total_ms": round(ms, 4), "avg_us": round(1e3 * ms / n, 2),
+                 "share": round(ms / total_ms, 4), "GBps": round(by / (ms / 1e3) / 1e9, 1)}
+            if fl > 0 and k not in ("local_avg", "global_avg"):
+                e.update(gemm_report(by, fl, ms, hbm, tc))
+            kernels[k] = e
+    avg_ms = prof["local_avg"].total_ms + prof["global_avg"].total_ms
+    avg_by = prof["local_avg"].bytes + prof["global_avg"].bytes
+    step_kinds = ("forward", "backward", "update_forward", "head")
+    step_ms = sum(prof[k].total_ms for k in step_kinds)
+    step_fl = sum(prof[k].flops for k in step_kinds)
+    step_by = sum(prof[k].bytes for k in step_kinds)
+    traffic = ncu_traffic(dom, w.name, w.P) if not (args.P or args.N) else None
+    roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm,
+                "unit": "GB/s", "frac": (achieved / hbm) if achieved else None,
+                "peak_source": f"{pk_src} (HBM copy)",
                 "traffic": traffic,
                 "algorithmic_bytes_per_launch": dom_bytes / max(1, dom_n),
                 "avg_launch_us": 1e3 * dom_ms / max(1, dom_n),
                 "timing": f"CUDA events around every {DOM_SAMPLE}th launch of this kernel inside the timed rounds",
                 "launches_timed": dom_n}
+    if dom_flops > 0:
+        roofline["tensor"] = gemm_report(dom_bytes, dom_flops, dom_ms, hbm, tc)
+    l2_bytes = torch.cuda.get_device_properties(dev).L2_cache_size
+    params_bytes = 4.0 * w.P * ha.ld
 
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1000 * T / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": w.precision,
             "data": "synthetic (seeded Gaussian mixture, CIFAR-10 / ImageNet shaped)",
-            "config": {"workload": w.name, "P": w.P, "S": w.S, "K1": w.K1, "K2": w.K2, "B": w.B,
-                       "dims": list(w.dims), "lr": w.lr, "N": w.N,
-                       "parallelism": f"{w.P} simulated learners per GPU" + (f" x {ws} replicas" if ws > 1 else ""),
-                       "l2": f"flushed between timed rounds ({L2_FLUSH_BYTES >> 20} MB write, untimed)",
-                       "master": "fp32", "gemm_operands": w.precision},
+            "config": run_config(w, ws),
             "roofline": roofline,
+            "gemm": dict(gemm_report(step_by, step_fl, step_ms, hbm, tc),
+                         note="all learner-step kernels of a round (forward, backward, "
+                              "update+forward, head) from the profiling pass; bf16 operands, "
+                              "fp32 accumulate; tensor fractions of the measured sustained "
+                              "bf16 dense rate"),
             "averaging": {"GBps": avg_by / (avg_ms / 1e3) / 1e9 if avg_ms > 0 else None,
-                          "frac_of_measured_hbm": (avg_by / (avg_ms / 1e3) / 1e9 / pk["hbm_gbs"]) if avg_ms > 0 else None,
-                          "frac_of_8TBps": (avg_by / (avg_ms / 1e3) / 8e12) if avg_ms > 0 else None},
+                          "frac_of_measured_hbm": (avg_by / (avg_ms / 1e3) / 1e9 / hbm) if avg_ms > 0 else None,
+                          "frac_of_8TBps": (avg_by / (avg_ms / 1e3) / 8e12) if avg_ms > 0 else None,
+                          "l2_assisted": params_bytes <= l2_bytes,
+                          "note": "in-round local and global averages; with all parameters "
+                                  "smaller than L2 part of each average is served from L2"},
             "kernels": kernels,
             "kernels_timing": "untimed profiling pass before the timed rounds, events around every launch",
             "ms_per_step_without_kernel_events": statistics.median(plain_ms),
@@ -378,16 +503,21 @@ def run_ours(args):
                        "h2d_bytes_per_step": w.P * rows * (w.dims[0] * es + 4),
                        "d2h_bytes_per_step": w.P * 4,
                        "api": "hier_avg_round_host (pinned host X, y; loss read back)"}
+        del Xh, yh
+
+    if rank == 0 and not args.no_sweep_point:
+        del ha, params, X, y
+        torch.cuda.empty_cache()
+        line["averaging_sweep"] = averaging_point(dev, flush, hbm)
 
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        Xc, yc = X.cpu(), y.cpu()
-        lc = [(Wl.cpu(), bl.cpu()) for Wl, bl in layers]
-        times, samples = oracle_block_time(w, Xc, yc, lc, 1)
-        line["cpu_baseline"] = {"value": samples / times[0], "unit": UNIT, "cores": cpu_cores(),
-                                "kind": "oracle",
-                                "sample": f"one local block: {w.K1} local steps of all {w.P} learners "
-                                          f"+ one local average ({samples} learner-samples), numpy "
-                                          f"(float64 BLAS products, multi-threaded BLAS)"}
+        X0, y0, lc = oracle_inputs_cpu(w, X0c, y0c)
+        smp = OracleSample(w, X0, y0, lc)
+        smp.run()                                           # warm-up sample
+        ts, ta = smp.run()
+        v = w.samples_per_round / smp.round_seconds(ts, ta)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                                "sample": smp.describe()}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:

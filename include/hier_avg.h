@@ -16,6 +16,8 @@
  *     bound to the handle); a NULL stream is the legacy default stream.  Only
  *     hier_avg_losses, hier_avg_check, hier_avg_round_host and the profile read
  *     synchronise.
+ *   - No call changes the calling thread's current CUDA device: a call that runs
+ *     work on the handle's device makes it current and restores the caller's.
  *   - Every call returns HA_OK (0) or a negative status; nothing aborts.
  *     hier_avg_strerror() names a status, hier_avg_last_error() gives the
  *     message of the handle's last failure.
@@ -171,7 +173,8 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host,
  * The call binds the handle to these buffers and to that array, clears the part
  * of the array the step uses, takes the step at the handle's counter t and
  * advances t.  It calls no device allocator.
- *   - The first call on a device looks up the array's device address; make that
+ *   - The first call in each CUDA context of a device (so once per device, and
+ *     again after a device reset) looks up the array's device address; make that
  *     first call before any stream capture on that device.
  *   - Every call, from any handle, shares the one array and leaves its contents
  *     behind; calls whose work overlaps on the GPU (other streams, other
@@ -197,6 +200,18 @@ int hier_avg_losses(hier_avg* h, float* loss_host);
  * HA_ETIMEOUT if a bounded wait inside a kernel expired (that kernel stopped
  * early and its outputs are invalid), HA_ECUDA on an asynchronous CUDA error. */
 int hier_avg_check(hier_avg* h);
+
+/* Failure-detection self-test (the paper has no counterpart: this checks the
+ * library's own failure detection).  Launches one kernel on the bound stream that
+ * runs the library's two kinds of bounded device wait -- an acquire spin on a global
+ * flag and an mbarrier phase wait, the waits that order split-K reductions and the
+ * TMA / tensor-core pipelines -- on conditions nothing will satisfy, each with a limit
+ * of limit_us microseconds at the device's peak SM clock (longer at a lower clock).
+ * Both expire; the kernel records the timeout in the handle's error word and returns
+ * with nothing in flight, so the CUDA context stays usable.  The next hier_avg_check
+ * returns HA_ETIMEOUT and clears the word; later calls work as before.
+ * Errors: HA_ESTATE before bind, HA_EINVAL for limit_us outside [1, 1e7], HA_ECUDA. */
+int hier_avg_wait_selftest(hier_avg* h, int64_t limit_us);
 
 /* Kernel timing with CUDA events recorded on the bound stream around every
  * launch of the handle.  enable = 1 starts (and clears) it, 0 stops it. */
@@ -228,9 +243,12 @@ int hier_avg_launches(const hier_avg* h, int64_t* launches);
 int hier_avg_profile_every(hier_avg* h, int every);
 
 /* Synchronise and read kind's totals since profiling was enabled: summed event
- * time in ms, number of launches, and the algorithmic bytes moved by them. */
+ * time in ms, number of launches, the algorithmic bytes moved by them (fp32 master
+ * read and written, activations read and written once) and their algorithmic flops
+ * (2 per multiply-add of the step's products: forward, dW and dX of every learner;
+ * P * ld additions per average).  Any output pointer may be NULL. */
 int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* launches,
-                          double* bytes);
+                          double* bytes, double* flops);
 
 const char* hier_avg_strerror(int status);
 const char* hier_avg_last_error(const hier_avg* h);

@@ -38,6 +38,7 @@ SIGNATURES = {
     "hier_avg_set_step": (c_int, [c_void_p, c_int64]),
     "hier_avg_losses": (c_int, [c_void_p, c_void_p]),
     "hier_avg_check": (c_int, [c_void_p]),
+    "hier_avg_wait_selftest": (c_int, [c_void_p, c_int64]),
     "hier_avg_profile": (c_int, [c_void_p, c_int]),
     "hier_avg_profile_kinds": (c_int, [c_void_p, ctypes.c_uint]),
     "hier_avg_launches": (c_int, [c_void_p, c_void_p]),
@@ -45,7 +46,7 @@ SIGNATURES = {
     "hier_avg_set_lr": (c_int, [c_void_p, ctypes.c_float]),
     "hier_avg_set_batch": (c_int, [c_void_p, c_int]),
     "hier_avg_profile_every": (c_int, [c_void_p, c_int]),
-    "hier_avg_profile_read": (c_int, [c_void_p, c_int, P_double, P_int64, P_double]),
+    "hier_avg_profile_read": (c_int, [c_void_p, c_int, P_double, P_int64, P_double, P_double]),
     "hier_avg_strerror": (c_char_p, [c_int]),
     "hier_avg_last_error": (c_char_p, [c_void_p]),
 }

@@ -15,6 +15,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace {
 
@@ -46,7 +47,7 @@ EncodeTiledFn encode_fn() {
 struct ProfRec {
   int kind;
   cudaEvent_t a, b;
-  double bytes;
+  double bytes, flops;
 };
 
 }  // namespace
@@ -118,6 +119,8 @@ struct hier_avg {
   template <class T>
   T* wsp(int64_t off) { return reinterpret_cast<T*>(ws + off); }
   int* err_word() { return wsp<int>(off_err); }
+  // A word next to the error word that no kernel ever writes (stays zero).
+  const int* never_set() { return wsp<int>(off_err) + 1; }
   float* loss() { return wsp<float>(off_loss); }
 
   cudaEvent_t ev() {
@@ -128,9 +131,10 @@ struct hier_avg {
     }
     return pool[pool_used++];
   }
-  // Bracket one launch with events when profiling is on.
+  // Bracket one launch with events when profiling is on.  bytes and flops: the
+  // launch's algorithmic memory traffic and arithmetic (multiply-adds count two).
   template <class F>
-  int timed(int kind, double bytes, F&& launch, const char* what) {
+  int timed(int kind, double bytes, double flops, F&& launch, const char* what) {
     cudaEvent_t a = nullptr, b = nullptr;
     bool on = (prof >> kind) & 1u;
     if (on) on = prof_seen[kind]++ % prof_every == 0;
@@ -144,7 +148,7 @@ struct hier_avg {
     if (e != cudaSuccess) return cuda(e, what);
     if (on && a && b) {
       cudaEventRecord(b, stream);
-      recs.push_back({kind, a, b, bytes});
+      recs.push_back({kind, a, b, bytes, flops});
     }
     return HA_OK;
   }
@@ -299,9 +303,28 @@ int build_maps(hier_avg* h) {
 int check_bound(hier_avg* h) {
   if (!h) return HA_EINVAL;
   if (!h->bound) return h->fail(HA_ESTATE, "hier_avg_bind has not been called");
-  cudaSetDevice(h->device);
   return HA_OK;
 }
+
+// Makes a device current for the lifetime of the object and gives the calling
+// thread its previous current device back afterwards, so that no entry point
+// changes the caller's device.
+class DeviceScope {
+ public:
+  explicit DeviceScope(int device) {
+    if (cudaGetDevice(&prev_) == cudaSuccess && prev_ != device)
+      changed_ = cudaSetDevice(device) == cudaSuccess;
+  }
+  ~DeviceScope() {
+    if (changed_) cudaSetDevice(prev_);
+  }
+  DeviceScope(const DeviceScope&) = delete;
+  DeviceScope& operator=(const DeviceScope&) = delete;
+
+ private:
+  int prev_ = 0;
+  bool changed_ = false;
+};
 
 // Algorithmic bytes of the big kernels (fp32 master read + write, activations).
 double bytes_forward(const hier_avg* h, int l) {
@@ -320,6 +343,12 @@ double bytes_backward(const hier_avg* h, int l) {
   const double act = h->prec == HA_PREC_BF16 ? 2.0 : 4.0;
   const double dx = l > 0 ? (B * in * act + in * 8.0) : 0.0;
   return P * (in * out * 8.0 + B * in * act + B * out * act + dx);
+}
+
+// Algorithmic flops of the learner-step products (2 per multiply-add): one
+// [B x in] x [in x out] product per learner for the forward, dW and dX each.
+double flops_gemm(const hier_avg* h, int l) {
+  return 2.0 * h->P * h->Bstep * double(h->dims[l]) * h->dims[l + 1];
 }
 
 // Arguments of the small last layer (input H_{L-1}, or X rows for a one-layer model).
@@ -370,7 +399,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     const int64_t r0 = h->cursor % h->N;   // this step's batch: rows r0 .. (mod N)
     const bool x_direct = r0 + B <= h->N;
     if (!x_direct) {
-      rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, [&] {
+      rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 2 * 3, 0.0, [&] {
         return ha::launch_gather_bf16(static_cast<const __nv_bfloat16*>(h->X), h->N, d0, B, h->Bn,
                                       h->pitch[0], r0, P, h->wsp<__nv_bfloat16>(h->off_H[0]), s);
       }, "gather");
@@ -414,7 +443,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       }
       a.err = h->err_word();
       const CUtensorMap& hin = a.x_direct ? h->tm_x : h->tm_h[l];
-      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), [&] {
+      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), flops_gemm(h, l), [&] {
         return ha::launch_tc_forward(h->tm_wf[l], hin, a, P, s);
       }, "forward");
       if (rc) return rc;
@@ -423,10 +452,11 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     if (h->head) {
       const ha::HeadArgs a = head_args(h);
       const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0));
-      rc = h->timed(HA_KERNEL_HEAD, hb, [&] { return ha::launch_head(a, P, s); }, "head");
+      const double hf = flops_gemm(h, L - 1) * (L > 1 ? 3 : 2);   // forward, dW (, dX)
+      rc = h->timed(HA_KERNEL_HEAD, hb, hf, [&] { return ha::launch_head(a, P, s); }, "head");
       if (rc) return rc;
     } else if (!h->fused_xent) {
-      rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, [&] {
+      rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, 0.0, [&] {
         return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, r0, B, h->Bn, C,
                                     h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
                                     h->wsp<__nv_bfloat16>(h->off_dZ[L]), h->loss(), P, s);
@@ -487,7 +517,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.err = h->err_word();
         if (next_rows && (rc = h->cuda(cudaStreamWaitEvent(s, next_rows, 0), "round_host: wait for the rows")))
           return rc;
-        rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h), [&] {
+        rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h), 2 * flops_gemm(h, 0), [&] {
           return ha::launch_tc_update_forward(h->tm_wf[0], hin, h->tm_x, h->tm_dz[1], f, s);
         }, "update+forward");
         if (rc) return rc;
@@ -499,14 +529,14 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       // the even static split, which work items that coarse would unbalance.
       const int64_t units = int64_t(a.n_tiles) * ((a.out + 63) / 64);
       if (a.has_dx || units < int64_t(kTargetCtas) * 64) {
-        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
           return ha::launch_tc_backward(h->tm_wb[l], hin, h->tm_dz[l + 1], a, P, s);
         }, "backward");
       } else {
         // no dX: independent units, handed out dynamically
         a.dyn = h->wsp<int>(h->off_dyn);
         a.ctas = kTargetCtas;
-        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
           return ha::launch_tc_update(h->tm_wb[l], hin, h->tm_dz[l + 1], a, s);
         }, "backward");
       }
@@ -514,7 +544,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     }
   } else {
     const int d0 = h->dims[0];
-    rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 4 * 2, [&] {
+    rc = h->timed(HA_KERNEL_GATHER, double(P) * B * d0 * 4 * 2, 0.0, [&] {
       return ha::launch_gather_f32(static_cast<const float*>(h->X), h->N, d0, B, h->cursor % h->N, P,
                                    h->wsp<float>(h->off_H[0]), s);
     }, "gather");
@@ -522,20 +552,20 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     for (int l = 0; l < L; ++l) {
       const bool last = l + 1 == L;
       float* outp = last ? h->wsp<float>(h->off_Z) : h->wsp<float>(h->off_H[l + 1]);
-      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), [&] {
+      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), flops_gemm(h, l), [&] {
         return ha::launch_fwd_f32(h->wsp<float>(h->off_H[l]), h->params + h->woff[l],
                                   h->params + h->boff[l], h->ld, h->dims[l], h->dims[l + 1], B,
                                   last ? 0 : 1, outp, P, s);
       }, "forward");
       if (rc) return rc;
     }
-    rc = h->timed(HA_KERNEL_XENT, double(P) * B * h->dims[L] * 4 * 2, [&] {
+    rc = h->timed(HA_KERNEL_XENT, double(P) * B * h->dims[L] * 4 * 2, 0.0, [&] {
       return ha::launch_xent_f32(h->wsp<float>(h->off_Z), h->y, h->N, h->cursor % h->N, B, h->dims[L],
                                  h->wsp<float>(h->off_dZ[L]), h->loss(), P, s);
     }, "xent");
     if (rc) return rc;
     for (int l = L - 1; l >= 0; --l) {
-      rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), [&] {
+      rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
         cudaError_t e = cudaSuccess;
         if (l > 0) ++h->launches;   // dX is its own launch
         if (l > 0)
@@ -556,19 +586,19 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
 }
 
 int do_local(hier_avg* h) {
-  return h->timed(HA_KERNEL_LOCAL_AVG, 8.0 * h->P * h->ld, [&] {
+  return h->timed(HA_KERNEL_LOCAL_AVG, 8.0 * h->P * h->ld, double(h->P) * h->ld, [&] {
     return ha::launch_group_mean(h->params, h->P, h->S, h->ld, h->ld, h->stream);
   }, "local average");
 }
 
 int do_local_global(hier_avg* h) {
-  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, [&] {
+  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, double(h->P) * h->ld, [&] {
     return ha::launch_local_global_mean(h->params, h->P, h->S, h->ld, h->ld, h->stream);
   }, "local+global average");
 }
 
 int do_global(hier_avg* h) {
-  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, [&] {
+  return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, double(h->P) * h->ld, [&] {
     return ha::launch_group_mean(h->params, h->P, h->P, h->ld, h->ld, h->stream);
   }, "global average");
 }
@@ -614,6 +644,25 @@ int do_round(hier_avg* h, const std::vector<cudaEvent_t>* ready = nullptr) {
   return G % h->K1 == 0 ? do_local_global(h) : do_global(h);
 }
 
+// Failure-detection self-test: the library's two kinds of bounded device wait, each
+// on a condition that nothing will ever satisfy.  Thread 0 waits with acquire order
+// for a global word to become 1 (it stays 0), then for the first phase of an mbarrier
+// that no thread arrives on.  Each wait gives up after `limit` cycles of SM clock and
+// records HA_DEVERR_TIMEOUT in the error word; the kernel then returns.  Nothing is in
+// flight when it exits (no copy, no MMA), so the context stays usable.
+__global__ void k_wait_selftest(const int* never_set, int* err, long long limit) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    ha::mbar_init(&bar, 1);
+    ha::fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    ha::spin_acquire_eq(never_set, 1, err, limit);
+    ha::mbar_wait(&bar, 0, err, limit);
+  }
+}
+
 }  // namespace
 
 extern "C" {
@@ -633,23 +682,26 @@ const char* hier_avg_strerror(int status) {
 
 const char* hier_avg_last_error(const hier_avg* h) { return h ? h->err.c_str() : "null handle"; }
 
-static int check_avg_args(const float* w, int64_t P, int64_t S, int64_t D, int64_t ld) {
+// groups: how many independent means one launch takes (one per grid row).
+static int check_avg_args(const float* w, int64_t P, int64_t S, int64_t D, int64_t ld,
+                          int64_t groups) {
   if (P < 1 || S < 1 || P % S != 0 || D < 0 || ld < D) return HA_EINVAL;
   if (D > 0 && !w) return HA_EINVAL;
   if (P > (int64_t(1) << 30) || D > (int64_t(1) << 40)) return HA_EINVAL;
+  if (groups > 65535) return HA_EUNSUPPORTED;   // the group index is a grid dimension
   return HA_OK;
 }
 
 int hier_avg_local_average_buffer(float* w_dev, int64_t P, int64_t S, int64_t D, int64_t ld,
                                   void* stream) {
-  if (int rc = check_avg_args(w_dev, P, S, D, ld)) return rc;
+  if (int rc = check_avg_args(w_dev, P, S, D, ld, S > 0 ? P / S : 0)) return rc;
   return ha::launch_group_mean(w_dev, P, S, D, ld, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? HA_OK
              : HA_ECUDA;
 }
 
 int hier_avg_global_average_buffer(float* w_dev, int64_t P, int64_t D, int64_t ld, void* stream) {
-  if (int rc = check_avg_args(w_dev, P, 1, D, ld)) return rc;
+  if (int rc = check_avg_args(w_dev, P, 1, D, ld, 1)) return rc;
   return ha::launch_group_mean(w_dev, P, P, D, ld, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? HA_OK
              : HA_ECUDA;
@@ -657,7 +709,7 @@ int hier_avg_global_average_buffer(float* w_dev, int64_t P, int64_t D, int64_t l
 
 int hier_avg_local_global_average_buffer(float* w_dev, int64_t P, int64_t S, int64_t D,
                                          int64_t ld, void* stream) {
-  if (int rc = check_avg_args(w_dev, P, S, D, ld)) return rc;
+  if (int rc = check_avg_args(w_dev, P, S, D, ld, 1)) return rc;
   return ha::launch_local_global_mean(w_dev, P, S, D, ld, static_cast<cudaStream_t>(stream)) ==
                  cudaSuccess
              ? HA_OK
@@ -740,7 +792,7 @@ int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t w
   if (cudaPointerGetAttributes(&attr, params_dev) != cudaSuccess || attr.type != cudaMemoryTypeDevice)
     return h->fail(HA_EINVAL, "bind: params is not device memory");
   h->device = attr.device;
-  cudaSetDevice(h->device);
+  DeviceScope scope(h->device);
   h->params = params_dev;
   h->ws = static_cast<uint8_t*>(workspace_dev);
   h->X = X_dev;
@@ -762,26 +814,31 @@ int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t w
 
 int hier_avg_step(hier_avg* h) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   return do_step(h);
 }
 
 int hier_avg_local_average(hier_avg* h) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   return do_local(h);
 }
 
 int hier_avg_global_average(hier_avg* h) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   return do_global(h);
 }
 
 int hier_avg_round(hier_avg* h) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   return do_round(h);
 }
 
 int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, float* loss_host) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   if (!X_host || !y_host || !loss_host) return h->fail(HA_EINVAL, "round_host: NULL host buffer");
   const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
   const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
@@ -869,7 +926,7 @@ int hier_avg_set_batch(hier_avg* h, int B) {
   if (!h || B < 1 || B > h->B) return HA_EINVAL;
   if (B < h->Bstep && h->bound && h->prec == HA_PREC_BF16) {
     // The bf16 path keeps Bn-row gradient tiles; rows from B on must add nothing to dW.
-    cudaSetDevice(h->device);
+    DeviceScope scope(h->device);
     for (int l = 1; l <= h->L; ++l)
       if (int rc = h->cuda(cudaMemsetAsync(h->ws + h->off_dZ[l], 0,
                                            static_cast<size_t>(h->P) * h->Bn * h->pitch[l] * 2,
@@ -901,6 +958,7 @@ int hier_avg_set_step(hier_avg* h, int64_t t) {
 
 int hier_avg_losses(hier_avg* h, float* loss_host) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   if (!loss_host) return HA_EINVAL;
   if (int rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost,
                                        h->stream), "losses: copy"))
@@ -910,6 +968,7 @@ int hier_avg_losses(hier_avg* h, float* loss_host) {
 
 int hier_avg_check(hier_avg* h) {
   if (int rc = check_bound(h)) return rc;
+  DeviceScope scope(h->device);
   int word = 0;
   if (int rc = h->cuda(cudaMemcpyAsync(&word, h->err_word(), 4, cudaMemcpyDeviceToHost, h->stream),
                        "check: copy"))
@@ -920,6 +979,22 @@ int hier_avg_check(hier_avg* h) {
     return h->fail(HA_ETIMEOUT, "a bounded device wait expired (error word %d)", word);
   }
   return HA_OK;
+}
+
+int hier_avg_wait_selftest(hier_avg* h, int64_t limit_us) {
+  if (int rc = check_bound(h)) return rc;
+  if (limit_us < 1 || limit_us > 10000000)
+    return h->fail(HA_EINVAL, "wait_selftest: limit %lld us is outside [1, 1e7]",
+                   (long long)limit_us);
+  DeviceScope scope(h->device);
+  int khz = 0;
+  if (int rc = h->cuda(cudaDeviceGetAttribute(&khz, cudaDevAttrClockRate, h->device),
+                       "wait_selftest: clock rate"))
+    return rc;
+  const long long cycles = static_cast<long long>(limit_us) * khz / 1000;
+  ++h->launches;
+  k_wait_selftest<<<1, 32, 0, h->stream>>>(h->never_set(), h->err_word(), cycles);
+  return h->cuda(cudaGetLastError(), "wait_selftest: launch");
 }
 
 int hier_avg_launches(const hier_avg* h, int64_t* launches) {
@@ -950,23 +1025,25 @@ int hier_avg_profile(hier_avg* h, int enable) {
 }
 
 int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* launches,
-                          double* bytes) {
+                          double* bytes, double* flops) {
   if (!h || kind < 0 || kind >= HA_KERNEL_KINDS) return HA_EINVAL;
   if (h->bound) {
     if (int rc = h->cuda(cudaStreamSynchronize(h->stream), "profile: sync")) return rc;
   }
-  double ms = 0, by = 0;
+  double ms = 0, by = 0, fl = 0;
   int64_t n = 0;
   for (const ProfRec& r : h->recs) {
     if (r.kind != kind) continue;
     float e = 0.f;
     if (cudaEventElapsedTime(&e, r.a, r.b) == cudaSuccess) ms += e;
     by += r.bytes;
+    fl += r.flops;
     ++n;
   }
   if (total_ms) *total_ms = ms;
   if (launches) *launches = n;
   if (bytes) *bytes = by;
+  if (flops) *flops = fl;
   return HA_OK;
 }
 
@@ -982,25 +1059,64 @@ int hier_avg_profile_read(hier_avg* h, int kind, double* total_ms, int64_t* laun
 namespace {
 
 constexpr int64_t kStaticScratchBytes = int64_t(32) << 20;   // 32 MiB
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-std::mutex g_scratch_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
 
-// Device address of g_static_scratch on the current device, looked up once per
-// device.  In host code the symbol's name is only a host-side stand-in.
-cudaError_t static_scratch(int device, void** out) {
-  if (device < 0 || device >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (!g_scratch_ptr[device]) {
+// Unique id of the current CUDA context (ids are never reused within a process), or
+// 0 if it cannot be read.
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
     void* p = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[device] = p;
-  }
-  *out = g_scratch_ptr[device];
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx ||
+      get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+std::mutex g_scratch_mutex;
+struct ScratchAddr {
+  unsigned long long ctx_id;
+  void* ptr;
+};
+std::vector<ScratchAddr> g_scratch_addr;   // one entry per CUDA context seen
+
+// Device address of g_static_scratch in the current context (the device must be
+// current).  In host code the symbol's name is only a host-side stand-in.  The
+// address is looked up once per context: a device reset creates a new context, in
+// which the module (and the array) is loaded again, so an address cached for the old
+// context is never reused.
+cudaError_t static_scratch(void** out) {
+  unsigned long long id = current_context_id();
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (id != 0)
+    for (const ScratchAddr& a : g_scratch_addr)
+      if (a.ctx_id == id) {
+        *out = a.ptr;
+        return cudaSuccess;
+      }
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+  if (e != cudaSuccess) return e;
+  if (id == 0) id = current_context_id();   // the lookup may have created the context
+  if (id != 0) g_scratch_addr.push_back({id, p});
+  *out = p;
   return cudaSuccess;
 }
 
@@ -1024,10 +1140,12 @@ extern "C" int hier_avg_step_static(hier_avg* h, float* params_dev, const void* 
   if (cudaPointerGetAttributes(&attr, params_dev) != cudaSuccess || attr.type != cudaMemoryTypeDevice)
     return h->fail(HA_EINVAL, "step_static: params is not device memory");
   int rc;
-  if ((rc = h->cuda(cudaSetDevice(attr.device), "step_static: set device"))) return rc;
+  DeviceScope scope(attr.device);
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess || cur != attr.device)
+    return h->fail(HA_ECUDA, "step_static: cannot make device %d current", attr.device);
   void* scratch = nullptr;
-  if ((rc = h->cuda(static_scratch(attr.device, &scratch), "step_static: scratch address")))
-    return rc;
+  if ((rc = h->cuda(static_scratch(&scratch), "step_static: scratch address"))) return rc;
   h->bound = false;
   h->device = attr.device;
   h->params = params_dev;

@@ -54,13 +54,15 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait until the phase with the given parity has completed.  Bounded.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
+// Wait until the phase with the given parity has completed.  Bounded by `limit`
+// cycles of SM clock.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err,
+                                          long long limit = kWaitLimitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (clock64() - t0 > kWaitLimitCycles) {
+    if (clock64() - t0 > limit) {
       if (err) atomicOr(err, HA_DEVERR_TIMEOUT);
       return false;
     }
@@ -93,14 +95,16 @@ __device__ __forceinline__ float4 ld_cluster_f4(const float* p, int rank) {
 __device__ __forceinline__ void red_release_add(int* p, int v) {
   asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
-// Wait, bounded, until *p == want, reading with acquire order.
-__device__ __forceinline__ bool spin_acquire_eq(const int* p, int want, int* err) {
+// Wait, bounded by `limit` cycles of SM clock, until *p == want, reading with
+// acquire order.
+__device__ __forceinline__ bool spin_acquire_eq(const int* p, int want, int* err,
+                                                long long limit = kWaitLimitCycles) {
   const long long t0 = clock64();
   while (true) {
     int v;
     asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     if (v == want) return true;
-    if (clock64() - t0 > kWaitLimitCycles) {
+    if (clock64() - t0 > limit) {
       if (err) atomicOr(err, HA_DEVERR_TIMEOUT);
       return false;
     }

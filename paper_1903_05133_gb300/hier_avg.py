@@ -8,7 +8,7 @@ function and method names are those of include/hier_avg.h without the
 from __future__ import annotations
 
 import ctypes
-from typing import List, Optional, Sequence, Tuple
+from typing import List, NamedTuple, Optional, Sequence, Tuple
 
 import torch
 
@@ -18,6 +18,13 @@ from ._lib import c_double, c_int, c_int64, c_void_p, check
 PREC = {"fp32": 0, "bf16": 1}
 KERNEL_KINDS = {"gather": 0, "forward": 1, "xent": 2, "backward": 3, "local_avg": 4,
                 "global_avg": 5, "head": 6, "update_forward": 7}
+
+
+class ProfileTotals(NamedTuple):
+    total_ms: float
+    launches: int
+    bytes: float
+    flops: float
 
 
 def _stream(stream) -> c_void_p:
@@ -171,6 +178,12 @@ class HierAvg:
     def check(self) -> None:
         check(self._lib.hier_avg_check(self.h), "check", self.h)
 
+    def wait_selftest(self, limit_ms: float) -> None:
+        """Run the library's bounded device waits on conditions nothing satisfies, each
+        limited to limit_ms; the next check() raises HA_ETIMEOUT (see the header)."""
+        check(self._lib.hier_avg_wait_selftest(self.h, int(round(limit_ms * 1000))),
+              "wait_selftest", self.h)
+
     def profile(self, enable) -> None:
         """Start (and clear) kernel timing: True for every kind, an iterable of kind
         names for a subset; False stops it."""
@@ -205,12 +218,13 @@ class HierAvg:
         """Time only every n-th launch of each enabled kind."""
         check(self._lib.hier_avg_profile_every(self.h, int(every)), "profile_every", self.h)
 
-    def profile_read(self, kind: str) -> Tuple[float, int, float]:
-        ms, n, by = c_double(), c_int64(), c_double()
+    def profile_read(self, kind: str) -> "ProfileTotals":
+        """(total_ms, launches, bytes, flops) of the timed launches of one kernel kind."""
+        ms, n, by, fl = c_double(), c_int64(), c_double(), c_double()
         check(self._lib.hier_avg_profile_read(self.h, KERNEL_KINDS[kind], ctypes.byref(ms),
-                                              ctypes.byref(n), ctypes.byref(by)),
+                                              ctypes.byref(n), ctypes.byref(by), ctypes.byref(fl)),
               "profile_read", self.h)
-        return ms.value, n.value, by.value
+        return ProfileTotals(ms.value, n.value, by.value, fl.value)
 
     def destroy(self) -> None:
         if self.h:

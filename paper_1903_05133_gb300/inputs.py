@@ -16,7 +16,7 @@ Learner j draws from its own generator seeded with ``seed * 1000003 + j``.
 """
 from __future__ import annotations
 
-from typing import List, Tuple
+from typing import List, Sequence, Tuple
 
 import torch
 
@@ -36,21 +36,24 @@ def class_means(w: Workload, device="cpu") -> torch.Tensor:
     return mu * w.sigma_mu
 
 
-def learner_data(w: Workload, device="cpu", N: int | None = None
-                 ) -> Tuple[torch.Tensor, torch.Tensor]:
-    """Per-learner datasets: X [P, N, d_0] (bf16, or fp32 for fp32 workloads), y [P, N] int32."""
+def learner_data(w: Workload, device="cpu", N: int | None = None,
+                 learners: Sequence[int] | None = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """Per-learner datasets: X [P, N, d_0] (bf16, or fp32 for fp32 workloads), y [P, N] int32.
+    With ``learners``, only those learners' data sets (the same bytes), stacked in
+    that order."""
     N = w.N if N is None else N
+    ids = list(range(w.P)) if learners is None else list(learners)
     dtype = torch.float32 if w.precision == "fp32" else torch.bfloat16
     mu = class_means(w, device)
-    X = torch.empty(w.P, N, w.dims[0], dtype=dtype, device=device)
-    y = torch.empty(w.P, N, dtype=torch.int32, device=device)
-    for j in range(w.P):
+    X = torch.empty(len(ids), N, w.dims[0], dtype=dtype, device=device)
+    y = torch.empty(len(ids), N, dtype=torch.int32, device=device)
+    for i, j in enumerate(ids):
         g = _gen(w.seed * 1000003 + j, device)
         yj = torch.randint(0, w.classes, (N,), generator=g, device=device, dtype=torch.int64)
         xj = torch.randn(N, w.dims[0], generator=g, device=device, dtype=torch.float32)
         xj += mu[yj]
-        X[j].copy_(xj)
-        y[j].copy_(yj.to(torch.int32))
+        X[i].copy_(xj)
+        y[i].copy_(yj.to(torch.int32))
     return X, y
 
 

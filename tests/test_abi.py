@@ -80,6 +80,7 @@ def test_calls_before_bind_fail_cleanly(lib):
     assert lib.hier_avg_step(h) == -4
     assert lib.hier_avg_round(h) == -4
     assert lib.hier_avg_local_average(h) == -4
+    assert lib.hier_avg_wait_selftest(h, 1000) == -4
     assert b"bind" in lib.hier_avg_last_error(h)
     assert lib.hier_avg_bind(h, None, None, 0, None, None, 1, None) == -1
     assert lib.hier_avg_set_step(h, 5) == 0
@@ -91,7 +92,7 @@ def test_calls_before_bind_fail_cleanly(lib):
     assert lib.hier_avg_profile_kinds(h, 1 << 8) == -1          # no such kernel kind
     assert lib.hier_avg_profile_kinds(h, 1 << 7) == 0
     assert lib.hier_avg_profile_kinds(h, (1 << 1) | (1 << 3)) == 0
-    assert lib.hier_avg_profile_read(h, 99, None, None, None) == -1
+    assert lib.hier_avg_profile_read(h, 99, None, None, None, None) == -1
     assert lib.hier_avg_set_global_steps(h, -1) == -1
     assert lib.hier_avg_set_global_steps(h, 43) == 0 and lib.hier_avg_set_global_steps(h, 0) == 0
     assert lib.hier_avg_set_global_steps(None, 5) == -1
@@ -114,6 +115,10 @@ def test_stateless_averages_validate(lib):
     assert lib.hier_avg_global_average_buffer(None, 0, 10, 10, None) == -1
     assert lib.hier_avg_local_global_average_buffer(None, 4, 2, 10, 10, None) == -1   # NULL
     assert lib.hier_avg_local_average_buffer(None, 4, 2, 0, 0, None) == 0        # empty: no-op
+    # more than 65535 clusters in one launch is rejected before any launch
+    assert lib.hier_avg_local_average_buffer(None, 2 * 65536, 2, 0, 0, None) == -6
+    assert lib.hier_avg_global_average_buffer(None, 2 * 65536, 0, 0, None) == 0
+    assert lib.hier_avg_local_global_average_buffer(None, 2 * 65536, 2, 0, 0, None) == 0
 
 
 def test_status_strings(lib):

@@ -25,9 +25,14 @@ def test_reference_arm_prints_one_json_line():
     assert line["value"] > 0 and line["higher_is_better"] is True
     assert line["steps"] == 2 and line["warmup"] == 1
     assert line["config"]["workload"].startswith("softmax")
+    # the same config dict as the GPU arm's line, so the two arms compare one workload
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_1903_05133_gb300 import configs
+    assert line["config"] == json.loads(json.dumps(bench.run_config(configs.SHORT["softmax"], 1)))
     cb = line["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"]
-    assert cb["unit"] == line["unit"] and cb["sample"]
+    assert cb["unit"] == line["unit"] and cb["sample"].startswith("extrapolated")
     e2e = line["e2e"]
     assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
