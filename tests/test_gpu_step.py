@@ -2,16 +2,22 @@
 the CUDA path, called through the C ABI, against the oracle on the same seeded
 inputs.  Errors are normwise per parameter tensor, max|gpu - oracle| / max|oracle|.
 
-Tolerances.  fp32 path: 1e-5.  bf16-operand path: 1e-2 for the parameters after a
-step, against an oracle that rounds the same operands to bf16.  A bf16 rounding or
-ReLU decision taken on a value within rounding distance of its threshold can go
-either way under two valid fp32 accumulation orders, and such flips propagate
-through the layers (a 1-ulp bf16 flip in H_l moves Z_{l+1} by ~1e-4 relative,
-which flips more decisions there).  The spread this causes is measured, not
-guessed: the oracle is run a second time with fp32 accumulation ("bf16_acc32"),
-and the GPU must be within max(tolerance, SPREAD * that oracle-vs-oracle error).
-The update w_new - w_old itself is checked the same way (2e-2 floor), in the max
-norm and in the Frobenius norm."""
+Per step (one step from a shared state, and every step of a teacher-forced round):
+the parameters after the step within 1e-5 (fp32 path) or 1e-2 (bf16-operand path,
+against an oracle that rounds the same operands to bf16), asserted outright.
+
+The update w_new - w_old of a bf16 step is also checked (2e-2, max and Frobenius
+norms).  A ReLU decision on a pre-activation within rounding distance of zero can go
+either way under two valid fp32 accumulation orders, which swaps one sample's term
+in one row of the update; so an update row beyond the bound is accepted only where
+such a flip is provable (the oracle's pre-activation in that row is below the
+worst-case difference of two fp32 summation orders), and every accepted row is
+counted and reported (none at the 16-learner workload, at most one row in a
+thousand at the full-size workloads).
+
+Whole rounds end to end (no teacher forcing): such flips compound over the round's
+steps, so the bound there is max(tolerance, SPREAD x the error between two valid
+oracles: bf16 operands with exact products, and with fp32 accumulation)."""
 import numpy as np
 import pytest
 import torch
@@ -81,63 +87,95 @@ def make_oracle(w, ha, X, y, params, learners=None, mode=None):
     return o
 
 
-# A ReLU decision on a pre-activation within rounding distance of zero can go
-# either way even when both sides accumulate to ~1e-7; it swaps one sample's term
-# in one row of that layer's update.  Rows beyond the limit are accepted only if
-# the oracle's own pre-activation in that row is near zero, and only a few.
-NEAR_ZERO = 1e-3          # |z| <= NEAR_ZERO * max|z| of the layer
-MAX_FLIP_ROWS = 0.01      # at most this fraction of rows (and at least 3)
+# A ReLU decision on a pre-activation within rounding distance of zero can go either
+# way in two correct implementations; it swaps one sample's term in one row of that
+# layer's update.  Two fp32 sums of the same K products in different orders differ by
+# at most 2 K u sum_k |h_k w_k| (u = 2^-24), so such a flip is possible only where the
+# exact pre-activation is smaller than that.  An update row beyond its bound is
+# accepted only if some sample's pre-activation in that row is (the "flip ratio"
+# |z| / (2 K u sum |h w|) is at most 1), and every accepted row is counted.
+U32 = 2.0 ** -24
 
 
-def _explained(o, k, L, bad):
-    """Rows flagged `bad` ([learners, out]) of tensor k explained by near-zero
-    pre-activations of the layer that tensor feeds."""
+def _flip_rows(o, k, L, bad, before):
+    """Rows flagged `bad` ([learners, out]) of tensor k that a provable ReLU flip
+    explains, as (count, flip ratios), or (0, ratios) if any row is not explained."""
     layer = k // 2
-    if layer >= L - 1 or not getattr(o.problem, "last_preacts", None):
-        return False
-    near = np.array([np.any(np.abs(o.problem.last_preacts[jj][layer]) <=
-                            NEAR_ZERO * np.max(np.abs(o.problem.last_preacts[jj][layer])), axis=0)
-                     for jj in range(bad.shape[0])])
-    return bool(np.all(near[bad])) and bad.sum() <= max(3, MAX_FLIP_ROWS * bad.size)
+    if layer >= L - 1 or before is None or not getattr(o.problem, "last_preacts", None):
+        return 0, []
+    X = o.problem.X
+    rows = oracle.batch_rows_from(o.cursor - o.B, o.B, X.shape[1])
+    n, ratios = 0, []
+    for jj in range(bad.shape[0]):
+        flagged = np.nonzero(bad[jj])[0]
+        if len(flagged) == 0:
+            continue
+        pre = o.problem.last_preacts[jj]
+        z = pre[layer]                                        # [B, out], the oracle's Z_l
+        if layer == 0:
+            H = oracle.bf16_round(X[jj, rows].astype(np.float32)).astype(np.float64)
+        else:
+            H = oracle.bf16_round(np.maximum(pre[layer - 1], 0).astype(np.float32)).astype(np.float64)
+        W = oracle.bf16_round(before[2 * layer][jj].astype(np.float32)).astype(np.float64)
+        K = W.shape[1]
+        for r in flagged:
+            bound = 2.0 * K * U32 * (np.abs(H) @ np.abs(W[r])) + 1e-300
+            ratio = float(np.min(np.abs(z[:, r]) / bound))
+            ratios.append(ratio)
+            if ratio > 1.0:
+                return 0, ratios
+            n += 1
+    return n, ratios
 
 
-def _check(name, k, g, want, ref, lim_floor, fn, o, L, report):
+def _check(name, k, g, want, lim, fn, o, L, report, stats, before=None):
     e = fn(g, want)
-    lim = max(lim_floor, SPREAD * fn(ref, want)) if ref is not None else lim_floor
     if report is not None:
         report.append((k, name, e, lim))
     if e <= lim:
         return e
-    if fn is rel_err:
+    if before is not None and fn is rel_err:
         scale = np.max(np.abs(want))
         rows = np.max(np.abs(g - want).reshape(g.shape[0], g.shape[1], -1), axis=2) / scale
-        if _explained(o, k, L, rows > lim):
+        n, ratios = _flip_rows(o, k, L, rows > lim, before)
+        if n:
+            if stats is not None:
+                stats["exempt_rows"] = stats.get("exempt_rows", 0) + n
+                stats.setdefault("exempt", []).append((k, name, round(e, 5), lim, n,
+                                                       [round(x, 4) for x in ratios]))
             return e
+        raise AssertionError(f"tensor {k}: {name} err {e:.3e} > {lim:.3e}; flip ratios {ratios}")
     raise AssertionError(f"tensor {k}: {name} err {e:.3e} > {lim:.3e}")
 
 
-def compare(ha, o, learners=None, tol=None, before=None, o_ref=None, report=None):
+def compare(ha, o, learners=None, tol=None, before=None, o_ref=None, report=None,
+            end_to_end=False, stats=None):
     """Check the GPU parameters against oracle `o` (and, with `before`, the update
-    itself).  With a second-order oracle `o_ref`, bf16 tolerances widen to SPREAD
-    times the oracle-vs-oracle error; rows beyond that must be explained by
-    near-zero ReLU inputs."""
+    itself).  Per step the parameter bound is `tol` outright.  End to end
+    (`end_to_end`, with a second oracle `o_ref`), the bound widens to SPREAD times
+    the oracle-vs-oracle error.  Update rows beyond their bound must be explained by
+    near-zero ReLU inputs; `stats` counts them."""
     tol = TOL[ha.precision] if tol is None else tol
     utol = UPDATE_TOL[ha.precision]
     learners = list(range(ha.P)) if learners is None else learners
     got = oracle_params(ha, ha.params, learners)
     worst = 0.0
+    if stats is not None:
+        stats.setdefault("exempt_rows", 0)
     for k, (g, want) in enumerate(zip(got, o.params)):
         g, want = g.astype(np.float64), want.astype(np.float64)
         ref = o_ref.params[k].astype(np.float64) if o_ref is not None else None
-        worst = max(worst, _check("param", k, g, want, ref, tol, rel_err, o, ha.L, report))
+        lim = tol
+        if end_to_end and ref is not None:
+            lim = max(tol, SPREAD * rel_err(ref, want))
+        worst = max(worst, _check("param", k, g, want, lim, rel_err, o, ha.L, report, stats))
         if before is None:
             continue
         b0 = before[k]
         if np.max(np.abs(want - b0)) == 0:
             continue
-        rb = ref - b0 if ref is not None else None
         for name, fn in (("update-max", rel_err), ("update-frob", frob_err)):
-            _check(name, k, g - b0, want - b0, rb, utol, fn, o, ha.L, report)
+            _check(name, k, g - b0, want - b0, utol, fn, o, ha.L, report, stats, before=before)
     return worst
 
 
@@ -184,13 +222,14 @@ def test_one_step_from_distinct_learners(w):
     ha, X, y = setup(w, layers)
     start = oracle_params(ha, ha.params)
     o = make_oracle(w, ha, X, y, start)
-    o_ref = make_oracle(w, ha, X, y, start, mode="bf16_acc32") if w.precision == "bf16" else None
     ha.step()
     ha.check()
     o.step()
-    if o_ref is not None:
-        o_ref.step()
-    compare(ha, o, before=[a.astype(np.float64) for a in start], o_ref=o_ref)
+    stats = {}
+    compare(ha, o, before=[a.astype(np.float64) for a in start], stats=stats)
+    print(w.name, "exempt update rows:", stats["exempt_rows"], stats.get("exempt", []))
+    if w is configs.MLP512_P16:
+        assert stats["exempt_rows"] == 0
     gl = ha.losses().numpy()
     assert np.allclose(gl, o.problem.last_loss, rtol=1e-3, atol=1e-4)
 
@@ -209,7 +248,9 @@ def test_full_run_against_oracle(w):
         if o_ref is not None:
             o_ref.round()
     ha.check()
-    compare(ha, o, o_ref=o_ref)
+    report = []
+    compare(ha, o, o_ref=o_ref, end_to_end=True, report=report)
+    print(w.name, "end to end (err, bound):", [(k, f"{e:.2e}", f"{lim:.2e}") for k, _, e, lim in report])
     # every learner holds the same parameters after the global average
     p = ha.params.cpu().numpy().view(np.uint32)
     assert np.all(p == p[0])
@@ -261,8 +302,8 @@ def test_fused_next_forward_equals_steps(w):
     n0 = ha1.launches()
     ha1.round()
     n_round = ha1.launches() - n0
-    _, n_fused, _ = ha1.profile_read("update_forward")
-    _, n_fwd, _ = ha1.profile_read("forward")
+    n_fused = ha1.profile_read("update_forward").launches
+    n_fwd = ha1.profile_read("forward").launches
     ha1.profile(False)
     steps, L = w.K1 * w.K2, len(w.dims) - 1
     assert n_fused == _fused_steps(w) > 0
@@ -309,7 +350,7 @@ def test_free_global_interval_against_oracle(w, G):
                 oo.round()
         ha.round()
     ha.check()
-    compare(ha, o, o_ref=o_ref)
+    compare(ha, o, o_ref=o_ref, end_to_end=True)
     p = ha.params.cpu().numpy().view(np.uint32)
     assert np.all(p == p[0])                      # the round ends with the global average
     assert ha.get_step() == 2 * G
@@ -357,7 +398,7 @@ def test_batch_schedule_against_oracle(w, sched):
                 oo.round()
         ha.round()
     ha.check()
-    compare(ha, o, o_ref=o_ref)
+    compare(ha, o, o_ref=o_ref, end_to_end=True)
     gl = ha.losses().numpy()
     assert np.allclose(gl, o.problem.last_loss, rtol=2e-3, atol=1e-4)
 
@@ -395,15 +436,14 @@ def test_round_teacher_forced(w):
     # (1e-2, and the update itself within 2e-2), every average bit-exact.
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
-    o_ref = make_oracle(w, ha, X, y, oracle_params(ha, ha.params), mode="bf16_acc32")
     worst = 0.0
+    stats = {}
     for b in range(w.K2):
         for k in range(w.K1):
-            before = _force(ha, o, o_ref)
+            before = _force(ha, o)
             ha.step()
             o.step()
-            o_ref.step()
-            worst = max(worst, compare(ha, o, before=before, o_ref=o_ref))
+            worst = max(worst, compare(ha, o, before=before, stats=stats))
         _force(ha, o)
         if b + 1 < w.K2:
             ha.local_average()
@@ -417,7 +457,8 @@ def test_round_teacher_forced(w):
         for g, want in zip(got, o.params):
             assert np.array_equal(g.view(np.uint32), want.view(np.uint32))
     ha.check()
-    print(f"{w.name}: worst per-step rel err {worst:.3e}")
+    print(f"{w.name}: worst per-step rel err {worst:.3e}; exempt update rows "
+          f"{stats['exempt_rows']} {stats.get('exempt', [])}")
 
 
 def test_mlp512_round_end_to_end():
@@ -432,7 +473,7 @@ def test_mlp512_round_end_to_end():
     o_ref.round()
     ha.check()
     report = []
-    compare(ha, o, o_ref=o_ref, report=report)
+    compare(ha, o, o_ref=o_ref, end_to_end=True, report=report)
     print(w.name, "end-to-end:", [(k, f"{e:.2e}", f"{lim:.2e}") for k, _, e, lim in report])
 
 
@@ -445,15 +486,18 @@ def test_full_size_step_sampled(w):
     learners = [0, w.P - 1]
     start = oracle_params(ha, ha.params, learners)
     o = make_oracle(w, ha, X, y, start, learners)
-    o_ref = make_oracle(w, ha, X, y, start, learners, mode="bf16_acc32")
     ha.step()
     ha.check()
     o.step()
-    o_ref.step()
-    report = []
-    compare(ha, o, learners, before=[a.astype(np.float64) for a in start], o_ref=o_ref,
-            report=report)
+    report, stats = [], {}
+    compare(ha, o, learners, before=[a.astype(np.float64) for a in start], report=report,
+            stats=stats)
     print(w.name, [(k, kind, f"{e:.2e}", f"{lim:.2e}") for k, kind, e, lim in report])
+    # parameters within 1e-2 outright; update rows beyond 2e-2 only where a ReLU flip is
+    # provable, at most one row in a thousand
+    print(w.name, "exempt update rows:", stats["exempt_rows"], stats.get("exempt", []))
+    rows = sum(ha.dims[1:-1]) * len(learners)
+    assert stats["exempt_rows"] <= rows // 1000, stats.get("exempt")
 
 
 # SMALL_BF16: the rows are copied step by step beside the kernels (two layers, cluster
