@@ -23,7 +23,8 @@ using ha::TcBwdArgs;
 using ha::TcFwdArgs;
 
 constexpr int64_t kAlign = 1024;
-constexpr int64_t kTargetCtas = 152;   // persistent forward: one CTA per SM of a GB300
+constexpr int64_t kTargetCtas = 152;   // persistent kernels: one CTA per SM of a GB300
+constexpr int64_t kPieceChunks = 48;   // chunks per piece of a split tile (forward, backward)
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -69,8 +70,10 @@ struct hier_avg {
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
   int64_t off_dyn = 0;                        // update kernel's work-item counters
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
-  std::vector<int> fwd_cq;                    // per layer: cluster split factor (1 = stream-K)
-  std::vector<int> bwd_ctas, bwd_tiles;       // per layer: stream-K CTAs, input slices
+  std::vector<int> fwd_cq;                    // per layer: cluster split factor (1 = dynamic)
+  std::vector<int> fwd_whole, fwd_np;         // per layer (dynamic): whole tiles, tail pieces
+  std::vector<int> bwd_ctas, bwd_tiles;       // per layer: CTAs, input slices of 128
+  std::vector<int> bwd_whole, bwd_np;         // per layer: whole tiles, tail pieces
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
   bool w_stream = true;                       // parameters exceed L2: stream W evict-first
   bool head = false;                          // d_L <= 16: fused last-layer kernel
@@ -196,13 +199,16 @@ int plan_layout(hier_avg* h) {
     h->fwd_ctas.assign(L, 1);
     h->fwd_tiles.assign(L, 1);
     h->fwd_cq.assign(L, 1);
+    h->fwd_whole.assign(L, 0);
+    h->fwd_np.assign(L, 1);
     h->bwd_ctas.assign(L, 1);
     h->bwd_tiles.assign(L, 1);
+    h->bwd_whole.assign(L, 0);
+    h->bwd_np.assign(L, 1);
     int64_t part_bytes = 16, max_tiles = 1;
     for (int l = 0; l < L; ++l) {
       const int64_t in = h->dims[l], out = h->dims[l + 1];
       const int64_t ftiles = (out + 127) / 128, btiles = (in + 127) / 128;
-      h->fwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, ftiles * P * ((in + 63) / 64)));
       h->fwd_tiles[l] = static_cast<int>(ftiles);
       // Few tiles: a cluster of cq CTAs per tile, reduced through distributed shared
       // memory (the stream-K fix-up through global memory costs a few microseconds of
@@ -212,10 +218,36 @@ int plan_layout(hier_avg* h) {
       if (cq >= 2) {
         h->fwd_cq[l] = static_cast<int>(cq);
         h->fwd_ctas[l] = static_cast<int>(ftiles * P * cq);
+      } else {
+        // Dynamic items.  First layer: the last tiles, one per SM, are split into pieces
+        // of kPieceChunks chunks, so that the work left when the whole tiles run out is
+        // fine grained (the update+forward kernel, which streams W_1 twice as long as a
+        // forward, gains most).  The split depends on the shapes only, so the forward
+        // and the update+forward sum every H_1 entry the same way.  Later layers keep
+        // whole tiles: there a piece's partial round trip costs more than the balance
+        // gains (measured).
+        const int64_t t_tail = l == 0 ? std::min<int64_t>(ftiles * P, kTargetCtas) : 0;
+        const int64_t np = (nk + kPieceChunks - 1) / kPieceChunks;
+        h->fwd_whole[l] = static_cast<int>(ftiles * P - t_tail);
+        h->fwd_np[l] = static_cast<int>(np);
+        const int64_t items = (ftiles * P - t_tail) + t_tail * np;
+        h->fwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, items));
+        if (np > 1) part_bytes = std::max(part_bytes, t_tail * np * 128 * h->Bn * 4);
       }
-      h->bwd_ctas[l] = static_cast<int>(std::min<int64_t>(kTargetCtas, btiles * P * ((out + 63) / 64)));
+      {
+        // Backward with dX (every layer but the first; the first runs the update-only
+        // kernel): dynamic items, the last tiles (one per SM) split into pieces whose dX
+        // partials are added in piece order.
+        const int64_t nc = (out + 63) / 64;
+        const int64_t t_tail = std::min<int64_t>(btiles * P, kTargetCtas);
+        const int64_t np = (nc + kPieceChunks - 1) / kPieceChunks;
+        h->bwd_whole[l] = static_cast<int>(btiles * P - t_tail);
+        h->bwd_np[l] = static_cast<int>(np);
+        h->bwd_ctas[l] = static_cast<int>(
+            std::min<int64_t>(kTargetCtas, (btiles * P - t_tail) + t_tail * np));
+        if (l > 0 && np > 1) part_bytes = std::max(part_bytes, t_tail * np * 128 * h->Bn * 4);
+      }
       h->bwd_tiles[l] = static_cast<int>(btiles);
-      part_bytes = std::max(part_bytes, int64_t(std::max(h->fwd_ctas[l], h->bwd_ctas[l])) * 128 * h->Bn * 4);
       max_tiles = std::max(max_tiles, std::max(ftiles, btiles) * P);
     }
     h->fused_xent = h->dims[L] <= 128;
@@ -418,8 +450,12 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.cq = h->fwd_cq[l];
       a.o_tiles = h->fwd_tiles[l];
       a.n_tiles = h->fwd_tiles[l] * P;
+      a.n_whole = h->fwd_whole[l];
+      a.np_tail = h->fwd_np[l];
+      a.piece_chunks = static_cast<int>(kPieceChunks);
       a.part = h->wsp<float>(h->off_part);
       a.counters = h->wsp<int>(h->off_cnt);
+      a.dyn = h->wsp<int>(h->off_dyn);
       a.x_direct = (l == 0 && x_direct) ? 1 : 0;
       a.w_stream = h->w_stream ? 1 : 0;
       a.share = shared ? h->S : 1;
@@ -485,6 +521,10 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.ctas = h->bwd_ctas[l];
       a.s_tiles = h->bwd_tiles[l];
       a.n_tiles = h->bwd_tiles[l] * P;
+      a.n_whole = h->bwd_whole[l];
+      a.np_tail = h->bwd_np[l];
+      a.piece_chunks = static_cast<int>(kPieceChunks);
+      a.dyn = h->wsp<int>(h->off_dyn);
       a.part = h->wsp<float>(h->off_part);
       a.counters = h->wsp<int>(h->off_cnt);
       a.err = h->err_word();
@@ -507,8 +547,13 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.cq = h->fwd_cq[0];
         f.o_tiles = h->fwd_tiles[0];
         f.n_tiles = h->fwd_tiles[0] * P;
+        f.n_whole = h->fwd_whole[0];
+        f.np_tail = h->fwd_np[0];
+        f.piece_chunks = static_cast<int>(kPieceChunks);
         f.part = h->wsp<float>(h->off_part);
         f.counters = h->wsp<int>(h->off_cnt);
+        f.dyn = h->wsp<int>(h->off_dyn);
+        f.share = 1;
         f.x_direct = 1;
         f.x_row0 = static_cast<int>(r1);
         f.hc_row0 = a.h_row0;
@@ -524,17 +569,14 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         if (fused) *fused = true;
         continue;
       }
-      // The first layer's backward (no dX) hands its independent units out dynamically
-      // when there are many of them per SM (work items of 8 chunks); a short layer keeps
-      // the even static split, which work items that coarse would unbalance.
-      const int64_t units = int64_t(a.n_tiles) * ((a.out + 63) / 64);
-      if (a.has_dx || units < int64_t(kTargetCtas) * 64) {
+      // The first layer's backward (no dX) runs the update-only kernel: independent
+      // runs of 8 chunks, claimed dynamically (measured faster than the backward
+      // kernel's items for short layers too: 3072-512-10 round 0.859 -> 0.850 ms).
+      if (a.has_dx) {
         rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
           return ha::launch_tc_backward(h->tm_wb[l], hin, h->tm_dz[l + 1], a, P, s);
         }, "backward");
       } else {
-        // no dX: independent units, handed out dynamically
-        a.dyn = h->wsp<int>(h->off_dyn);
         a.ctas = kTargetCtas;
         rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
           return ha::launch_tc_update(h->tm_wb[l], hin, h->tm_dz[l + 1], a, s);

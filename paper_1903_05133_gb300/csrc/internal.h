@@ -85,15 +85,20 @@ struct TcFwdArgs {
   __nv_bfloat16* h_out;       // mode 0: H_{l+1} [P][Bn][pitch_out]
   int pitch_out;              // mode 0: H pitch; mode 2: dZ_L pitch
   float* z_out;               // mode 1: Z_L [P][B][out]
-  // persistent stream-K schedule: `ctas` CTAs share the n_tiles x ceil(in/64) units
-  // (tile = learner x 128 outputs) evenly.  A split tile is finished by the CTA that
-  // holds its first chunk; each other contributor writes its partial to its slot of
-  // part [ctas][128][Bn] and bumps counters[tile] (reset to 0 by the finisher), and
-  // the finisher adds the partials in CTA order.
+  // Schedule over n_tiles = P x o_tiles tiles (learner x 128 outputs), each reduced over
+  // ceil(in/64) chunks.  cq > 1: cluster split-K, ctas = n_tiles * cq.  Otherwise
+  // dynamic: `ctas` CTAs claim work items from dyn[0] (dyn[1] counts the CTAs done;
+  // both zero on entry, reset on exit).  Tiles [0, n_whole) are one item each; tiles
+  // [n_whole, n_tiles) are split into np_tail pieces of piece_chunks chunks.  Piece p
+  // of tail tile tt = tau - n_whole writes its partial to part[((tt * np_tail + p) *
+  // 128 + row) * Bn + col] and counts itself in counters[tt]; the last one adds the
+  // tile's partials in piece order, runs the epilogue and resets counters[tt] to 0.
   int ctas, n_tiles, o_tiles;
-  int cq;                     // > 1: cluster split-K, ctas = n_tiles * cq (no part/counters)
+  int cq;
+  int n_whole, np_tail, piece_chunks;
   float* part;
   int* counters;
+  int* dyn;
   // first layer: the batch tile is read straight from X (rows x_row0 .. of learner j)
   int x_direct, x_row0;
   int hc_row0;                // update+forward: rows of this step's batch in its map
@@ -118,12 +123,16 @@ struct TcBwdArgs {
   int pitch_in;
   int h_row0;                 // first batch row of H_{l-1} in its tensor map (X rows for l = 0)
   int w_stream;               // load and store W with the L2 evict-first policy
-  // persistent stream-K schedule over n_tiles = P x ceil(in/128) tiles x ceil(out/64)
-  // chunks, same partial/counter protocol as the forward
+  // n_tiles = P x s_tiles tiles (learner x 128 inputs) of ceil(out/64) chunks each,
+  // claimed dynamically by `ctas` CTAs from dyn[0] (dyn[1] counts the CTAs done; both
+  // zero on entry, reset on exit).  k_tc_backward: tiles [0, n_whole) whole, tiles
+  // [n_whole, n_tiles) in np_tail pieces of piece_chunks chunks, dX partials and
+  // counters as the forward's.  k_tc_update: runs of up to 8 chunks.
   int ctas, n_tiles, s_tiles;
+  int n_whole, np_tail, piece_chunks;
   float* part;
   int* counters;
-  int* dyn;                   // update-only kernel: [0] work items claimed, [1] CTAs done
+  int* dyn;
   int* err;
 };
 int tc_fwd_smem_bytes();

@@ -95,6 +95,13 @@ __device__ __forceinline__ float4 ld_cluster_f4(const float* p, int rank) {
 __device__ __forceinline__ void red_release_add(int* p, int v) {
   asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
+// GPU-scope acquire-release fence: with a CTA barrier before it, it orders every write
+// the CTA's threads made before the barrier ahead of this thread's next (relaxed)
+// atomic, for any thread that observes that atomic and then fences.
+__device__ __forceinline__ void fence_acq_rel_gpu() {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+
 // Wait, bounded by `limit` cycles of SM clock, until *p == want, reading with
 // acquire order.
 __device__ __forceinline__ bool spin_acquire_eq(const int* p, int want, int* err,

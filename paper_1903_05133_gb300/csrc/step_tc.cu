@@ -30,33 +30,45 @@ namespace {
 
 
 // ------------------------------------------------------------------ forward
-// Persistent stream-K forward.  The work of one layer is a list of units
-// u = (tile, chunk): tile = (learner j, 128 output features), chunk = 64 input
-// features.  CTA g of G owns the contiguous units [g*U/G, (g+1)*U/G), so every SM
-// streams the same number of chunks and the TMA ring runs straight across tile
-// boundaries.  A tile whose chunks are spread over several CTAs is finished by
-// the CTA that holds its first chunk (see tile_end) with the partials of the
-// others added in CTA order (deterministic).
-// Small layers (at most 76 tiles, so at least two CTAs per tile) run in cluster
-// split-K mode instead: tile t gets a cluster of cq CTAs, rank k taking chunks
-// [k*nk/cq, (k+1)*nk/cq); at the end ranks 1.. leave their partial in shared
-// memory and rank 0 adds them in rank order through distributed shared memory and
-// runs the epilogue.  No global partials, no waiting on other clusters.
+// Forward of one layer on the tensor cores.  The work is a list of tiles: tile =
+// (learner j, 128 output features), reduced over the layer's input in chunks of 64
+// features.  Two schedules:
+//  * Dynamic (layers with many tiles).  Work items are handed out from a global
+//    counter, so an SM that streams its weights faster simply takes more of them
+//    (per-SM streaming rates differ by up to 1.8x under full load, and a static split
+//    waits for the slowest SM).  Most tiles are one item each.  The tiles of the
+//    last clusters of learners (the "tail": at least one tile per SM) are split into
+//    fixed pieces of kPieceChunks chunks, so that the work left at the end is fine
+//    grained.  Which tiles are split and where depends on the layer's shape only.
+//    Each piece writes its partial sum to a slot of its own; the piece that
+//    completes a tile (an atomic count per tile) adds the tile's partials in piece
+//    order and runs the epilogue.  The sum of every output therefore has one fixed
+//    order, whichever CTA computed which piece.  No CTA waits for another.
+//  * Cluster split-K (layers with at most 76 tiles): tile t gets a cluster of cq
+//    CTAs, rank k taking chunks [k*nk/cq, (k+1)*nk/cq); at the end ranks 1.. leave
+//    their partial in shared memory and rank 0 adds them in rank order through
+//    distributed shared memory and runs the epilogue.
 // Warps 0-7 convert the fp32 weight tiles to bf16 and own the accumulator rows:
 // warp w serves TMEM lanes 32*(w%4).., converts K half w/4 of those 32 rows, and
 // the two warps on the same lanes split the batch columns in interleaved 16-column
-// blocks (group w/4 takes blocks 2m + w/4).  Warp 8 streams the weight tiles,
-// warp 9 issues the MMAs, warp 10 streams the batch tiles and publishes this CTA's
-// split-tile partial.  Every role that waits has a warp of its own: a lane blocked
-// in an mbarrier wait would hold up the other lanes of its warp.
+// blocks (group w/4 takes blocks 2m + w/4).  Warp 8 claims the work items and
+// streams the weight tiles, warp 9 issues the MMAs, warp 10 streams the batch tiles.
+// Every role that waits has a warp of its own: a lane blocked in an mbarrier wait
+// would hold up the other lanes of its warp.  Warp 8 announces each claimed item to
+// the other roles through a small queue in shared memory.
 // The bf16 A tile (128 rows x 64 K) lives in tensor memory, double-buffered, so
 // shared memory holds only the two TMA rings: the fp32 weight tiles (two
 // 128-byte-swizzled 128 x 32 boxes per chunk, released by the converter warps as
 // soon as they have read them, so conversion and MMA latency stay out of the
 // weight stream) and the bf16 batch tiles (Bn x 128 bytes, released by the MMA),
 // plus (fused cross-entropy only) a staging area for the epilogue.  A chunk takes
-// about 4 us from TMA issue to arrival under full load, so both rings are as deep
+// about 4-5 us from TMA issue to arrival under full load, so both rings are as deep
 // as shared memory allows.
+// Right after a local average (TcFwdArgs::share > 1) the members of a cluster hold
+// identical weights and all read the first member's copy.  (Ordering the items so
+// that the members' items for one weight tile are claimed together measured no
+// faster: the CTAs sharing a tile drift apart over its chunks by more than the time
+// the tile stays in L2.)
 constexpr int kFwdConv = 256;
 constexpr int kFwdThreads = kFwdConv + 96;
 constexpr int kFwdWRingMax = 6, kFwdHRingMax = 8;
@@ -64,6 +76,7 @@ constexpr int kFwdWf32 = 128 * 64 * 4;                 // 32 KB fp32 W tile (2 b
 constexpr int kFwdWBox = 128 * 32 * 4;                 // one 128 x 32 fp32 box
 constexpr int kFwdSmemMax = 227 * 1024;
 constexpr int kXentSmem = (2 * 128 * 65 + 4 * 64) * 4; // logits, gradients, statistics
+constexpr int kBarBytes = 768;                         // mbarriers, queue, flags
 // The tensor core's fp32 accumulation loses precision roughly in proportion to the
 // number of MMAs chained into one accumulator, so the accumulator is promoted:
 // every kSegChunks chunks (16 MMAs) the partial sum is folded into fp32 registers
@@ -73,6 +86,7 @@ constexpr int kSegChunks = 4;
 constexpr uint32_t kFwdTmemCols = 256;
 constexpr uint32_t kFwdTmemA = 128;
 constexpr int kFwdHidden = 0, kFwdXent = 2;   // TcFwdArgs::mode (1 = logits)
+constexpr int kQueue = 8;                     // claimed work items announced ahead
 
 // Layout: W ring | epilogue staging (mode 2) | batch ring | barriers.
 __host__ __device__ constexpr int fwd_wring(int mode, int Bn) {
@@ -82,14 +96,16 @@ __host__ __device__ constexpr int fwd_h_off(int mode, int Bn) {
   return fwd_wring(mode, Bn) * kFwdWf32 + (mode == 2 ? kXentSmem : 0);
 }
 __host__ __device__ constexpr int fwd_hring(int mode, int Bn) {
-  return (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode, Bn)) / (Bn * 128) < kFwdHRingMax
-             ? (kFwdSmemMax - 1024 - 512 - fwd_h_off(mode, Bn)) / (Bn * 128)
+  return (kFwdSmemMax - 1024 - kBarBytes - fwd_h_off(mode, Bn)) / (Bn * 128) < kFwdHRingMax
+             ? (kFwdSmemMax - 1024 - kBarBytes - fwd_h_off(mode, Bn)) / (Bn * 128)
              : kFwdHRingMax;
 }
 __host__ __device__ constexpr int fwd_bar_off(int mode, int Bn) {
   return fwd_h_off(mode, Bn) + fwd_hring(mode, Bn) * Bn * 128;
 }
-__host__ __device__ constexpr int fwd_smem(int mode, int Bn) { return fwd_bar_off(mode, Bn) + 512 + 1024; }
+__host__ __device__ constexpr int fwd_smem(int mode, int Bn) {
+  return fwd_bar_off(mode, Bn) + kBarBytes + 1024;
+}
 static_assert(fwd_hring(2, 64) >= 6 && fwd_hring(0, 64) == 8 && fwd_hring(0, 32) == 8 &&
                   fwd_smem(2, 64) <= kFwdSmemMax && fwd_smem(0, 64) <= kFwdSmemMax &&
                   fwd_smem(0, 48) <= kFwdSmemMax && fwd_smem(0, 32) <= kFwdSmemMax &&
@@ -121,6 +137,136 @@ struct GroupSync {
     return ok;
   }
 };
+
+// One work item of a forward layer: chunks [c_lo, c_hi) of tile tau (learner
+// tau / o_tiles, outputs 128 * (tau % o_tiles) ..), piece `piece` of the tile's np
+// pieces (np = 1: the whole tile).
+struct FwdItem {
+  int tau, c_lo, c_hi, piece, np;
+};
+
+// Work item `it` of the dynamic schedule: items [0, n_whole) are the whole tiles
+// [0, n_whole) in tile order; then come the pieces of the tail tiles [n_whole,
+// n_tiles), tile by tile, the pieces of a tile in order.
+template <class Args>
+__device__ __forceinline__ FwdItem fwd_item(const Args& a, int nk, int it) {
+  FwdItem f;
+  if (it < a.n_whole) {
+    f.tau = it;
+    f.c_lo = 0;
+    f.c_hi = nk;
+    f.piece = 0;
+    f.np = 1;
+  } else {
+    const int np = a.np_tail, i2 = it - a.n_whole, tt = i2 / np, p = i2 - tt * np;
+    f.tau = a.n_whole + tt;
+    f.c_lo = p * a.piece_chunks;
+    f.c_hi = f.c_lo + a.piece_chunks < nk ? f.c_lo + a.piece_chunks : nk;
+    f.piece = p;
+    f.np = np;
+  }
+  return f;
+}
+
+// The queue through which the claiming warp announces work items: items[q] holds
+// the k-th claimed item (k % kQueue == q), -1 once there are no more.
+struct ItemQueue {
+  uint64_t* full;    // [kQueue] item written
+  uint64_t* empty;   // [kQueue] read by every consuming warp
+  int* items;        // [kQueue]
+  // Producer (one lane): publish the k-th item.
+  __device__ __forceinline__ bool put(int k, int it, int* err) {
+    const int q = k % kQueue;
+    if (k >= kQueue && !mbar_wait(&empty[q], ((k / kQueue) - 1) & 1, err)) return false;
+    items[q] = it;
+    mbar_arrive(&full[q]);
+    return true;
+  }
+  // Consumer (a whole warp): the k-th item, read by every lane; lane 0 then frees the
+  // slot for this warp.  -1: no more items (or a wait expired).
+  __device__ __forceinline__ int take(int k, int lane, int* err) {
+    const int q = k % kQueue;
+    if (!wait_warp(&full[q], (k / kQueue) & 1, err)) return -1;
+    const int it = items[q];
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty[q]);
+    return it;
+  }
+};
+
+// The partial of a split tile: written by its piece, read by the piece that
+// completes the tile.  Slot (tail tile tt, piece p) = part[((tt * np + p) * 128 + r) * Bn].
+__device__ __forceinline__ void store_partial(float* dst, const float* acc, int gr, int Bn) {
+#pragma unroll
+  for (int m = 0; m < 2; ++m) {
+    const int cb = (2 * m + gr) * 16;
+    if (cb < Bn) {
+#pragma unroll
+      for (int q = 0; q < 16; q += 4)
+        __stcg(reinterpret_cast<float4*>(dst + cb + q),
+               make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                           acc[16 * m + q + 3]));
+    }
+  }
+}
+
+// A piece of a split tile ends: its partial goes to its slot; the piece that
+// completes the tile (the last to count itself in) replaces acc with the sum of all
+// the tile's partials in piece order (P_0 + P_1 + ... with IEEE fp32 adds, its own
+// read back like the others) and returns true: it runs the epilogue.  Every
+// converter thread calls it (`flag` is a shared word; false on an expired wait too).
+__device__ __forceinline__ bool piece_end(const TcFwdArgs& a, const FwdItem& f, int t, int r, int gr,
+                                          float* acc, GroupSync& gsync, volatile int* flag,
+                                          bool& ok) {
+  const int tt = f.tau - a.n_whole;
+  const float* slots = a.part + static_cast<int64_t>(tt) * f.np * 128 * a.Bn;
+  store_partial(a.part + ((static_cast<int64_t>(tt) * f.np + f.piece) * 128 + r) * a.Bn, acc, gr,
+                a.Bn);
+  if (!gsync()) { ok = false; return false; }   // every converter thread's partial is written
+  if (t == 0) {
+    fence_acq_rel_gpu();           // release: the CTA's partial before the count
+    const int before = atomicAdd(a.counters + tt, 1);
+    const int last = before == f.np - 1;
+    if (last) {
+      fence_acq_rel_gpu();         // acquire: every other piece's partial before the reads
+      a.counters[tt] = 0;          // ready for the next launch
+    }
+    *flag = last;
+  }
+  if (!gsync()) { ok = false; return false; }
+  if (!*flag) return false;
+  // acc = P_0 + P_1 + ... in piece order; the loads of two pieces are in flight at once
+  for (int m = 0; m < 2; ++m) {
+    const int cb = (2 * m + gr) * 16;
+    if (cb >= a.Bn) continue;
+#pragma unroll
+    for (int q = 0; q < 16; q += 4) {
+      const float* src = slots + static_cast<int64_t>(r) * a.Bn + cb + q;
+      const int64_t pstride = static_cast<int64_t>(128) * a.Bn;
+      float4 s0 = __ldcg(reinterpret_cast<const float4*>(src));
+      for (int p = 1; p < f.np; p += 2) {
+        const float4 v1 = __ldcg(reinterpret_cast<const float4*>(src + p * pstride));
+        float4 v2 = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (p + 1 < f.np) v2 = __ldcg(reinterpret_cast<const float4*>(src + (p + 1) * pstride));
+        s0.x = __fadd_rn(s0.x, v1.x);
+        s0.y = __fadd_rn(s0.y, v1.y);
+        s0.z = __fadd_rn(s0.z, v1.z);
+        s0.w = __fadd_rn(s0.w, v1.w);
+        if (p + 1 < f.np) {
+          s0.x = __fadd_rn(s0.x, v2.x);
+          s0.y = __fadd_rn(s0.y, v2.y);
+          s0.z = __fadd_rn(s0.z, v2.z);
+          s0.w = __fadd_rn(s0.w, v2.w);
+        }
+      }
+      acc[16 * m + q] = s0.x;
+      acc[16 * m + q + 1] = s0.y;
+      acc[16 * m + q + 2] = s0.z;
+      acc[16 * m + q + 3] = s0.w;
+    }
+  }
+  return true;
+}
 
 // Epilogue of the last layer when every class fits in one 128-row tile: the
 // softmax cross-entropy gradient straight from the accumulator (no logits
@@ -193,23 +339,23 @@ __device__ __forceinline__ int cta_of(int u, int U, int G) {
   return g;
 }
 
+// kDyn: dynamic work items (compiled separately from cluster split-K, so that each
+// schedule carries only its own code and registers).
+template <bool kDyn>
 __global__ void __launch_bounds__(kFwdThreads, 1)
     k_tc_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
                  const TcFwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = blockIdx.x, G = gridDim.x;
+  const int g = blockIdx.x;
   const int nk = (a.in + 63) / 64;
-  const int U = a.n_tiles * nk;
-  const int cq = a.cq > 1 ? a.cq : 1, part = g % cq;       // cluster split-K rank
-  const int u0 = cq > 1 ? (g / cq) * nk + part * nk / cq : unit_begin(g, U, G);
-  const int u1 = cq > 1 ? (g / cq) * nk + (part + 1) * nk / cq : unit_begin(g + 1, U, G);
-  const int n_local = u1 - u0;
+  constexpr bool dyn = kDyn;
+  const int cq = kDyn ? 1 : a.cq, part = g % cq;           // cluster split-K rank
+  const int n_items = a.n_whole + (a.n_tiles - a.n_whole) * a.np_tail;
   const int nw = fwd_wring(a.mode, a.Bn), nh = fwd_hring(a.mode, a.Bn);
   const int hbytes = a.Bn * 128;
   const int h_row0 = a.x_direct ? a.x_row0 : 0;           // batch rows inside the H (or X) map
-  const int tile0 = u0 / nk, c0 = u0 - tile0 * nk;         // first unit's tile and chunk
   uint8_t* xent_sm = smem + nw * kFwdWf32;
   uint8_t* h_base = smem + fwd_h_off(a.mode, a.Bn);
   uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + fwd_bar_off(a.mode, a.Bn));
@@ -222,10 +368,15 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   uint64_t* accr = accf + 2;               // [2] accumulator segment drained
   uint64_t* gbar = accr + 2;               // converter-group barrier
   uint64_t* done = gbar + 1;
-  uint64_t* pready = done + 1;             // this CTA's split-tile partial is written
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
+  ItemQueue queue{done + 1, done + 1 + kQueue, nullptr};
+  queue.items = reinterpret_cast<int*>(done + 1 + 2 * kQueue);
+  int* last_flag = queue.items + kQueue;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(last_flag + 1);
   auto wf = [&](int s) { return smem + s * kFwdWf32; };
   auto hb = [&](int s) { return h_base + s * hbytes; };
+  // Cluster split-K: this CTA's one item.  Dynamic: the k-th claimed item.
+  const FwdItem cl_item{g / cq, part * nk / cq, (part + 1) * nk / cq, 0, 1};
+  constexpr int kConsumers = 2 + kFwdConv / 32;            // MMA, batch and converter warps
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kFwdWRingMax; ++s) {
@@ -242,9 +393,13 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       mbar_init(&accf[b], 1);
       mbar_init(&accr[b], kFwdConv);
     }
+    if (dyn)
+      for (int q = 0; q < kQueue; ++q) {
+        mbar_init(&queue.full[q], 1);
+        mbar_init(&queue.empty[q], kConsumers);
+      }
     mbar_init(gbar, kFwdConv);
     mbar_init(done, 1);
-    mbar_init(pready, kFwdConv / 32);
     fence_barrier_init();
   }
   if (warp == 9) {
@@ -257,86 +412,114 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   const uint32_t tmem = *tmem_slot;
   grid_dep_wait();                       // the previous kernel's results are visible
 
+  // The k-th item of this CTA for a consuming warp (-1: none left).
+  auto next_item = [&](int k, FwdItem& f) -> bool {
+    if (!dyn) {
+      f = cl_item;
+      return k == 0;
+    }
+    const int it = queue.take(k, lane, a.err);
+    if (it < 0) return false;
+    f = fwd_item(a, nk, it);
+    return true;
+  };
+
   if (warp == 8) {
     if (lane == 0) {
+      // claim (dynamic), announce, and stream the weight tiles
       tma_prefetch_desc(&tm_w);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
-      int issued = 0, tau = tile0, c = c0;
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
+      int i = 0, issued = 0;
+      bool ok = true;
+      int next = dyn ? atomicAdd(a.dyn, 1) : 0;
+      for (int k = 0; ok; ++k) {
+        FwdItem f;
+        if (dyn) {
+          const int it = next < n_items ? next : -1;
+          if (!queue.put(k, it, a.err) || it < 0) break;
+          next = atomicAdd(a.dyn, 1);           // the next claim, hidden behind these loads
+          f = fwd_item(a, nk, it);
+        } else {
+          if (k > 0) break;
+          f = cl_item;
+        }
+        const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
         // learners whose rows are identical (a.share > 1) read one copy: the group's first
         const int jw = a.share > 1 ? (j / a.share) * a.share : j;
-        const int s = i % nw;
-        if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
-        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, jw, stream);
-        tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, jw, stream);
-        issued = i + 1;
-        if (++c == nk) { c = 0; ++tau; }
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
+          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, jw, stream);
+          tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, jw, stream);
+          issued = i + 1;
+        }
       }
       // Every load issued must have landed before the CTA may exit.
-      for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
-        mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
+      for (int u = issued - nw > 0 ? issued - nw : 0; u < issued; ++u)
+        mbar_wait(&wfull[u % nw], (u / nw) & 1, a.err);
     }
     if (cq > 1) {
       cluster_sync_all();   // the two barriers of the cluster reduction (see below)
       cluster_sync_all();
     }
   } else if (warp == 10) {
-    if (lane == 0) {
-      // Batch tiles.  Also: if the first tile began in an earlier CTA (which
-      // finishes it), publish this CTA's partial once the converter warps have
-      // written it (release order makes the partial visible before the count).
-      tma_prefetch_desc(&tm_h);
-      bool publish = cq == 1 && c0 != 0 && n_local > 0;
-      int issued = 0, tau = tile0, c = c0;
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.o_tiles;
-        const int s = i % nh;
-        if (publish && mbar_test(pready, 0)) {
-          red_release_add(a.counters + tile0, 1);
-          publish = false;
+    // batch tiles
+    if (lane == 0) tma_prefetch_desc(&tm_h);
+    int i = 0, issued = 0;
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        const int j = f.tau / a.o_tiles;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nh;
+          if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&hfull[s], a.Bn * 128);
+          tma_load_3d(hb(s), &tm_h, &hfull[s], c * 64, h_row0, j);
+          issued = i + 1;
         }
-        if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&hfull[s], a.Bn * 128);
-        tma_load_3d(hb(s), &tm_h, &hfull[s], c * 64, h_row0, j);
-        issued = i + 1;
-        if (++c == nk) { c = 0; ++tau; }
       }
-      for (int i = issued - nh > 0 ? issued - nh : 0; i < issued; ++i)
-        mbar_wait(&hfull[i % nh], (i / nh) & 1, a.err);
-      if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+      ok = __all_sync(0xffffffffu, ok);
     }
+    if (lane == 0)
+      for (int u = issued - nh > 0 ? issued - nh : 0; u < issued; ++u)
+        mbar_wait(&hfull[u % nh], (u / nh) & 1, a.err);
     if (cq > 1) {
       cluster_sync_all();
       cluster_sync_all();
     }
   } else if (warp == 9) {
-    if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(128, a.Bn);
-      int q = -1, c = c0, p = 0;        // accumulator segment index, chunk, position in run
-      for (int i = 0; i < n_local; ++i) {
-        const bool tlast = i == n_local - 1 || c == nk - 1;
-        const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
-        const int sh = i % nh, b = i & 1;
-        if (first) ++q;
-        const int ab = q & 1;
-        if (first && q >= 2 && !mbar_wait(&accr[ab], ((q >> 1) - 1) & 1, a.err)) break;
-        if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) break;
-        if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) break;
-        tc_fence_after();
-        const uint32_t at = tmem + kFwdTmemA + 32 * b;
-        const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh)));
-        const uint32_t d = tmem + 64 * ab;
+    const uint32_t idesc = umma_idesc_bf16(128, a.Bn);
+    int q = -1, i = 0;                 // accumulator segment index, chunk counter
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        for (int c = f.c_lo, p = 0; c < f.c_hi; ++c, ++p, ++i) {
+          const bool tlast = c == f.c_hi - 1;
+          const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+          const int sh = i % nh, b = i & 1;
+          if (first) ++q;
+          const int ab = q & 1;
+          if (first && q >= 2 && !mbar_wait(&accr[ab], ((q >> 1) - 1) & 1, a.err)) { ok = false; break; }
+          if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+          if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t at = tmem + kFwdTmemA + 32 * b;
+          const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh)));
+          const uint32_t d = tmem + 64 * ab;
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
-        tc_commit(&hempty[sh]);
-        tc_commit(&wfree[b]);
-        if (last) tc_commit(&accf[ab]);
-        ++p;
-        if (++c == nk) { c = 0; p = 0; }
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
+          tc_commit(&hempty[sh]);
+          tc_commit(&wfree[b]);
+          if (last) tc_commit(&accf[ab]);
+        }
       }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
       tc_commit(done);
       mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
     }
@@ -345,8 +528,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       cluster_sync_all();
     }
   } else {
-    // ---- warps 0-7: fp32 -> bf16 A tile (and H_0^T for the first layer), the
-    // accumulator drains and the tile epilogues
+    // ---- warps 0-7: fp32 -> bf16 A tile, the accumulator drains and the epilogues
     const int t = threadIdx.x;
     const int r = t & 127, gr = t >> 7;                    // accumulator row, column group
     const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
@@ -376,57 +558,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       ++drained;
       return true;
     };
-    // Tile tau is complete in this CTA's registers (or in this CTA's part of it).
-    // A tile split over CTAs g_first .. g_last is finished by g_first, the CTA that
-    // holds its first chunk and, in stream-K order, reaches it last; every other
-    // contributor writes its partial to its own slot and publishes it without
-    // waiting.  The finisher adds the partials in CTA order.
-    auto tile_end = [&](int tau, bool whole, float bias) -> bool {
+    // Tile tau's sum is in acc: bias, activation or cross-entropy, store.
+    auto epilogue = [&](int tau, float bias) {
       const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-      if (!whole) {
-        if (tau * nk < u0) {
-          float* mine = a.part + (static_cast<int64_t>(g) * 128 + r) * a.Bn;
-#pragma unroll
-          for (int m = 0; m < 2; ++m) {
-            const int cb = (2 * m + gr) * 16;
-            if (cb < a.Bn) {
-#pragma unroll
-              for (int q = 0; q < 16; q += 4)
-                __stcg(reinterpret_cast<float4*>(mine + cb + q),
-                       make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
-                                   acc[16 * m + q + 3]));
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(pready);
-#pragma unroll
-          for (int q = 0; q < 32; ++q) acc[q] = 0.f;
-          return true;
-        }
-        const int g_last = cta_of((tau + 1) * nk - 1, U, G);
-        if (t == 0) {
-          const bool ok = spin_acquire_eq(a.counters + tau, g_last - g, a.err);
-          if (ok) a.counters[tau] = 0;   // ready for the next launch
-        }
-        if (!gsync()) return false;
-        for (int gg = g + 1; gg <= g_last; ++gg) {
-          const float* src = a.part + (static_cast<int64_t>(gg) * 128 + r) * a.Bn;
-#pragma unroll
-          for (int m = 0; m < 2; ++m) {
-            const int cb = (2 * m + gr) * 16;
-            if (cb < a.Bn) {
-#pragma unroll
-              for (int q = 0; q < 16; q += 4) {
-                const float4 v = __ldcg(reinterpret_cast<const float4*>(src + cb + q));
-                acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v.x);
-                acc[16 * m + q + 1] = __fadd_rn(acc[16 * m + q + 1], v.y);
-                acc[16 * m + q + 2] = __fadd_rn(acc[16 * m + q + 2], v.z);
-                acc[16 * m + q + 3] = __fadd_rn(acc[16 * m + q + 3], v.w);
-              }
-            }
-          }
-        }
-      }
       const int o = ot * 128 + r;
       const bool valid = o < a.out;
       if (a.mode == kFwdXent) {
@@ -452,79 +586,78 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           }
         }
       }
-#pragma unroll
-      for (int q = 0; q < 32; ++q) acc[q] = 0.f;
-      return true;
     };
     bool ok = true;
-    int tau = tile0, c = c0, p = 0;
-    float tbias = 0.f;                 // bias of row r of the current tile, loaded early
+    int i = 0;
     int ep_tau = -1;                   // cluster split-K: this CTA's tile
     float ep_bias = 0.f;
-    for (int i = 0; i < n_local && ok; ++i) {
-      const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-      const bool tlast = i == n_local - 1 || c == nk - 1;
-      if (p == 0) {
-        const int o = ot * 128 + r;
-        tbias = o < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
-      }
-      const int sw = i % nw, bb = i & 1;
-      if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
-      if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
-      tc_fence_after();
-      {
-        // Row 32*(warp%4) + lane, K half warp/4: 32 floats from the swizzled box
-        // (16-byte chunk q of row r sits at chunk q ^ (r%8)), packed to bf16 pairs,
-        // stored as 16 TMEM columns of this lane.
-        const int row = 32 * (warp & 3) + lane, half = warp >> 2;
-        const uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
-        uint32_t pk[16];
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
+      const int ob = ot * 128 + r;
+      const float tbias = ob < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + ob] : 0.f;
+      for (int c = f.c_lo, p = 0; c < f.c_hi && ok; ++c, ++p, ++i) {
+        const bool tlast = c == f.c_hi - 1;
+        const int sw = i % nw, bb = i & 1;
+        if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+        if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+        {
+          // Row 32*(warp%4) + lane, K half warp/4: 32 floats from the swizzled box
+          // (16-byte chunk q of row r sits at chunk q ^ (r%8)), packed to bf16 pairs,
+          // stored as 16 TMEM columns of this lane.
+          const int row = 32 * (warp & 3) + lane, half = warp >> 2;
+          const uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
+          uint32_t pk[16];
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const float4 x = *reinterpret_cast<const float4*>(src + ((q ^ (row & 7)) << 4));
-          pk[2 * q] = pack_bf16x2(x.x, x.y);
-          pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
+          for (int q = 0; q < 8; ++q) {
+            const float4 x = *reinterpret_cast<const float4*>(src + ((q ^ (row & 7)) << 4));
+            pk[2 * q] = pack_bf16x2(x.x, x.y);
+            pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
+          }
+          tmem_st16(tbase + kFwdTmemA + 32 * bb + 16 * half, pk);
         }
-        tmem_st16(tbase + kFwdTmemA + 32 * bb + 16 * half, pk);
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&wempty[sw]);   // the fp32 tile is no longer needed
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&conv[bb]);
-      if (p % kSegChunks == 0) ++qc;
-      if (tlast) {
-        while (ok && drained <= qc)
-          if (!drain()) ok = false;
-        if (ok && cq > 1) {
-          // cluster split-K: rank 0 keeps its partial in registers, the others
-          // leave theirs in the (now idle) weight ring for rank 0 to read
-          ep_tau = tau;
-          ep_bias = tbias;
-          if (part != 0) {
-            float* red = reinterpret_cast<float*>(smem) + r * a.Bn;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&wempty[sw]);   // the fp32 tile is no longer needed
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&conv[bb]);
+        if (p % kSegChunks == 0) ++qc;
+        if (tlast) {
+          while (ok && drained <= qc)
+            if (!drain()) ok = false;
+          if (!ok) break;
+          if (!dyn) {
+            // cluster split-K: rank 0 keeps its partial in registers, the others
+            // leave theirs in the (now idle) weight ring for rank 0 to read
+            ep_tau = f.tau;
+            ep_bias = tbias;
+            if (part != 0) {
+              float* red = reinterpret_cast<float*>(smem) + r * a.Bn;
 #pragma unroll
-            for (int m = 0; m < 2; ++m) {
-              const int cb = (2 * m + gr) * 16;
-              if (cb < a.Bn) {
+              for (int m = 0; m < 2; ++m) {
+                const int cb = (2 * m + gr) * 16;
+                if (cb < a.Bn) {
 #pragma unroll
-                for (int q = 0; q < 16; q += 4)
-                  *reinterpret_cast<float4*>(red + cb + q) =
-                      make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
-                                  acc[16 * m + q + 3]);
+                  for (int q = 0; q < 16; q += 4)
+                    *reinterpret_cast<float4*>(red + cb + q) =
+                        make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                                    acc[16 * m + q + 3]);
+                }
               }
             }
+          } else {
+            const bool fin = f.np == 1 || piece_end(a, f, t, r, gr, acc, gsync, last_flag, ok);
+            if (ok && fin) epilogue(f.tau, tbias);
+#pragma unroll
+            for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+            ok = __all_sync(0xffffffffu, ok);
           }
-        } else if (ok) {
-          const bool whole = (tau != tile0 || c0 == 0) && c == nk - 1;
-          ok = __all_sync(0xffffffffu, tile_end(tau, whole, tbias));
+        } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
+          if (!drain()) ok = false;   // one segment behind the MMAs
         }
-      } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
-        if (!drain()) ok = false;   // one segment behind the MMAs
       }
-      ++p;
-      if (++c == nk) { c = 0; p = 0; ++tau; }
     }
     if (cq > 1) {
       // Cluster split-K finish: rank 0 adds the partials of ranks 1.. (left in their
@@ -549,7 +682,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
             }
           }
         }
-        tile_end(ep_tau, true, ep_bias);
+        epilogue(ep_tau, ep_bias);
       }
       cluster_sync_all();   // rank 0 has read them: every CTA may exit
     }
@@ -561,24 +694,37 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kFwdTmemCols);
   }
+  if (dyn && threadIdx.x == 0) {
+    // the last CTA out resets the claim counters for the next launch (every claim of
+    // every CTA precedes that CTA's increment here)
+    __threadfence();
+    if (atomicAdd(a.dyn + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+      a.dyn[0] = 0;
+      a.dyn[1] = 0;
+    }
+  }
 }
 
+
 // ------------------------------------------------------------------ backward
-// Persistent stream-K backward of one layer.  Unit u = (tile, chunk): tile = (learner
-// j, input features i0 .. i0+127), chunk = output rows o0 .. o0+63 of W_l.  CTA g of G
-// owns the contiguous units [g*U/G, (g+1)*U/G).  Per unit:
+// Backward of one layer on the tensor cores.  Tile = (learner j, input features i0 ..
+// i0+127), chunk = output rows o0 .. o0+63 of W_l.  Per chunk:
 //   dW^T[i][o] = sum_b H_{l-1}[b][i] dZ_l[b][o]    both operands MN-major, read as stored
 //                                                  (H tile of the tile, dZ tile of the chunk)
 //   W[o][i]   -= lr dW^T[i][o]                     fp32, in shared memory, then TMA-stored
 //   dH^T[i][b] += sum_o W[o][i] dZ_l[b][o]          pre-update weights (A = W^T, bf16, in TMEM)
 // so W is read once and written once.  dH^T of a tile accumulates over its chunks (with
-// the same every-kSegChunks promotion as the forward); a tile split over CTAs is
-// finished, as in the forward, by the CTA holding its first chunk.  The tile epilogue
-// applies the ReLU mask of H_{l-1}, writes dZ_{l-1} and updates b_{l-1}.
+// the same every-kSegChunks promotion as the forward), and the tile epilogue applies
+// the ReLU mask of H_{l-1}, writes dZ_{l-1} and updates b_{l-1}.  Without dX (the
+// first layer) only dW and the update remain.
+// The work is claimed dynamically like the forward's: whole tiles, then the last
+// tiles (one per SM) split into pieces of TcBwdArgs::piece_chunks chunks; a piece
+// writes its dH^T partial to its slot, and the piece that completes a tile adds the
+// tile's partials in piece order and runs the epilogue (no CTA waits for another).
 // Warps 0-3: thread t owns input feature i0 + t (TMEM lane t): it converts its column
 // of the fp32 chunk to the bf16 A tile, applies the update in shared memory and runs
-// the tile epilogue.  Warp 4 loads W chunks and H tiles, warp 5 issues the MMAs, warp
-// 6 loads dZ tiles and publishes a split tile's partial, warp 7 TMA-stores updated
+// the tile epilogue.  Warp 4 claims the work items and loads W chunks and each item's
+// H tile, warp 5 issues the MMAs, warp 6 loads dZ tiles, warp 7 TMA-stores updated
 // chunks (bulk stores: per-thread row stores of the same bytes ran at half the speed)
 // and frees their slots once read.  Each waiting role has a warp of its own: a lane
 // blocked in an mbarrier wait holds up the other lanes of its warp.
@@ -596,16 +742,73 @@ __host__ __device__ constexpr int bwd_wring(int Bn) { return (void)Bn, 5; }
 __host__ __device__ constexpr int bwd_h_off(int Bn) { return bwd_wring(Bn) * kBwdWf32; }
 __host__ __device__ constexpr int bwd_z_off(int Bn) { return bwd_h_off(Bn) + 2 * 2 * Bn * 128; }
 __host__ __device__ constexpr int bwd_zring(int Bn) {
-  return (kBwdSmemMax - 1024 - 512 - bwd_z_off(Bn)) / (Bn * 128) < kBwdZRingMax
-             ? (kBwdSmemMax - 1024 - 512 - bwd_z_off(Bn)) / (Bn * 128)
+  return (kBwdSmemMax - 1024 - kBarBytes - bwd_z_off(Bn)) / (Bn * 128) < kBwdZRingMax
+             ? (kBwdSmemMax - 1024 - kBarBytes - bwd_z_off(Bn)) / (Bn * 128)
              : kBwdZRingMax;
 }
 __host__ __device__ constexpr int bwd_bar_off(int Bn) { return bwd_z_off(Bn) + bwd_zring(Bn) * Bn * 128; }
-__host__ __device__ constexpr int bwd_smem(int Bn) { return bwd_bar_off(Bn) + 512 + 1024; }
+__host__ __device__ constexpr int bwd_smem(int Bn) { return bwd_bar_off(Bn) + kBarBytes + 1024; }
 static_assert(bwd_zring(64) >= 4 && bwd_zring(48) >= 6 && bwd_zring(32) >= 8 && bwd_zring(16) >= 8 &&
                   bwd_smem(64) <= kBwdSmemMax && bwd_smem(48) <= kBwdSmemMax &&
                   bwd_smem(32) <= kBwdSmemMax && bwd_smem(16) <= kBwdSmemMax,
               "backward shared-memory plan");
+
+// The backward's counterpart of piece_end: thread t holds row t of the tile's dH^T
+// partial (all Bn columns) in accx.  Slot (tail tile tt, piece p) =
+// part[((tt * np + p) * 128 + t) * Bn].
+__device__ __forceinline__ bool bwd_piece_end(const TcBwdArgs& a, const FwdItem& f, int t,
+                                              float* accx, GroupSync& gsync, volatile int* flag,
+                                              bool& ok) {
+  const int tt = f.tau - a.n_whole;
+  const int64_t pstride = static_cast<int64_t>(128) * a.Bn;
+  float* mine = a.part + (static_cast<int64_t>(tt) * f.np + f.piece) * pstride +
+                static_cast<int64_t>(t) * a.Bn;
+#pragma unroll
+  for (int cb = 0; cb < 64; cb += 4)
+    if (cb < a.Bn)
+      __stcg(reinterpret_cast<float4*>(mine + cb),
+             make_float4(accx[cb], accx[cb + 1], accx[cb + 2], accx[cb + 3]));
+  if (!gsync()) { ok = false; return false; }   // every converter thread's partial is written
+  if (t == 0) {
+    fence_acq_rel_gpu();           // release: the CTA's partial before the count
+    const int before = atomicAdd(a.counters + tt, 1);
+    const int last = before == f.np - 1;
+    if (last) {
+      fence_acq_rel_gpu();         // acquire: every other piece's partial before the reads
+      a.counters[tt] = 0;          // ready for the next launch
+    }
+    *flag = last;
+  }
+  if (!gsync()) { ok = false; return false; }
+  if (!*flag) return false;
+  // accx = P_0 + P_1 + ... in piece order; two pieces' loads in flight at once
+  const float* src = a.part + static_cast<int64_t>(tt) * f.np * pstride + static_cast<int64_t>(t) * a.Bn;
+#pragma unroll
+  for (int cb = 0; cb < 64; cb += 4) {
+    if (cb >= a.Bn) continue;
+    float4 s0 = __ldcg(reinterpret_cast<const float4*>(src + cb));
+    for (int p = 1; p < f.np; p += 2) {
+      const float4 v1 = __ldcg(reinterpret_cast<const float4*>(src + p * pstride + cb));
+      float4 v2 = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (p + 1 < f.np) v2 = __ldcg(reinterpret_cast<const float4*>(src + (p + 1) * pstride + cb));
+      s0.x = __fadd_rn(s0.x, v1.x);
+      s0.y = __fadd_rn(s0.y, v1.y);
+      s0.z = __fadd_rn(s0.z, v1.z);
+      s0.w = __fadd_rn(s0.w, v1.w);
+      if (p + 1 < f.np) {
+        s0.x = __fadd_rn(s0.x, v2.x);
+        s0.y = __fadd_rn(s0.y, v2.y);
+        s0.z = __fadd_rn(s0.z, v2.z);
+        s0.w = __fadd_rn(s0.w, v2.w);
+      }
+    }
+    accx[cb] = s0.x;
+    accx[cb + 1] = s0.y;
+    accx[cb + 2] = s0.z;
+    accx[cb + 3] = s0.w;
+  }
+  return true;
+}
 
 __global__ void __launch_bounds__(kBwdThreads, 1)
     k_tc_backward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
@@ -613,14 +816,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = blockIdx.x, G = gridDim.x;
   const int nc = (a.out + 63) / 64;
-  const int U = a.n_tiles * nc;
-  const int u0 = unit_begin(g, U, G), u1 = unit_begin(g + 1, U, G);
-  const int n_local = u1 - u0;
+  const int n_items = a.n_whole + (a.n_tiles - a.n_whole) * a.np_tail;
   const int nw = bwd_wring(a.Bn), nz = bwd_zring(a.Bn);
   const int tbytes = a.Bn * 128;                           // one [Bn][64] bf16 tile
-  const int tile0 = u0 / nc, c0 = u0 - tile0 * nc;
   uint8_t* h_base = smem + bwd_h_off(a.Bn);
   uint8_t* z_base = smem + bwd_z_off(a.Bn);
   uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + bwd_bar_off(a.Bn));
@@ -629,7 +828,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   uint64_t* zfull = upd + kBwdWRingMax;
   uint64_t* zempty = zfull + kBwdZRingMax;   // dZ tile consumed by both MMAs
   uint64_t* hfull = zempty + kBwdZRingMax;   // [2]
-  uint64_t* hempty = hfull + 2;              // [2] tile epilogue done
+  uint64_t* hempty = hfull + 2;              // [2] the item's epilogue (or last MMA) is done
   uint64_t* conv = hempty + 2;               // [2] W^T written to TMEM
   uint64_t* afree = conv + 2;                // [2] W^T consumed by the dX MMA
   uint64_t* dwdone = afree + 2;              // [2] dW^T of the chunk complete
@@ -638,11 +837,14 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   uint64_t* xr = xf + 2;                     // [2] dH^T segment drained
   uint64_t* gbar = xr + 2;
   uint64_t* done = gbar + 1;
-  uint64_t* pready = done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
+  ItemQueue queue{done + 1, done + 1 + kQueue, nullptr};
+  queue.items = reinterpret_cast<int*>(done + 1 + 2 * kQueue);
+  int* last_flag = queue.items + kQueue;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(last_flag + 1);
   auto wf = [&](int s) { return smem + s * kBwdWf32; };
   auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
   auto zb = [&](int s) { return z_base + s * tbytes; };
+  constexpr int kConsumers = 3 + kBwdConv / 32;             // MMA, dZ, store + converter warps
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kBwdWRingMax; ++s) {
@@ -664,9 +866,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       mbar_init(&xf[b], 1);
       mbar_init(&xr[b], kBwdConv / 32);
     }
+    for (int q = 0; q < kQueue; ++q) {
+      mbar_init(&queue.full[q], 1);
+      mbar_init(&queue.empty[q], kConsumers);
+    }
     mbar_init(gbar, kBwdConv);
     mbar_init(done, 1);
-    mbar_init(pready, kBwdConv / 32);
     fence_barrier_init();
   }
   if (warp == 5) {
@@ -679,121 +884,137 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   const uint32_t tmem = *tmem_slot;
   grid_dep_wait();                       // the previous kernel's results are visible
 
+  auto next_item = [&](int k, FwdItem& f) -> bool {
+    const int it = queue.take(k, lane, a.err);
+    if (it < 0) return false;
+    f = fwd_item(a, nc, it);
+    return true;
+  };
+
   if (warp == 4) {
     if (lane == 0) {
-      // W chunks, and each tile's H tile (two 64-feature boxes) ahead of its first chunk
+      // claim, announce, and load: each item's H tile (two 64-feature boxes) ahead of
+      // its first W chunk, then its W chunks
       tma_prefetch_desc(&tm_w);
       tma_prefetch_desc(&tm_h);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
-      int issued = 0, tau = tile0, c = c0, kt = 0;
+      int i = 0, issued = 0;
       bool ok = true;
-      for (int i = 0; i < n_local && ok; ++i) {
-        const int j = tau / a.s_tiles, i0 = (tau - j * a.s_tiles) * 128;
-        if (i == 0 || c == 0) {
-          const int hbuf = kt & 1;
-          if (kt >= 2 && !mbar_wait(&hempty[hbuf], ((kt >> 1) - 1) & 1, a.err)) { ok = false; break; }
-          mbar_arrive_expect_tx(&hfull[hbuf], 2 * tbytes);
-          tma_load_3d(hb(hbuf), &tm_h, &hfull[hbuf], i0, a.h_row0, j);
-          tma_load_3d(hb(hbuf) + tbytes, &tm_h, &hfull[hbuf], i0 + 64, a.h_row0, j);
-          ++kt;
+      int next = atomicAdd(a.dyn, 1);
+      for (int k = 0; ok; ++k) {
+        const int it = next < n_items ? next : -1;
+        if (!queue.put(k, it, a.err) || it < 0) break;
+        next = atomicAdd(a.dyn, 1);           // the next claim, hidden behind these loads
+        const FwdItem f = fwd_item(a, nc, it);
+        const int j = f.tau / a.s_tiles, i0 = (f.tau - j * a.s_tiles) * 128;
+        const int hbuf = k & 1;
+        if (k >= 2 && !mbar_wait(&hempty[hbuf], ((k >> 1) - 1) & 1, a.err)) break;
+        mbar_arrive_expect_tx(&hfull[hbuf], 2 * tbytes);
+        tma_load_3d(hb(hbuf), &tm_h, &hfull[hbuf], i0, a.h_row0, j);
+        tma_load_3d(hb(hbuf) + tbytes, &tm_h, &hfull[hbuf], i0 + 64, a.h_row0, j);
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
+          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], i0, c * 64, j, stream);
+          issued = i + 1;
         }
-        const int s = i % nw;
-        if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
-        mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
-        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], i0, c * 64, j, stream);
-        issued = i + 1;
-        if (++c == nc) { c = 0; ++tau; }
       }
-      for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
-        mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
-      for (int k = kt - 2 > 0 ? kt - 2 : 0; k < kt; ++k) mbar_wait(&hfull[k & 1], (k >> 1) & 1, a.err);
+      for (int u = issued - nw > 0 ? issued - nw : 0; u < issued; ++u)
+        mbar_wait(&wfull[u % nw], (u / nw) & 1, a.err);
     }
   } else if (warp == 6) {
-    if (lane == 0) {
-      // dZ tiles; also publishes this CTA's partial of a split first tile (see the
-      // forward).
-      tma_prefetch_desc(&tm_dz);
-      bool publish = a.has_dx && c0 != 0 && n_local > 0;
-      int issued = 0, tau = tile0, c = c0;
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.s_tiles;
-        const int s = i % nz;
-        if (publish && mbar_test(pready, 0)) {
-          red_release_add(a.counters + tile0, 1);
-          publish = false;
+    // dZ tiles of each chunk
+    if (lane == 0) tma_prefetch_desc(&tm_dz);
+    int i = 0, issued = 0;
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        const int j = f.tau / a.s_tiles;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nz;
+          if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&zfull[s], tbytes);
+          tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j);
+          issued = i + 1;
         }
-        if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&zfull[s], tbytes);
-        tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j);
-        issued = i + 1;
-        if (++c == nc) { c = 0; ++tau; }
       }
-      for (int i = issued - nz > 0 ? issued - nz : 0; i < issued; ++i)
-        mbar_wait(&zfull[i % nz], (i / nz) & 1, a.err);
-      if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
+      ok = __all_sync(0xffffffffu, ok);
     }
+    if (lane == 0)
+      for (int u = issued - nz > 0 ? issued - nz : 0; u < issued; ++u)
+        mbar_wait(&zfull[u % nz], (u / nz) & 1, a.err);
   } else if (warp == 7) {
-    if (lane == 0) {
-      // Store each updated chunk; its slot is released once the TMA has read it
-      // (two stores in flight).
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
-      int tau = tile0, c = c0, stored = 0;
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.s_tiles, i0 = (tau - j * a.s_tiles) * 128;
-        const int s = i % nw;
-        if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
-        tma_store_3d_hint(&tm_w, wf(s), i0, c * 64, j, stream);
-        tma_store_commit();
-        stored = i + 1;
-        if (i > 0) {
-          tma_store_wait_read_1();
-          mbar_arrive(&wempty[(i - 1) % nw]);
+    // Store each updated chunk; its slot is released once the TMA has read it (two
+    // stores in flight).
+    const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+    int i = 0;
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        const int j = f.tau / a.s_tiles, i0 = (f.tau - j * a.s_tiles) * 128;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) { ok = false; break; }
+          tma_store_3d_hint(&tm_w, wf(s), i0, c * 64, j, stream);
+          tma_store_commit();
+          if (i > 0) {
+            tma_store_wait_read_1();
+            mbar_arrive(&wempty[(i - 1) % nw]);
+          }
         }
-        if (++c == nc) { c = 0; ++tau; }
       }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
       tma_store_wait_read_all();   // (before the shared memory is released)
-      if (stored > 0) mbar_arrive(&wempty[(stored - 1) % nw]);
+      if (i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
     }
   } else if (warp == 5) {
-    if (lane == 0) {
-      const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
-      const uint32_t idesc_dx = umma_idesc_bf16(128, a.Bn);
-      const int kb = a.Bn / 16;   // K = Bn for dW
-      int tau = tile0, c = c0, p = 0, q = -1, kt = -1;
-      for (int i = 0; i < n_local; ++i) {
-        const bool tlast = i == n_local - 1 || c == nc - 1;
-        const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
-        const int sz = i % nz, b = i & 1;
-        if (p == 0) {
-          ++kt;
-          if (!mbar_wait(&hfull[kt & 1], (kt >> 1) & 1, a.err)) break;
-        }
-        if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) break;
-        if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) break;
-        tc_fence_after();
-        const uint32_t hs = smem_u32(hb(kt & 1)), zs = smem_u32(zb(sz));
-        for (int kk = 0; kk < kb; ++kk)
-          tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
-                      umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
-        tc_commit(&dwdone[b]);
-        if (a.has_dx) {
-          if (first) ++q;
-          const int xb = q & 1;
-          if (first && q >= 2 && !mbar_wait(&xr[xb], ((q >> 1) - 1) & 1, a.err)) break;
-          if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) break;
+    const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
+    const uint32_t idesc_dx = umma_idesc_bf16(128, a.Bn);
+    const int kb = a.Bn / 16;   // K = Bn for dW
+    int i = 0, q = -1;
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        if (!mbar_wait(&hfull[k & 1], (k >> 1) & 1, a.err)) ok = false;
+        const uint32_t hs = smem_u32(hb(k & 1));
+        for (int c = f.c_lo, p = 0; ok && c < f.c_hi; ++c, ++p, ++i) {
+          const bool tlast = c == f.c_hi - 1;
+          const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+          const int sz = i % nz, b = i & 1;
+          if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) { ok = false; break; }
+          if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
           tc_fence_after();
-          const uint64_t zd = umma_desc_sw128(zs);
+          const uint32_t zs = smem_u32(zb(sz));
+          for (int kk = 0; kk < kb; ++kk)
+            tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
+                        umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+          tc_commit(&dwdone[b]);
+          if (a.has_dx) {
+            if (first) ++q;
+            const int xb = q & 1;
+            if (first && q >= 2 && !mbar_wait(&xr[xb], ((q >> 1) - 1) & 1, a.err)) { ok = false; break; }
+            if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+            tc_fence_after();
+            const uint64_t zd = umma_desc_sw128(zs);
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            tc_mma_bf16_ta(tmem + 64 * xb, tmem + kBwdTmemA + 32 * b + 8 * kk, zd + 2 * kk, idesc_dx,
-                           (!first || kk > 0) ? 1u : 0u);
-          tc_commit(&afree[b]);
-          if (last) tc_commit(&xf[xb]);
+            for (int kk = 0; kk < 4; ++kk)
+              tc_mma_bf16_ta(tmem + 64 * xb, tmem + kBwdTmemA + 32 * b + 8 * kk, zd + 2 * kk, idesc_dx,
+                             (!first || kk > 0) ? 1u : 0u);
+            tc_commit(&afree[b]);
+            if (last) tc_commit(&xf[xb]);
+          }
+          tc_commit(&zempty[sz]);
         }
-        tc_commit(&zempty[sz]);
-        ++p;
-        if (++c == nc) { c = 0; p = 0; ++tau; }
       }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
       tc_commit(done);
       mbar_wait(done, 0, a.err);
     }
@@ -826,46 +1047,13 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       ++drained;
       return true;
     };
-    // End of tile tau in this CTA (has_dx): finish it, or publish this CTA's part.
-    auto tile_end = [&](int tau, bool whole, int kt) -> bool {
+    // dZ_{l-1}[b][i] = dH[b][i] * (H_{l-1}[b][i] > 0), b < B; b_{l-1}[i] -= lr sum_b.
+    // (The item's H tile landed long ago; the wait makes the TMA's writes visible here.)
+    auto epilogue = [&](int tau, int k) -> bool {
       const int j = tau / a.s_tiles, fi = (tau - j * a.s_tiles) * 128 + t;
-      if (!whole) {
-        if (tau * nc < u0) {
-          float* mine = a.part + (static_cast<int64_t>(g) * 128 + t) * a.Bn;
-#pragma unroll
-          for (int cb = 0; cb < 64; cb += 4)
-            if (cb < a.Bn)
-              __stcg(reinterpret_cast<float4*>(mine + cb),
-                     make_float4(accx[cb], accx[cb + 1], accx[cb + 2], accx[cb + 3]));
-          __syncwarp();
-          if (lane == 0) mbar_arrive(pready);
-          return true;
-        }
-        const int g_last = cta_of((tau + 1) * nc - 1, U, G);
-        if (t == 0) {
-          const bool ok = spin_acquire_eq(a.counters + tau, g_last - g, a.err);
-          if (ok) a.counters[tau] = 0;
-        }
-        if (!gsync()) return false;
-        for (int gg = g + 1; gg <= g_last; ++gg) {
-          const float* src = a.part + (static_cast<int64_t>(gg) * 128 + t) * a.Bn;
-#pragma unroll
-          for (int cb = 0; cb < 64; cb += 4) {
-            if (cb < a.Bn) {
-              const float4 v = __ldcg(reinterpret_cast<const float4*>(src + cb));
-              accx[cb] = __fadd_rn(accx[cb], v.x);
-              accx[cb + 1] = __fadd_rn(accx[cb + 1], v.y);
-              accx[cb + 2] = __fadd_rn(accx[cb + 2], v.z);
-              accx[cb + 3] = __fadd_rn(accx[cb + 3], v.w);
-            }
-          }
-        }
-      }
-      // dZ_{l-1}[b][i] = dH[b][i] * (H_{l-1}[b][i] > 0), b < B; b_{l-1}[i] -= lr sum_b.
-      // (The H tile landed long ago; the wait makes the TMA's writes visible here.)
-      if (!wait_warp(&hfull[kt & 1], (kt >> 1) & 1, a.err)) return false;
+      if (!wait_warp(&hfull[k & 1], (k >> 1) & 1, a.err)) return false;
       if (fi < a.in) {
-        const uint8_t* hcol = hb(kt & 1) + (t >> 6) * a.Bn * 128;
+        const uint8_t* hcol = hb(k & 1) + (t >> 6) * a.Bn * 128;
         __nv_bfloat16* dz = a.dz_prev + static_cast<int64_t>(j) * a.Bn * a.pitch_in + fi;
         float db = 0.f;
 #pragma unroll
@@ -884,70 +1072,71 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       return true;
     };
     bool ok = true;
-    int tau = tile0, c = c0, p = 0, kt = -1;
-    for (int i = 0; i < n_local && ok; ++i) {
-      const bool tlast = i == n_local - 1 || c == nc - 1;
-      const int sw = i % nw, b = i & 1;
-      if (p == 0) ++kt;
-      if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
-      float* w = reinterpret_cast<float*>(wf(sw));
-      float wv[64];
+    int i = 0;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      for (int c = f.c_lo, p = 0; ok && c < f.c_hi; ++c, ++p, ++i) {
+        const bool tlast = c == f.c_hi - 1;
+        const int sw = i % nw, b = i & 1;
+        if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+        float* w = reinterpret_cast<float*>(wf(sw));
+        float wv[64];
 #pragma unroll
-      for (int o = 0; o < 64; ++o) wv[o] = w[o * 128 + t];
-      if (a.has_dx) {
-        if (i >= 2 && !wait_warp(&afree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        for (int o = 0; o < 64; ++o) wv[o] = w[o * 128 + t];
+        if (a.has_dx) {
+          if (i >= 2 && !wait_warp(&afree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int q = 0; q < 16; ++q) pk[q] = pack_bf16x2(wv[32 * hh + 2 * q], wv[32 * hh + 2 * q + 1]);
+            tmem_st16(tbase + kBwdTmemA + 32 * b + 16 * hh, pk);
+          }
+          tmem_st_wait();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&conv[b]);
+        }
+        if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          uint32_t pk[16];
+        for (int qb = 0; qb < 4; ++qb) {
+          float d[16];
+          tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
+          tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 16; ++q) pk[q] = pack_bf16x2(wv[32 * hh + 2 * q], wv[32 * hh + 2 * q + 1]);
-          tmem_st16(tbase + kBwdTmemA + 32 * b + 16 * hh, pk);
+          for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
         }
-        tmem_st_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&conv[b]);
-      }
-      if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
-      tc_fence_after();
+        if (lane == 0) mbar_arrive(&dwfree[b]);
 #pragma unroll
-      for (int qb = 0; qb < 4; ++qb) {
-        float d[16];
-        tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
-        tmem_ld_wait();
+        for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&upd[sw]);
+        if (a.has_dx) {
+          if (p % kSegChunks == 0) ++qc;
+          if (tlast) {
+            while (ok && drained <= qc)
+              if (!drain()) ok = false;
+            if (ok) {
+              const bool fin = f.np == 1 || bwd_piece_end(a, f, t, accx, gsync, last_flag, ok);
+              if (ok && fin && !epilogue(f.tau, k)) ok = false;
+              ok = __all_sync(0xffffffffu, ok);
 #pragma unroll
-        for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&dwfree[b]);
-#pragma unroll
-      for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&upd[sw]);
-      if (a.has_dx) {
-        if (p % kSegChunks == 0) ++qc;
-        if (tlast) {
-          while (ok && drained <= qc)
+              for (int q = 0; q < 64; ++q) accx[q] = 0.f;
+            }
+          } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
             if (!drain()) ok = false;
-          if (ok) {
-            const bool whole = (tau != tile0 || c0 == 0) && c == nc - 1;
-            ok = __all_sync(0xffffffffu, tile_end(tau, whole, kt));
-#pragma unroll
-            for (int q = 0; q < 64; ++q) accx[q] = 0.f;
           }
-        } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
-          if (!drain()) ok = false;
+        }
+        if (tlast) {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&hempty[k & 1]);   // the H tile may be replaced
         }
       }
-      if (tlast) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&hempty[kt & 1]);   // the H tile may be replaced
-      }
-      ++p;
-      if (++c == nc) { c = 0; p = 0; ++tau; }
     }
   }
   tc_fence_before();
@@ -956,6 +1145,14 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kBwdTmemCols);
+  }
+  if (threadIdx.x == 0) {
+    // the last CTA out resets the claim counters for the next launch
+    __threadfence();
+    if (atomicAdd(a.dyn + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+      a.dyn[0] = 0;
+      a.dyn[1] = 0;
+    }
   }
 }
 
@@ -968,7 +1165,6 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
 // the other roles through a small queue in shared memory; the last CTA to finish
 // resets the counters.  Roles as in k_tc_backward, without the dX path.
 constexpr int kRun = 8;                 // chunks per work item
-constexpr int kQueue = 8;               // queued work items
 __host__ __device__ constexpr int upd_smem(int Bn) { return bwd_smem(Bn) + 512; }
 static_assert(upd_smem(64) <= kBwdSmemMax && upd_smem(48) <= kBwdSmemMax &&
                   upd_smem(32) <= kBwdSmemMax && upd_smem(16) <= kBwdSmemMax,
@@ -1240,11 +1436,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
 // Z_1' = X' W_1'^T (X' = the next batch, W_1' = W_1 after this step's update), can be
 // computed by the kernel that produces W_1': this step's first-layer backward.  Then
 // W_1 is read once per step instead of twice (update + next forward: 8 bytes per
-// weight instead of 12).  The kernel keeps the forward's units and schedule exactly
-// (tile = learner j x 128 outputs, chunk = 64 inputs; stream-K or cluster split-K with
-// the same split, the same 4 MMAs per chunk and the same every-kSegChunks promotion),
-// so Z_1' is bit-identical to what k_tc_forward computes from the stored W_1'.  Per
-// chunk:
+// weight instead of 12).  The kernel keeps the forward's work items and arithmetic
+// exactly (tile = learner j x 128 outputs, chunk = 64 inputs; the same dynamic items
+// and tail pieces, or cluster split-K with the same split; the same 4 MMAs per chunk,
+// the same every-kSegChunks promotion from the item's first chunk, the same piece
+// order), so Z_1' is bit-identical to what k_tc_forward computes from the stored W_1'.
+// Per chunk:
 //   dW[o][i]  = sum_b dZ_1[b][o] X[b][i]      M = 128 outputs, N = 64 inputs, K = Bn
 //                                             (dZ tile and X tile both MN-major)
 //   W[o][i]  -= lr dW[o][i]                   fp32, in the shared-memory W tile, which is
@@ -1253,39 +1450,43 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
 //                                             the thread that owns output row o
 // and the tile epilogue writes H_1' = relu(Z' + b_1) (b_1 already updated by the layer
 // above).  Warps 0-7 own the accumulator rows as in the forward (row 32*(w%4) + lane,
-// input half w/4) and do the update, the bf16 conversion and the drains; warp 8 loads
-// W tiles, warp 9 issues the MMAs (the dW MMAs of chunk i before the forward MMAs of
-// chunk i-1, so the update of one chunk overlaps the dW of the next), warp 10 loads
-// the batch tiles (X and X' rows of the chunk) and publishes a split tile's partial,
-// warp 11 stores updated W tiles and frees their slots, warp 12 loads the dZ tile of
-// each tile visited.  A CTA visits few tiles (one in cluster mode, a handful in
-// stream-K mode), so the dZ tile has one buffer and the shared memory goes to a
-// five-deep weight ring.
+// input half w/4) and do the update, the bf16 conversion and the drains; warp 8 claims
+// the work items and loads W tiles, warp 9 issues the MMAs (the dW MMAs of chunk i
+// before the forward MMAs of chunk i-1, so the update of one chunk overlaps the dW of
+// the next), warp 10 loads the batch tiles (X and X' rows of the chunk), warp 11
+// stores updated W tiles and frees their slots, warp 12 loads the dZ tile of each
+// item (two buffers when shared memory allows, so the next item's is loaded ahead).
 constexpr int kUfConv = 256;
 constexpr int kUfThreads = kUfConv + 160;
-constexpr int kUfZBufs = 1;     // dZ tile buffers
 // TMEM columns: Z'^T accumulators at 0 and 64, bf16 A tiles at 128 and 160, dW
 // accumulators at 256 and 320.
 constexpr uint32_t kUfTmemCols = 512, kUfTmemA = 128, kUfTmemDW = 256;
 
-// Layout: W ring | dZ tile(s) ([Bn][128] bf16, two boxes each) | batch ring (X box, X'
+// Layout: W ring | dZ tiles ([Bn][128] bf16, two boxes each) | batch ring (X box, X'
 // box per chunk) | barriers.
+// nz: dZ tile buffers, two in dynamic mode when shared memory allows (the next item's
+// tile loads while this one's is in use), one in cluster mode (one item per CTA).
 __host__ __device__ constexpr int uf_wring(int Bn) { return (void)Bn, 5; }
+__host__ __device__ constexpr int uf_zbufs(int Bn, bool dyn) { return dyn && Bn <= 32 ? 2 : 1; }
 __host__ __device__ constexpr int uf_z_off(int Bn) { return uf_wring(Bn) * kFwdWf32; }
-__host__ __device__ constexpr int uf_h_off(int Bn) { return uf_z_off(Bn) + kUfZBufs * 2 * Bn * 128; }
-__host__ __device__ constexpr int uf_hring(int Bn) {
-  return (kFwdSmemMax - 1024 - 512 - uf_h_off(Bn)) / (2 * Bn * 128) < kFwdHRingMax
-             ? (kFwdSmemMax - 1024 - 512 - uf_h_off(Bn)) / (2 * Bn * 128)
+__host__ __device__ constexpr int uf_h_off(int Bn, int nz) { return uf_z_off(Bn) + nz * 2 * Bn * 128; }
+__host__ __device__ constexpr int uf_hring(int Bn, int nz) {
+  return (kFwdSmemMax - 1024 - kBarBytes - uf_h_off(Bn, nz)) / (2 * Bn * 128) < kFwdHRingMax
+             ? (kFwdSmemMax - 1024 - kBarBytes - uf_h_off(Bn, nz)) / (2 * Bn * 128)
              : kFwdHRingMax;
 }
-__host__ __device__ constexpr int uf_bar_off(int Bn) { return uf_h_off(Bn) + uf_hring(Bn) * 2 * Bn * 128; }
-__host__ __device__ constexpr int uf_smem(int Bn) { return uf_bar_off(Bn) + 512 + 1024; }
+__host__ __device__ constexpr int uf_bar_off(int Bn, int nz) {
+  return uf_h_off(Bn, nz) + uf_hring(Bn, nz) * 2 * Bn * 128;
+}
+__host__ __device__ constexpr int uf_smem(int Bn, int nz) { return uf_bar_off(Bn, nz) + kBarBytes + 1024; }
 // (the cluster split-K partial [128][Bn] fp32 is staged in the batch ring: hring >= 2)
-static_assert(uf_hring(64) >= 3 && uf_hring(48) >= 4 && uf_hring(32) >= 6 && uf_hring(16) == 8 &&
-                  uf_smem(64) <= kFwdSmemMax && uf_smem(48) <= kFwdSmemMax &&
-                  uf_smem(32) <= kFwdSmemMax && uf_smem(16) <= kFwdSmemMax,
+static_assert(uf_hring(64, 1) >= 3 && uf_hring(48, 1) >= 4 && uf_hring(32, 1) >= 7 &&
+                  uf_hring(32, 2) >= 6 && uf_hring(16, 2) == 8 && uf_smem(64, 1) <= kFwdSmemMax &&
+                  uf_smem(48, 1) <= kFwdSmemMax && uf_smem(32, 2) <= kFwdSmemMax &&
+                  uf_smem(16, 2) <= kFwdSmemMax,
               "update+forward shared-memory plan");
 
+template <bool kDyn>
 __global__ void __launch_bounds__(kUfThreads, 1)
     k_tc_update_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_hc,
                         const __grid_constant__ CUtensorMap tm_hn, const __grid_constant__ CUtensorMap tm_dz,
@@ -1293,25 +1494,22 @@ __global__ void __launch_bounds__(kUfThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = blockIdx.x, G = gridDim.x;
+  const int g = blockIdx.x;
   const int nk = (a.in + 63) / 64;
-  const int U = a.n_tiles * nk;
-  const int cq = a.cq > 1 ? a.cq : 1, part = g % cq;
-  const int u0 = cq > 1 ? (g / cq) * nk + part * nk / cq : unit_begin(g, U, G);
-  const int u1 = cq > 1 ? (g / cq) * nk + (part + 1) * nk / cq : unit_begin(g + 1, U, G);
-  const int n_local = u1 - u0;
-  const int nw = uf_wring(a.Bn), nh = uf_hring(a.Bn);
+  constexpr bool dyn = kDyn;
+  const int cq = kDyn ? 1 : a.cq, part = g % cq;
+  const int n_items = a.n_whole + (a.n_tiles - a.n_whole) * a.np_tail;
+  const int nz = uf_zbufs(a.Bn, dyn), nw = uf_wring(a.Bn), nh = uf_hring(a.Bn, nz);
   const int tbytes = a.Bn * 128;                            // one [Bn][64] bf16 box
-  const int tile0 = u0 / nk, c0 = u0 - tile0 * nk;
   uint8_t* z_base = smem + uf_z_off(a.Bn);
-  uint8_t* h_base = smem + uf_h_off(a.Bn);
-  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + uf_bar_off(a.Bn));
+  uint8_t* h_base = smem + uf_h_off(a.Bn, nz);
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + uf_bar_off(a.Bn, nz));
   uint64_t* wempty = wfull + kFwdWRingMax;   // W tile stored back (the TMA has read it)
   uint64_t* upd = wempty + kFwdWRingMax;     // W tile updated in shared memory
   uint64_t* hfull = upd + kFwdWRingMax;
   uint64_t* hempty = hfull + kFwdHRingMax;   // X and X' boxes consumed by both MMAs
-  uint64_t* zfull = hempty + kFwdHRingMax;   // [kUfZBufs <= 2]
-  uint64_t* zempty = zfull + 2;              // [..] dZ tile consumed by the tile's dW MMAs
+  uint64_t* zfull = hempty + kFwdHRingMax;   // [2]
+  uint64_t* zempty = zfull + 2;              // [2] dZ tile consumed by the item's dW MMAs
   uint64_t* dwdone = zempty + 2;             // [2] dW of the chunk complete
   uint64_t* dwfree = dwdone + 2;             // [2] dW read by the update
   uint64_t* conv = dwfree + 2;               // [2] A tile written to TMEM
@@ -1320,11 +1518,15 @@ __global__ void __launch_bounds__(kUfThreads, 1)
   uint64_t* accr = accf + 2;                 // [2] accumulator segment drained
   uint64_t* gbar = accr + 2;
   uint64_t* done = gbar + 1;
-  uint64_t* pready = done + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pready + 1);
+  ItemQueue queue{done + 1, done + 1 + kQueue, nullptr};
+  queue.items = reinterpret_cast<int*>(done + 1 + 2 * kQueue);
+  int* last_flag = queue.items + kQueue;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(last_flag + 1);
   auto wf = [&](int s) { return smem + s * kFwdWf32; };
   auto zb = [&](int s) { return z_base + s * 2 * tbytes; };
   auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
+  const FwdItem cl_item{g / cq, part * nk / cq, (part + 1) * nk / cq, 0, 1};
+  constexpr int kConsumers = 4 + kUfConv / 32;   // MMA, batch, store, dZ and converter warps
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kFwdWRingMax; ++s) {
@@ -1346,9 +1548,13 @@ __global__ void __launch_bounds__(kUfThreads, 1)
       mbar_init(&accf[b], 1);
       mbar_init(&accr[b], kUfConv);
     }
+    if (dyn)
+      for (int q = 0; q < kQueue; ++q) {
+        mbar_init(&queue.full[q], 1);
+        mbar_init(&queue.empty[q], kConsumers);
+      }
     mbar_init(gbar, kUfConv);
     mbar_init(done, 1);
-    mbar_init(pready, kUfConv / 32);
     fence_barrier_init();
   }
   if (warp == 9) {
@@ -1361,169 +1567,212 @@ __global__ void __launch_bounds__(kUfThreads, 1)
   const uint32_t tmem = *tmem_slot;
   grid_dep_wait();                       // dZ_1 and b_1 of the layer above are visible
 
+  auto next_item = [&](int k, FwdItem& f) -> bool {
+    if (!dyn) {
+      f = cl_item;
+      return k == 0;
+    }
+    const int it = queue.take(k, lane, a.err);
+    if (it < 0) return false;
+    f = fwd_item(a, nk, it);
+    return true;
+  };
+  // (the batch and dZ tiles are re-read for every output tile: kept in L2 ahead of
+  // the streamed W)
+  const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
+
   if (warp == 8) {
     if (lane == 0) {
+      // claim (dynamic), announce, and stream the weight tiles
       tma_prefetch_desc(&tm_w);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
-      int issued = 0, tau = tile0, c = c0;
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-        const int s = i % nw;
-        if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
-        tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j, stream);
-        tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j, stream);
-        issued = i + 1;
-        if (++c == nk) { c = 0; ++tau; }
+      int i = 0, issued = 0;
+      bool ok = true;
+      int next = dyn ? atomicAdd(a.dyn, 1) : 0;
+      for (int k = 0; ok; ++k) {
+        FwdItem f;
+        if (dyn) {
+          const int it = next < n_items ? next : -1;
+          if (!queue.put(k, it, a.err) || it < 0) break;
+          next = atomicAdd(a.dyn, 1);           // the next claim, hidden behind these loads
+          f = fwd_item(a, nk, it);
+        } else {
+          if (k > 0) break;
+          f = cl_item;
+        }
+        const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
+          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j, stream);
+          tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j, stream);
+          issued = i + 1;
+        }
       }
-      for (int i = issued - nw > 0 ? issued - nw : 0; i < issued; ++i)
-        mbar_wait(&wfull[i % nw], (i / nw) & 1, a.err);
+      for (int u = issued - nw > 0 ? issued - nw : 0; u < issued; ++u)
+        mbar_wait(&wfull[u % nw], (u / nw) & 1, a.err);
     }
     if (cq > 1) {
       cluster_sync_all();
       cluster_sync_all();
     }
   } else if (warp == 10) {
+    // the X and X' boxes of each chunk
     if (lane == 0) {
-      // The X and X' boxes of each chunk; publishes this CTA's partial of a split first
-      // tile (see the forward).
       tma_prefetch_desc(&tm_hc);
       tma_prefetch_desc(&tm_hn);
-      bool publish = cq == 1 && c0 != 0 && n_local > 0;
-      int issued = 0, tau = tile0, c = c0;
-      // (the batch and dZ tiles are re-read for every output tile: kept in L2 ahead of
-      // the streamed W)
-      const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.o_tiles;
-        if (publish && mbar_test(pready, 0)) {
-          red_release_add(a.counters + tile0, 1);
-          publish = false;
-        }
-        const int s = i % nh;
-        if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&hfull[s], 2 * tbytes);
-        tma_load_3d_hint(hb(s), &tm_hc, &hfull[s], c * 64, a.hc_row0, j, keep);
-        tma_load_3d_hint(hb(s) + tbytes, &tm_hn, &hfull[s], c * 64, a.x_row0, j, keep);
-        issued = i + 1;
-        if (++c == nk) { c = 0; ++tau; }
-      }
-      for (int i = issued - nh > 0 ? issued - nh : 0; i < issued; ++i)
-        mbar_wait(&hfull[i % nh], (i / nh) & 1, a.err);
-      if (publish && mbar_wait(pready, 0, a.err)) red_release_add(a.counters + tile0, 1);
     }
+    int i = 0, issued = 0;
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        const int j = f.tau / a.o_tiles;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nh;
+          if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&hfull[s], 2 * tbytes);
+          tma_load_3d_hint(hb(s), &tm_hc, &hfull[s], c * 64, a.hc_row0, j, keep);
+          tma_load_3d_hint(hb(s) + tbytes, &tm_hn, &hfull[s], c * 64, a.x_row0, j, keep);
+          issued = i + 1;
+        }
+      }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0)
+      for (int u = issued - nh > 0 ? issued - nh : 0; u < issued; ++u)
+        mbar_wait(&hfull[u % nh], (u / nh) & 1, a.err);
     if (cq > 1) {
       cluster_sync_all();
       cluster_sync_all();
     }
   } else if (warp == 12) {
-    if (lane == 0 && n_local > 0) {
-      // The dZ tile (128 outputs x Bn) of each tile this CTA visits.
-      tma_prefetch_desc(&tm_dz);
-      const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
-      const int n_visits = (u1 - 1) / nk - tile0 + 1;
-      int zissued = 0;
-      for (int v = 0; v < n_visits; ++v) {
-        const int tau = tile0 + v, j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-        const int zs = v % kUfZBufs;
-        if (v >= kUfZBufs && !mbar_wait(&zempty[zs], ((v / kUfZBufs) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&zfull[zs], 2 * tbytes);
-        tma_load_3d_hint(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j, keep);
-        tma_load_3d_hint(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j, keep);
-        zissued = v + 1;
+    // the dZ tile (128 outputs x Bn) of each item
+    if (lane == 0) tma_prefetch_desc(&tm_dz);
+    int zissued = 0;
+    bool ok = true;
+    FwdItem f;
+    for (int v = 0; ok && next_item(v, f); ++v) {
+      if (lane == 0) {
+        const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
+        const int zs = v % nz;
+        if (v >= nz && !mbar_wait(&zempty[zs], ((v / nz) - 1) & 1, a.err)) {
+          ok = false;
+        } else {
+          mbar_arrive_expect_tx(&zfull[zs], 2 * tbytes);
+          tma_load_3d_hint(zb(zs), &tm_dz, &zfull[zs], ot * 128, 0, j, keep);
+          tma_load_3d_hint(zb(zs) + tbytes, &tm_dz, &zfull[zs], ot * 128 + 64, 0, j, keep);
+          zissued = v + 1;
+        }
       }
-      for (int v = zissued - kUfZBufs > 0 ? zissued - kUfZBufs : 0; v < zissued; ++v)
-        mbar_wait(&zfull[v % kUfZBufs], (v / kUfZBufs) & 1, a.err);
+      ok = __all_sync(0xffffffffu, ok);
     }
+    if (lane == 0)
+      for (int v = zissued - nz > 0 ? zissued - nz : 0; v < zissued; ++v)
+        mbar_wait(&zfull[v % nz], (v / nz) & 1, a.err);
     if (cq > 1) {
       cluster_sync_all();
       cluster_sync_all();
     }
   } else if (warp == 11) {
-    if (lane == 0) {
-      // Store each updated W tile; its slot is released once the TMA has read it.  In
-      // cluster mode (a short layer) each slot is released as soon as its own store has
-      // been read; in stream-K mode one store behind, two in flight (releasing at once
-      // let the fast SMs take bandwidth from the slow ones, whose end sets the kernel's).
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
-      int tau = tile0, c = c0, stored = 0, released = 0;
-      for (int i = 0; i < n_local; ++i) {
-        const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-        const int s = i % nw;
-        if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
-        tma_store_3d_hint(&tm_w, wf(s), c * 64, ot * 128, j, stream);
-        tma_store_3d_hint(&tm_w, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
-        tma_store_commit();
-        stored = i + 1;
-        if (cq > 1) {
-          tma_store_wait_read_all();
-          mbar_arrive(&wempty[s]);
-          released = stored;
-        } else if (i > 0) {
-          tma_store_wait_read_1();
-          mbar_arrive(&wempty[(i - 1) % nw]);
-          released = i;
+    // Store each updated W tile; its slot is released once the TMA has read it.  In
+    // cluster mode (a short layer) each slot is released as soon as its own store has
+    // been read; otherwise one store behind, two in flight.
+    const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+    int i = 0, released = 0;
+    bool ok = true;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) { ok = false; break; }
+          tma_store_3d_hint(&tm_w, wf(s), c * 64, ot * 128, j, stream);
+          tma_store_3d_hint(&tm_w, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
+          tma_store_commit();
+          if (cq > 1) {
+            tma_store_wait_read_all();
+            mbar_arrive(&wempty[s]);
+            released = i + 1;
+          } else if (i > 0) {
+            tma_store_wait_read_1();
+            mbar_arrive(&wempty[(i - 1) % nw]);
+            released = i;
+          }
         }
-        if (++c == nk) { c = 0; ++tau; }
       }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
       tma_store_wait_read_all();   // (before the shared memory is released)
-      if (stored > released) mbar_arrive(&wempty[(stored - 1) % nw]);
+      if (i > released) mbar_arrive(&wempty[(i - 1) % nw]);
     }
     if (cq > 1) {
       cluster_sync_all();
       cluster_sync_all();
     }
   } else if (warp == 9) {
-    if (lane == 0) {
-      const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
-      const uint32_t idesc_fw = umma_idesc_bf16(128, a.Bn);
-      const int kb = a.Bn / 16;
-      // Forward MMAs of chunk k into accumulator segment qq (first/last: of the segment).
-      auto fwd = [&](int k, bool first, bool last, int qq) -> bool {
-        const int ab = qq & 1, bb = k & 1, sh = k % nh;
-        if (first && qq >= 2 && !mbar_wait(&accr[ab], ((qq >> 1) - 1) & 1, a.err)) return false;
-        if (!mbar_wait(&conv[bb], (k >> 1) & 1, a.err)) return false;
-        tc_fence_after();
-        const uint32_t at = tmem + kUfTmemA + 32 * bb;
-        const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh) + tbytes));
-        const uint32_t d = tmem + 64 * ab;
+    const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
+    const uint32_t idesc_fw = umma_idesc_bf16(128, a.Bn);
+    const int kb = a.Bn / 16;
+    // Forward MMAs of chunk k into accumulator segment qq (first/last: of the segment).
+    auto fwd = [&](int k, bool first, bool last, int qq) -> bool {
+      const int ab = qq & 1, bb = k & 1, sh = k % nh;
+      if (first && qq >= 2 && !mbar_wait(&accr[ab], ((qq >> 1) - 1) & 1, a.err)) return false;
+      if (!mbar_wait(&conv[bb], (k >> 1) & 1, a.err)) return false;
+      tc_fence_after();
+      const uint32_t at = tmem + kUfTmemA + 32 * bb;
+      const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh) + tbytes));
+      const uint32_t d = tmem + 64 * ab;
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc_fw, (!first || kk > 0) ? 1u : 0u);
-        tc_commit(&hempty[sh]);
-        tc_commit(&afree[bb]);
-        if (last) tc_commit(&accf[ab]);
-        return true;
-      };
-      int c = c0, p = 0, q = -1, zv = -1;
-      int pend = -1, pend_q = 0;
-      bool pend_first = false, pend_last = false, ok = true;
-      for (int i = 0; i < n_local; ++i) {
-        const bool tlast = i == n_local - 1 || c == nk - 1;
-        const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
-        if (first) ++q;
-        const int sh = i % nh, bb = i & 1;
-        if (p == 0) {
-          ++zv;
-          if (!mbar_wait(&zfull[zv % kUfZBufs], (zv / kUfZBufs) & 1, a.err)) { ok = false; break; }
+      for (int kk = 0; kk < 4; ++kk)
+        tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc_fw, (!first || kk > 0) ? 1u : 0u);
+      tc_commit(&hempty[sh]);
+      tc_commit(&afree[bb]);
+      if (last) tc_commit(&accf[ab]);
+      return true;
+    };
+    int i = 0, q = -1;
+    int pend = -1, pend_q = 0;
+    bool pend_first = false, pend_last = false, ok = true;
+    FwdItem f;
+    for (int v = 0; ok && next_item(v, f); ++v) {
+      if (lane == 0) {
+        const int zs = v % nz;
+        // The pending forward (last chunk of the previous item) goes first if this
+        // item's dZ tile has not arrived yet, so that the converters can close that item.
+        if (pend >= 0 && !mbar_test(&zfull[zs], (v / nz) & 1)) {
+          if (!fwd(pend, pend_first, pend_last, pend_q)) ok = false;
+          pend = -1;
         }
-        if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
-        if (i >= 2 && !mbar_wait(&dwfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t zs = smem_u32(zb(zv % kUfZBufs)), hs = smem_u32(hb(sh));
-        for (int kk = 0; kk < kb; ++kk)
-          tc_mma_bf16(tmem + kUfTmemDW + 64 * bb, umma_desc_sw128_mn(zs + kk * 2048, tbytes),
-                      umma_desc_sw128_mn(hs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
-        tc_commit(&dwdone[bb]);
-        if (tlast) tc_commit(&zempty[zv % kUfZBufs]);
-        if (pend >= 0 && !fwd(pend, pend_first, pend_last, pend_q)) { ok = false; break; }
-        pend = i;
-        pend_first = first;
-        pend_last = last;
-        pend_q = q;
-        ++p;
-        if (++c == nk) { c = 0; p = 0; }
+        if (ok && !mbar_wait(&zfull[zs], (v / nz) & 1, a.err)) ok = false;
+        const uint32_t zsa = smem_u32(zb(zs));
+        for (int c = f.c_lo, p = 0; ok && c < f.c_hi; ++c, ++p, ++i) {
+          const bool tlast = c == f.c_hi - 1;
+          const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+          if (first) ++q;
+          const int sh = i % nh, bb = i & 1;
+          if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
+          if (i >= 2 && !mbar_wait(&dwfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t hs = smem_u32(hb(sh));
+          for (int kk = 0; kk < kb; ++kk)
+            tc_mma_bf16(tmem + kUfTmemDW + 64 * bb, umma_desc_sw128_mn(zsa + kk * 2048, tbytes),
+                        umma_desc_sw128_mn(hs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+          tc_commit(&dwdone[bb]);
+          if (tlast) tc_commit(&zempty[zs]);
+          if (pend >= 0 && !fwd(pend, pend_first, pend_last, pend_q)) { ok = false; break; }
+          pend = i;
+          pend_first = first;
+          pend_last = last;
+          pend_q = q;
+        }
       }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
       if (ok && pend >= 0) fwd(pend, pend_first, pend_last, pend_q);
       tc_commit(done);
       mbar_wait(done, 0, a.err);   // no MMA may be in flight at teardown
@@ -1563,55 +1812,18 @@ __global__ void __launch_bounds__(kUfThreads, 1)
       ++drained;
       return true;
     };
-    // As the forward's tile_end, hidden layer only: H_1'[j][b][o] = relu(Z' + b_1).
-    auto tile_end = [&](int tau, bool whole, float bias) -> bool {
+    // As the forward's hidden-layer epilogue: H_1'[j][b][o] = relu(Z' + b_1).  The
+    // cluster build loads the bias of its one tile up front (cl_bias); the dynamic build,
+    // short of registers, at the epilogue.
+    const int cl_o = (cl_item.tau % a.o_tiles) * 128 + r;
+    const float cl_bias = !kDyn && cl_o < a.out
+                              ? a.bias[static_cast<int64_t>(cl_item.tau / a.o_tiles) * a.ld + cl_o]
+                              : 0.f;
+    auto epilogue = [&](int tau) {
       const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-      if (!whole) {
-        if (tau * nk < u0) {
-          float* mine = a.part + (static_cast<int64_t>(g) * 128 + r) * a.Bn;
-#pragma unroll
-          for (int m = 0; m < 2; ++m) {
-            const int cb = (2 * m + gr) * 16;
-            if (cb < a.Bn) {
-#pragma unroll
-              for (int q = 0; q < 16; q += 4)
-                __stcg(reinterpret_cast<float4*>(mine + cb + q),
-                       make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
-                                   acc[16 * m + q + 3]));
-            }
-          }
-          __syncwarp();
-          if (lane == 0) mbar_arrive(pready);
-#pragma unroll
-          for (int q = 0; q < 32; ++q) acc[q] = 0.f;
-          return true;
-        }
-        const int g_last = cta_of((tau + 1) * nk - 1, U, G);
-        if (t == 0) {
-          const bool ok = spin_acquire_eq(a.counters + tau, g_last - g, a.err);
-          if (ok) a.counters[tau] = 0;
-        }
-        if (!gsync()) return false;
-        for (int gg = g + 1; gg <= g_last; ++gg) {
-          const float* src = a.part + (static_cast<int64_t>(gg) * 128 + r) * a.Bn;
-#pragma unroll
-          for (int m = 0; m < 2; ++m) {
-            const int cb = (2 * m + gr) * 16;
-            if (cb < a.Bn) {
-#pragma unroll
-              for (int q = 0; q < 16; q += 4) {
-                const float4 v = __ldcg(reinterpret_cast<const float4*>(src + cb + q));
-                acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v.x);
-                acc[16 * m + q + 1] = __fadd_rn(acc[16 * m + q + 1], v.y);
-                acc[16 * m + q + 2] = __fadd_rn(acc[16 * m + q + 2], v.z);
-                acc[16 * m + q + 3] = __fadd_rn(acc[16 * m + q + 3], v.w);
-              }
-            }
-          }
-        }
-      }
       const int o = ot * 128 + r;
       if (o < a.out) {
+        const float bias = kDyn ? a.bias[static_cast<int64_t>(j) * a.ld + o] : cl_bias;
 #pragma unroll
         for (int m = 0; m < 2; ++m) {
           const int cb = (2 * m + gr) * 16;
@@ -1623,93 +1835,86 @@ __global__ void __launch_bounds__(kUfThreads, 1)
                   __float2bfloat16_rn(fmaxf(__fadd_rn(acc[16 * m + q], bias), 0.f));
         }
       }
-#pragma unroll
-      for (int q = 0; q < 32; ++q) acc[q] = 0.f;
-      return true;
     };
-    bool ok = true;
-    int tau = tile0, c = c0, p = 0;
-    float tbias = 0.f;
-    int ep_tau = -1;
-    float ep_bias = 0.f;
-    for (int i = 0; i < n_local && ok; ++i) {
-      const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
-      const bool tlast = i == n_local - 1 || c == nk - 1;
-      if (p == 0) {
-        const int o = ot * 128 + r;
-        tbias = o < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + o] : 0.f;
-      }
-      const int sw = i % nw, bb = i & 1;
-      if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
-      if (!wait_warp(&dwdone[bb], (i >> 1) & 1, a.err)) { ok = false; break; }
-      tc_fence_after();
-      float d[32];
-      tmem_ld16(tbase + kUfTmemDW + 64 * bb + 32 * half, d);
-      tmem_ld16(tbase + kUfTmemDW + 64 * bb + 32 * half + 16, d + 16);
-      tmem_ld_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&dwfree[bb]);
-      // W[o][32*half + 4q ..] sits in 16-byte chunk q ^ (o % 8) of row o of box `half`
-      uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
-      uint32_t pk[16];
+    bool ok = true, have_ep = false;   // have_ep: cluster split-K, this CTA's part is done
+    int i = 0;
+    FwdItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      for (int c = f.c_lo, p = 0; c < f.c_hi && ok; ++c, ++p, ++i) {
+        const bool tlast = c == f.c_hi - 1;
+        const int sw = i % nw, bb = i & 1;
+        if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+        if (!wait_warp(&dwdone[bb], (i >> 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+        float d[32];
+        tmem_ld16(tbase + kUfTmemDW + 64 * bb + 32 * half, d);
+        tmem_ld16(tbase + kUfTmemDW + 64 * bb + 32 * half + 16, d + 16);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&dwfree[bb]);
+        // W[o][32*half + 4q ..] sits in 16-byte chunk q ^ (o % 8) of row o of box `half`
+        uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
+        uint32_t pk[16];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        float4* pw = reinterpret_cast<float4*>(src + ((q ^ (row & 7)) << 4));
-        float4 x = *pw;
-        x.x = __fsub_rn(x.x, __fmul_rn(a.lr, d[4 * q]));
-        x.y = __fsub_rn(x.y, __fmul_rn(a.lr, d[4 * q + 1]));
-        x.z = __fsub_rn(x.z, __fmul_rn(a.lr, d[4 * q + 2]));
-        x.w = __fsub_rn(x.w, __fmul_rn(a.lr, d[4 * q + 3]));
-        *pw = x;
-        pk[2 * q] = pack_bf16x2(x.x, x.y);
-        pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&upd[sw]);
-      if (i >= 2 && !wait_warp(&afree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
-      tc_fence_after();
-      tmem_st16(tbase + kUfTmemA + 32 * bb + 16 * half, pk);
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&conv[bb]);
-      if (p % kSegChunks == 0) ++qc;
-      if (tlast) {
-        while (ok && drained <= qc)
-          if (!drain()) ok = false;
-        if (ok && cq > 1) {
-          ep_tau = tau;
-          ep_bias = tbias;
-          if (part != 0) {
-            // the batch ring is idle once the last segment is drained
-            float* red = reinterpret_cast<float*>(h_base) + r * a.Bn;
+        for (int q = 0; q < 8; ++q) {
+          float4* pw = reinterpret_cast<float4*>(src + ((q ^ (row & 7)) << 4));
+          float4 x = *pw;
+          x.x = __fsub_rn(x.x, __fmul_rn(a.lr, d[4 * q]));
+          x.y = __fsub_rn(x.y, __fmul_rn(a.lr, d[4 * q + 1]));
+          x.z = __fsub_rn(x.z, __fmul_rn(a.lr, d[4 * q + 2]));
+          x.w = __fsub_rn(x.w, __fmul_rn(a.lr, d[4 * q + 3]));
+          *pw = x;
+          pk[2 * q] = pack_bf16x2(x.x, x.y);
+          pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&upd[sw]);
+        if (i >= 2 && !wait_warp(&afree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+        tmem_st16(tbase + kUfTmemA + 32 * bb + 16 * half, pk);
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&conv[bb]);
+        if (p % kSegChunks == 0) ++qc;
+        if (tlast) {
+          while (ok && drained <= qc)
+            if (!drain()) ok = false;
+          if (!ok) break;
+          if (!dyn) {
+            have_ep = true;
+            if (part != 0) {
+              // the batch ring is idle once the last segment is drained
+              float* red = reinterpret_cast<float*>(h_base) + r * a.Bn;
 #pragma unroll
-            for (int m = 0; m < 2; ++m) {
-              const int cb = (2 * m + gr) * 16;
-              if (cb < a.Bn) {
+              for (int m = 0; m < 2; ++m) {
+                const int cb = (2 * m + gr) * 16;
+                if (cb < a.Bn) {
 #pragma unroll
-                for (int q = 0; q < 16; q += 4)
-                  *reinterpret_cast<float4*>(red + cb + q) =
-                      make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
-                                  acc[16 * m + q + 3]);
+                  for (int q = 0; q < 16; q += 4)
+                    *reinterpret_cast<float4*>(red + cb + q) =
+                        make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2],
+                                    acc[16 * m + q + 3]);
+                }
               }
             }
+          } else {
+            const bool fin = f.np == 1 || piece_end(a, f, t, r, gr, acc, gsync, last_flag, ok);
+            if (ok && fin) epilogue(f.tau);
+#pragma unroll
+            for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+            ok = __all_sync(0xffffffffu, ok);
           }
-        } else if (ok) {
-          const bool whole = (tau != tile0 || c0 == 0) && c == nk - 1;
-          ok = __all_sync(0xffffffffu, tile_end(tau, whole, tbias));
+        } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
+          if (!drain()) ok = false;
         }
-      } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
-        if (!drain()) ok = false;
       }
-      ++p;
-      if (++c == nk) { c = 0; p = 0; ++tau; }
     }
     if (cq > 1) {
       cluster_sync_all();
-      if (part == 0 && __all_sync(0xffffffffu, ok && ep_tau >= 0)) {
+      if (part == 0 && __all_sync(0xffffffffu, ok && have_ep)) {
         for (int rk = 1; rk < cq; ++rk) {
           const float* red = reinterpret_cast<const float*>(h_base) + r * a.Bn;
 #pragma unroll
@@ -1727,7 +1932,7 @@ __global__ void __launch_bounds__(kUfThreads, 1)
             }
           }
         }
-        tile_end(ep_tau, true, ep_bias);
+        epilogue(cl_item.tau);
       }
       cluster_sync_all();
     }
@@ -1738,6 +1943,13 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kUfTmemCols);
+  }
+  if (dyn && threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(a.dyn + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+      a.dyn[0] = 0;
+      a.dyn[1] = 0;
+    }
   }
 }
 
@@ -1824,34 +2036,40 @@ int tc_fwd_smem_bytes() { return kFwdSmemMax; }
 int tc_bwd_smem_bytes() { return kBwdSmemMax; }
 
 cudaError_t tc_configure() {
-  cudaError_t e = cudaFuncSetAttribute(k_tc_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(k_tc_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        kFwdSmemMax);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tc_forward<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFwdSmemMax);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tc_update_forward<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kFwdSmemMax);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_update, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_tc_update_forward, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(k_tc_update_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               kFwdSmemMax);
 }
 
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s) {
   (void)P;
-  // Cooperative: the finisher of a split tile waits for the other contributors,
-  // so every CTA of the grid must be resident at once (the launch fails otherwise).
-  // (Cluster split-K needs no cooperative launch: no cluster waits on another.)
-  return launch_pdl(k_tc_forward, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s,
-                    a.cq <= 1, a.cq > 1 ? a.cq : 1, w_fwd, h_in, a);
+  // No CTA waits for another (dynamic items; cluster split-K reduces inside a cluster),
+  // so an ordinary launch.
+  if (a.cq > 1)
+    return launch_pdl(k_tc_forward<false>, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s,
+                      false, a.cq, w_fwd, h_in, a);
+  return launch_pdl(k_tc_forward<true>, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s,
+                    false, 1, w_fwd, h_in, a);
 }
 
 cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
                                const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s) {
   (void)P;
-  // Cooperative for the same reason as the forward (split dX tiles); without dX no CTA
-  // waits on another, and the cooperative attribute costs ~2 us per launch.
-  return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s,
-                    a.has_dx != 0, 1, w_bwd, h_in, dz, a);
+  // dynamic work items, no CTA waits for another: an ordinary launch
+  return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
+                    w_bwd, h_in, dz, a);
 }
 
 cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
@@ -1864,9 +2082,12 @@ cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
 cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_cur,
                                      const CUtensorMap& x_next, const CUtensorMap& dz,
                                      const TcFwdArgs& a, cudaStream_t s) {
-  // cooperative in stream-K mode, as the forward
-  return launch_pdl(k_tc_update_forward, dim3(a.ctas), dim3(kUfThreads), uf_smem(a.Bn), s,
-                    a.cq <= 1, a.cq > 1 ? a.cq : 1, w_fwd, h_cur, x_next, dz, a);
+  // an ordinary launch, as the forward
+  if (a.cq > 1)
+    return launch_pdl(k_tc_update_forward<false>, dim3(a.ctas), dim3(kUfThreads),
+                      uf_smem(a.Bn, uf_zbufs(a.Bn, false)), s, false, a.cq, w_fwd, h_cur, x_next, dz, a);
+  return launch_pdl(k_tc_update_forward<true>, dim3(a.ctas), dim3(kUfThreads),
+                    uf_smem(a.Bn, uf_zbufs(a.Bn, true)), s, false, 1, w_fwd, h_cur, x_next, dz, a);
 }
 
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,

@@ -11,8 +11,8 @@ norms).  A ReLU decision on a pre-activation within rounding distance of zero ca
 either way under two valid fp32 accumulation orders, which swaps one sample's term
 in one row of the update; so an update row beyond the bound is accepted only where
 such a flip is provable (the oracle's pre-activation in that row is below the
-worst-case difference of two fp32 summation orders), and every accepted row is
-counted and reported (none at the 16-learner workload, at most one row in a
+worst-case difference of two fp32 summation orders plus two bf16 rounding decisions
+of the inputs), and every accepted row is counted and reported (none at the 16-learner workload, at most one row in a
 thousand at the full-size workloads).
 
 Whole rounds end to end (no teacher forcing): such flips compound over the round's
@@ -90,11 +90,15 @@ def make_oracle(w, ha, X, y, params, learners=None, mode=None):
 # A ReLU decision on a pre-activation within rounding distance of zero can go either
 # way in two correct implementations; it swaps one sample's term in one row of that
 # layer's update.  Two fp32 sums of the same K products in different orders differ by
-# at most 2 K u sum_k |h_k w_k| (u = 2^-24), so such a flip is possible only where the
-# exact pre-activation is smaller than that.  An update row beyond its bound is
-# accepted only if some sample's pre-activation in that row is (the "flip ratio"
-# |z| / (2 K u sum |h w|) is at most 1), and every accepted row is counted.
+# at most 2 K u sum_k |h_k w_k| (u = 2^-24); and the bf16 inputs h_k of the two can
+# differ where an earlier layer's value sat on a rounding boundary, each such decision
+# moving z by at most 2^-8 |h_k w_k|.  So a flip is possible only where the exact
+# pre-activation is below 2 K u sum |h w| + 2 * 2^-8 max |h w| (the order bound plus two
+# input decisions).  An update row beyond its bound is accepted only if some sample's
+# pre-activation in that row is (the "flip ratio" |z| / that bound is at most 1), and
+# every accepted row is counted.
 U32 = 2.0 ** -24
+U_BF16 = 2.0 ** -8
 
 
 def _flip_rows(o, k, L, bad, before):
@@ -119,7 +123,8 @@ def _flip_rows(o, k, L, bad, before):
         W = oracle.bf16_round(before[2 * layer][jj].astype(np.float32)).astype(np.float64)
         K = W.shape[1]
         for r in flagged:
-            bound = 2.0 * K * U32 * (np.abs(H) @ np.abs(W[r])) + 1e-300
+            prod = np.abs(H) * np.abs(W[r])                    # [B, K]
+            bound = 2.0 * K * U32 * prod.sum(axis=1) + 2.0 * U_BF16 * prod.max(axis=1) + 1e-300
             ratio = float(np.min(np.abs(z[:, r]) / bound))
             ratios.append(ratio)
             if ratio > 1.0:
@@ -201,6 +206,19 @@ HEAD_C13 = configs.Workload("mlp_bf16_c13", P=4, S=2, K1=1, K2=2, rounds=1, dims
 HEAD_F128 = configs.Workload("mlp_bf16_head_f128", P=20, S=4, K1=3, K2=2, rounds=1,
                              dims=(256, 320, 10), precision="bf16", N=120, B=24, lr=0.05,
                              sigma_mu=0.1, init="he")
+# Dynamic work items with both whole tiles and tail tiles split into pieces (3136
+# inputs = 49 chunks: pieces of 48 and 1 chunk), 32 learners in clusters of 4: the
+# pieces of a tile are summed in piece order by whichever CTA completes the tile.
+FUSE_PIECES = configs.Workload("mlp_bf16_pieces", P=32, S=4, K1=3, K2=2, rounds=1,
+                               dims=(3136, 1024, 10), precision="bf16", N=160, B=32, lr=0.05,
+                               sigma_mu=0.1, init="he")
+# The backward's pieces: the second layer's dX sums over 3136 outputs (49 chunks), so
+# its tiles are split and their dX partials added in piece order.
+BWD_PIECES = configs.Workload("mlp_bf16_bwd_pieces", P=32, S=4, K1=2, K2=2, rounds=1,
+                              dims=(256, 256, 3136, 10), precision="bf16", N=128, B=32, lr=0.05,
+                              sigma_mu=0.1, init="he")
+
+
 SMALL_FP32 = configs.Workload("tiny_mlp_fp32", P=4, S=2, K1=2, K2=2, rounds=1,
                               dims=(100, 37, 10), precision="fp32", N=40, B=7, lr=0.05,
                               sigma_mu=0.1, init="he")
@@ -212,7 +230,8 @@ SMALL_FP32 = configs.Workload("tiny_mlp_fp32", P=4, S=2, K1=2, K2=2, rounds=1,
 # epilogue (RAGGED_BF16: 13 classes over a 200-wide ragged input; WIDE_SOFTMAX_BF16),
 # and the standalone CE kernel (MANY_CLASSES_BF16: 300 classes over 3 tiles).
 STEP_CASES = [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16, HEAD_C13,
-              WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16, configs.MLP512_P16]
+              WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16, configs.MLP512_P16, FUSE_PIECES,
+              BWD_PIECES]
 
 
 @pytest.mark.parametrize("w", STEP_CASES, ids=lambda w: w.name)
@@ -236,7 +255,7 @@ def test_one_step_from_distinct_learners(w):
 
 @pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16,
                                HEAD_C13, WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16,
-                               HEAD_F128], ids=lambda w: w.name)
+                               HEAD_F128, FUSE_PIECES, BWD_PIECES], ids=lambda w: w.name)
 def test_full_run_against_oracle(w):
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
@@ -294,7 +313,7 @@ def _fused_steps(w):
 
 
 @pytest.mark.parametrize("w", [SMALL_BF16, configs.MLP512_P16.replace(N=512), FUSE_STREAMK,
-                               FUSE_THREE], ids=lambda w: w.name)
+                               FUSE_THREE, FUSE_PIECES, BWD_PIECES], ids=lambda w: w.name)
 def test_fused_next_forward_equals_steps(w):
     ha1, X, y = setup(w, perturb=(0.01, 0.01))
     ha2, _, _ = setup(w, perturb=(0.01, 0.01))

@@ -24,8 +24,9 @@ pytestmark = pytest.mark.gpu
 SMALL_BF16 = configs.Workload("tiny_mlp_bf16", P=4, S=2, K1=2, K2=2, rounds=1,
                               dims=(256, 192, 10), precision="bf16", N=96, B=48, lr=0.05,
                               sigma_mu=0.1, init="he")
-# 3072-2048-2048-10 with 16 learners: ~23 MiB of the 32 MiB array
-LARGER_BF16 = configs.MLP2048_P64.replace(name="mlp2048_P16_static", P=16, N=256)
+# 3072-2048-2048-10 with 8 learners (one cluster): ~24 MiB of the 32 MiB array,
+# with split-tile partials and counters in use
+LARGER_BF16 = configs.MLP2048_P64.replace(name="mlp2048_P8_static", P=8, N=256)
 
 
 def _static_matches_bound(lib, w):
