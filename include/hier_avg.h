@@ -98,7 +98,9 @@ void hier_avg_destroy(hier_avg* h);
  * ([d_{l+1}, d_l] row-major), offsets[2l+1] = start of b_{l+1} ([d_{l+1}]). */
 int hier_avg_param_layout(const hier_avg* h, int64_t* D, int64_t* ld, int64_t* offsets);
 
-/* Bytes of device workspace hier_avg_bind needs. */
+/* Bytes of device workspace hier_avg_bind needs: a step's scratch and, for the bf16
+ * path with S > 1, the cluster means [P / S, ld] fp32 that hier_avg_round's local
+ * averages write. */
 int hier_avg_workspace_bytes(const hier_avg* h, int64_t* bytes);
 
 /* Attach device memory (all borrowed, caller-owned) and the stream:
@@ -128,7 +130,11 @@ int hier_avg_global_average(hier_avg* h);
 
 /* One global round of Algorithm 1: K2 x (K1 x step, local average), then the
  * global average; the last local average is fused with the global one
- * (bit-identical to doing them in turn).  Within the round, a step whose successor
+ * (bit-identical to doing them in turn).  The other local averages write each
+ * cluster's mean once, into the workspace, and the step that follows reads every
+ * learner's parameters from its cluster's mean and writes the learner's row: the
+ * values are those of the full write-back, and when the round returns every row of
+ * params_dev holds its learner's parameters.  Within the round, a step whose successor
  * starts no local block and reads a contiguous batch also computes that successor's
  * first-layer output from the weights it has just updated (bf16 path, two or more
  * layers), so W_1 is read once per step; the results are those of calling
@@ -180,9 +186,10 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host,
  *     behind; calls whose work overlaps on the GPU (other streams, other
  *     threads) race on it.  After a call, later hier_avg_step / round calls of
  *     the same handle also use the array until hier_avg_bind is called again.
- * Errors: HA_ENOMEM (with a message naming both sizes) when the configuration
- * needs more than 32 MiB of scratch (hier_avg_workspace_bytes), HA_EINVAL for
- * NULL or misaligned buffers or N < 1, HA_ECUDA. */
+ * Errors: HA_ENOMEM (with a message naming both sizes) when one step of the
+ * configuration needs more than 32 MiB of scratch (hier_avg_workspace_bytes less
+ * the cluster means, which only rounds use; a round of a handle bound this way
+ * averages in place), HA_EINVAL for NULL or misaligned buffers or N < 1, HA_ECUDA. */
 int hier_avg_step_static(hier_avg* h, float* params_dev, const void* X_dev,
                          const int32_t* y_dev, int64_t N, void* stream);
 

@@ -103,8 +103,10 @@ __device__ __forceinline__ void head_body(const HeadArgs& a, uint8_t* smem, int 
   int* ys = reinterpret_cast<int*>(bls + kHeadMaxC);            // [64]      labels
   __nv_bfloat16* gqa = reinterpret_cast<__nv_bfloat16*>(ys + 64);           // [64][kGA]  g_q
   __nv_bfloat16* gqt = gqa + 64 * kGA;                                      // [16][kGT]  g_q^T
-  float* W = a.W + static_cast<int64_t>(j) * a.ld;
+  float* W = a.W + static_cast<int64_t>(j) * a.ld;                 // written
   float* bL = a.bias + static_cast<int64_t>(j) * a.ld;
+  const int64_t src_row = static_cast<int64_t>(j / a.src_div) * a.ld; // read
+  const float* Wr = a.W_src + src_row;
 
   // ---- 1. stage the slice (padding rows zero) and the labels, form the partial logits
   const int vpr = kc / 8;                                       // 16-byte vectors per H row
@@ -118,12 +120,12 @@ __device__ __forceinline__ void head_body(const HeadArgs& a, uint8_t* smem, int 
   for (int idx = t; idx < kHeadMaxC * wpr; idx += kHeadThreads) {
     const int c = idx / wpr, v = idx - c * wpr;
     float4 w = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (c < C) w = *reinterpret_cast<const float4*>(W + static_cast<int64_t>(c) * in + k0 + v * 4);
+    if (c < C) w = *reinterpret_cast<const float4*>(Wr + static_cast<int64_t>(c) * in + k0 + v * 4);
     __nv_bfloat162* d = reinterpret_cast<__nv_bfloat162*>(wq + c * FP + v * 4);
     d[0] = __floats2bfloat162_rn(w.x, w.y);
     d[1] = __floats2bfloat162_rn(w.z, w.w);
   }
-  if (t < kHeadMaxC) bls[t] = t < C ? bL[t] : 0.f;
+  if (t < kHeadMaxC) bls[t] = t < C ? a.bias_src[src_row + t] : 0.f;
   if (t >= 64 && t < 64 + B) ys[t - 64] = a.y[static_cast<int64_t>(j) * a.N + (a.row0 + t - 64) % a.N];
   sync();
   for (int tile = warp; tile < (Bn / 16) * 2; tile += kHeadThreads / 32) {
@@ -203,11 +205,11 @@ __device__ __forceinline__ void head_body(const HeadArgs& a, uint8_t* smem, int 
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       const int c = (lane >> 2) + 8 * h;
-      w32[h] = c < C ? *reinterpret_cast<const float2*>(W + static_cast<int64_t>(c) * in + k0 + f)
+      w32[h] = c < C ? *reinterpret_cast<const float2*>(Wr + static_cast<int64_t>(c) * in + k0 + f)
                      : make_float2(0.f, 0.f);
     }
     bp32 = (a.has_dx && lane < 4)
-               ? *reinterpret_cast<const float2*>(a.bias_prev + static_cast<int64_t>(j) * a.ld + k0 + f)
+               ? *reinterpret_cast<const float2*>(a.bias_prev_src + src_row + k0 + f)
                : make_float2(0.f, 0.f);
   };
   float2 nw32[2], nbp32;

@@ -67,6 +67,10 @@ struct hier_avg {
   std::vector<int> pitch;                       // per width index l = 0..L
   std::vector<int64_t> off_H, off_dZ;
   int64_t off_Z = 0, off_loss = 0, off_err = 0, ws_bytes = 0;
+  // Cluster means [P / S, ld] of a compact local average inside a round (bf16 path,
+  // S > 1): after the step part of the workspace, which is all a single step needs.
+  int64_t off_M = 0, ws_step_bytes = 0;
+  bool m_ok = false;                          // the bound workspace holds the means
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
   int64_t off_dyn = 0;                        // update kernel's work-item counters
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
@@ -87,6 +91,7 @@ struct hier_avg {
   int64_t N = 0;
   cudaStream_t stream = nullptr;
   std::vector<CUtensorMap> tm_wf, tm_wb, tm_h, tm_dz;
+  std::vector<CUtensorMap> tm_wf_m, tm_wb_m;  // the same weight views of the cluster means
   CUtensorMap tm_x;                           // X [P][N][d_0] as the first layer's batch tile
   int64_t t = 0;
   int64_t cursor = 0;                         // rows each learner has read (next batch: mod N)
@@ -122,6 +127,7 @@ struct hier_avg {
   template <class T>
   T* wsp(int64_t off) { return reinterpret_cast<T*>(ws + off); }
   int* err_word() { return wsp<int>(off_err); }
+  float* means() { return wsp<float>(off_M); }
   // A word next to the error word that no kernel ever writes (stays zero).
   const int* never_set() { return wsp<int>(off_err) + 1; }
   float* loss() { return wsp<float>(off_loss); }
@@ -263,6 +269,8 @@ int plan_layout(hier_avg* h) {
   h->off_Z = take(P * B * h->dims[L] * 4);
   h->off_loss = take(P * 4);
   h->off_err = take(16);
+  h->ws_step_bytes = off;
+  if (h->prec == HA_PREC_BF16 && h->S > 1) h->off_M = take((P / h->S) * h->ld * 4);
   h->ws_bytes = off;
   return HA_OK;
 }
@@ -296,6 +304,8 @@ int build_maps(hier_avg* h) {
   h->w_stream = static_cast<double>(h->P) * h->ld * 4 > static_cast<double>(l2);
   h->tm_wf.resize(L);
   h->tm_wb.resize(L);
+  h->tm_wf_m.resize(h->m_ok ? L : 0);
+  h->tm_wb_m.resize(h->m_ok ? L : 0);
   h->tm_h.resize(L);
   h->tm_dz.resize(L + 1);
   const uint64_t P = h->P, Bn = h->Bn;
@@ -309,6 +319,16 @@ int build_maps(hier_avg* h) {
     if ((rc = make_map(h, &h->tm_wb[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
                        h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
       return rc;
+    if (h->m_ok) {
+      float* Wm = h->means() + h->woff[l];
+      const uint64_t G = P / h->S;
+      if ((rc = make_map(h, &h->tm_wf_m[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Wm, in, out, G, in * 4,
+                         h->ld * 4, 32, 128, CU_TENSOR_MAP_SWIZZLE_128B)))
+        return rc;
+      if ((rc = make_map(h, &h->tm_wb_m[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, Wm, in, out, G, in * 4,
+                         h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
+        return rc;
+    }
     const uint64_t pin = h->pitch[l];
     if ((rc = make_map(h, &h->tm_h[l], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, h->ws + h->off_H[l], pin,
                        Bn, P, pin * 2, Bn * pin * 2, 64, static_cast<uint32_t>(Bn),
@@ -384,7 +404,17 @@ double flops_gemm(const hier_avg* h, int l) {
 }
 
 // Arguments of the small last layer (input H_{L-1}, or X rows for a one-layer model).
-ha::HeadArgs head_args(hier_avg* h) {
+// Where a step reads the parameters from: learner j's own row (div 1), or, in the
+// first step after a compact local average, row j / S of the cluster means.
+struct ParamSrc {
+  const float* base;
+  int div;
+};
+ParamSrc param_src(hier_avg* h, bool means) {
+  return means ? ParamSrc{h->means(), h->S} : ParamSrc{h->params, 1};
+}
+
+ha::HeadArgs head_args(hier_avg* h, ParamSrc src) {
   const int L = h->L;
   ha::HeadArgs a{};
   a.C = h->dims[L];
@@ -398,12 +428,16 @@ ha::HeadArgs head_args(hier_avg* h) {
   a.lr = h->lr;
   a.W = h->params + h->woff[L - 1];
   a.bias = h->params + h->boff[L - 1];
+  a.W_src = src.base + h->woff[L - 1];
+  a.bias_src = src.base + h->boff[L - 1];
+  a.src_div = src.div;
   a.x_rows = L == 1;
   a.H = L == 1 ? static_cast<const __nv_bfloat16*>(h->X) : h->wsp<__nv_bfloat16>(h->off_H[L - 1]);
   a.y = h->y;
   a.has_dx = L > 1;
   if (L > 1) {
     a.bias_prev = h->params + h->boff[L - 2];
+    a.bias_prev_src = src.base + h->boff[L - 2];
     a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[L - 1]);
   }
   a.loss = h->loss();
@@ -413,17 +447,21 @@ ha::HeadArgs head_args(hier_avg* h) {
 // One step.  h1_ready: H_1 of this step was written by the previous step's
 // update+forward kernel (skip the first layer's forward).  fuse_next: the caller runs
 // the next step right after this one with nothing in between, so this step may
-// compute the next step's H_1; *fused reports whether it did.  shared: the caller has
-// just averaged each local cluster, so its S learners hold identical parameters and
-// the forwards read one copy per cluster (the same values: results are unchanged).
+// compute the next step's H_1; *fused reports whether it did.  from_means: the caller
+// has just taken a compact local average (do_local_means), so every learner's
+// parameters are its cluster's mean: every kernel reads them from row j / S of the
+// means and writes learner j's own row.  Every weight and bias is updated exactly once
+// per step, so after this step every learner row holds its parameters again.
 // next_rows (round_host): recorded once the next step's rows are on the device; the
 // update+forward kernel, which reads them, waits for it.
 int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
-            bool shared = false, cudaEvent_t next_rows = nullptr) {
+            bool from_means = false, cudaEvent_t next_rows = nullptr) {
   const int L = h->L, P = h->P, B = h->Bstep;
   if (fused) *fused = false;
   cudaStream_t s = h->stream;
   int rc;
+  const bool means = from_means && h->m_ok;
+  const ParamSrc src = param_src(h, means);
   if (h->prec == HA_PREC_BF16) {
     const int d0 = h->dims[0];
     // The first layer reads its batch tile straight from X unless the batch wraps
@@ -445,7 +483,10 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.B = B;
       a.Bn = h->Bn;
       a.ld = h->ld;
-      a.bias = h->params + h->boff[l];
+      a.bias = src.base + h->boff[l];
+      a.b_div = src.div;
+      a.w_div = src.div;
+      a.bias_out = h->params + h->boff[l];
       a.ctas = h->fwd_ctas[l];
       a.cq = h->fwd_cq[l];
       a.o_tiles = h->fwd_tiles[l];
@@ -458,7 +499,6 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.dyn = h->wsp<int>(h->off_dyn);
       a.x_direct = (l == 0 && x_direct) ? 1 : 0;
       a.w_stream = h->w_stream ? 1 : 0;
-      a.share = shared ? h->S : 1;
       a.x_row0 = static_cast<int>(r0);
       if (l + 1 < L) {
         a.mode = 0;
@@ -480,13 +520,13 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.err = h->err_word();
       const CUtensorMap& hin = a.x_direct ? h->tm_x : h->tm_h[l];
       rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), flops_gemm(h, l), [&] {
-        return ha::launch_tc_forward(h->tm_wf[l], hin, a, P, s);
+        return ha::launch_tc_forward(means ? h->tm_wf_m[l] : h->tm_wf[l], hin, a, P, s);
       }, "forward");
       if (rc) return rc;
     }
     const int C = h->dims[L];
     if (h->head) {
-      const ha::HeadArgs a = head_args(h);
+      const ha::HeadArgs a = head_args(h, src);
       const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0));
       const double hf = flops_gemm(h, L - 1) * (L > 1 ? 3 : 2);   // forward, dW (, dX)
       rc = h->timed(HA_KERNEL_HEAD, hb, hf, [&] { return ha::launch_head(a, P, s); }, "head");
@@ -494,7 +534,8 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
     } else if (!h->fused_xent) {
       rc = h->timed(HA_KERNEL_XENT, double(P) * B * C * 4 * 3, 0.0, [&] {
         return ha::launch_xent_bf16(h->wsp<float>(h->off_Z), h->y, h->N, r0, B, h->Bn, C,
-                                    h->pitch[L], h->lr, h->params + h->boff[L - 1], h->ld,
+                                    h->pitch[L], h->lr, src.base + h->boff[L - 1], src.div,
+                                    h->params + h->boff[L - 1], h->ld,
                                     h->wsp<__nv_bfloat16>(h->off_dZ[L]), h->loss(), P, s);
       }, "xent");
       if (rc) return rc;
@@ -508,11 +549,15 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.ld = h->ld;
       a.lr = h->lr;
       a.has_dx = l > 0;
+      a.src_div = src.div;
       if (a.has_dx) {
         a.bias_prev = h->params + h->boff[l - 1];
+        a.bias_prev_src = src.base + h->boff[l - 1];
         a.dz_prev = h->wsp<__nv_bfloat16>(h->off_dZ[l]);
         a.pitch_in = h->pitch[l];
       }
+      const CUtensorMap& wl = means ? h->tm_wb_m[l] : h->tm_wb[l];   // W read ...
+      const CUtensorMap& ws = h->tm_wb[l];                           // ... and written
       // H_{l-1}: the layer's input rows, straight from X for the first layer when
       // the forward read them there too.
       const bool from_x = l == 0 && x_direct;
@@ -539,7 +584,9 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.B = B;
         f.Bn = h->Bn;
         f.ld = h->ld;
-        f.bias = h->params + h->boff[0];
+        f.bias = h->params + h->boff[0];   // b_1 after this step's update (row j)
+        f.b_div = 1;
+        f.w_div = src.div;                 // W_1 before it (from the means after an average)
         f.mode = 0;
         f.h_out = h->wsp<__nv_bfloat16>(h->off_H[1]);
         f.pitch_out = h->pitch[1];
@@ -553,7 +600,6 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.part = h->wsp<float>(h->off_part);
         f.counters = h->wsp<int>(h->off_cnt);
         f.dyn = h->wsp<int>(h->off_dyn);
-        f.share = 1;
         f.x_direct = 1;
         f.x_row0 = static_cast<int>(r1);
         f.hc_row0 = a.h_row0;
@@ -563,7 +609,8 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         if (next_rows && (rc = h->cuda(cudaStreamWaitEvent(s, next_rows, 0), "round_host: wait for the rows")))
           return rc;
         rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h), 2 * flops_gemm(h, 0), [&] {
-          return ha::launch_tc_update_forward(h->tm_wf[0], hin, h->tm_x, h->tm_dz[1], f, s);
+          return ha::launch_tc_update_forward(means ? h->tm_wf_m[0] : h->tm_wf[0], h->tm_wf[0], hin,
+                                              h->tm_x, h->tm_dz[1], f, s);
         }, "update+forward");
         if (rc) return rc;
         if (fused) *fused = true;
@@ -574,12 +621,12 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       // kernel's items for short layers too: 3072-512-10 round 0.859 -> 0.850 ms).
       if (a.has_dx) {
         rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
-          return ha::launch_tc_backward(h->tm_wb[l], hin, h->tm_dz[l + 1], a, P, s);
+          return ha::launch_tc_backward(wl, ws, hin, h->tm_dz[l + 1], a, P, s);
         }, "backward");
       } else {
         a.ctas = kTargetCtas;
         rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
-          return ha::launch_tc_update(h->tm_wb[l], hin, h->tm_dz[l + 1], a, s);
+          return ha::launch_tc_update(wl, ws, hin, h->tm_dz[l + 1], a, s);
         }, "backward");
       }
       if (rc) return rc;
@@ -633,6 +680,18 @@ int do_local(hier_avg* h) {
   }, "local average");
 }
 
+// The local average inside a round, written compactly: each cluster's mean once, to
+// row g of the means [P / S, ld], instead of to its S learner rows.  The next step
+// reads every learner's parameters from there (do_step's from_means) and writes the
+// learner rows, so the values every kernel sees are those of the full write-back.
+// Algorithmic bytes: P rows read, P / S rows written.
+int do_local_means(hier_avg* h) {
+  return h->timed(HA_KERNEL_LOCAL_AVG, 4.0 * h->P * h->ld + 4.0 * (h->P / h->S) * h->ld,
+                  double(h->P) * h->ld, [&] {
+    return ha::launch_group_mean_to(h->params, h->P, h->S, h->ld, h->ld, h->means(), h->stream);
+  }, "local average");
+}
+
 int do_local_global(hier_avg* h) {
   return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, double(h->P) * h->ld, [&] {
     return ha::launch_local_global_mean(h->params, h->P, h->S, h->ld, h->ld, h->stream);
@@ -650,7 +709,9 @@ int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 // One global round (Algorithm 1, Sec. 3.1): G local steps, a local average after every
 // K1-th, the global average after the G-th (fused with the local average that closes
 // the round when K1 divides G).  G = K1 * K2 unless set: Sec. 3.1 leaves beta = G / K1
-// free in practice.
+// free in practice.  The local averages inside the round are compact (do_local_means)
+// when the workspace holds the means; the global average writes every learner row, so
+// the round ends with all P rows in place.
 // The round launches no cooperative kernel: every forward layer runs in cluster split-K
 // mode and only the first layer's backward (no dX) runs on the tensor cores.
 bool cooperative_free(const hier_avg* h) {
@@ -669,6 +730,7 @@ bool cooperative_free(const hier_avg* h) {
 int do_round(hier_avg* h, const std::vector<cudaEvent_t>* ready = nullptr) {
   int rc;
   const int G = round_steps(h);
+  const bool compact = h->m_ok;
   bool h1_ready = false;
   for (int r = 1; r <= G; ++r) {
     const int k = r - 1;
@@ -678,10 +740,10 @@ int do_round(hier_avg* h, const std::vector<cudaEvent_t>* ready = nullptr) {
       return rc;
     const bool block_end = r % h->K1 == 0;              // a local average follows step r
     const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
-    if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local,
+    if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local && compact,
                       ready && r == 1 && G > 1 ? (*ready)[1] : nullptr)))
       return rc;
-    if (r < G && block_end && (rc = do_local(h))) return rc;
+    if (r < G && block_end && (rc = compact ? do_local_means(h) : do_local(h))) return rc;
   }
   return G % h->K1 == 0 ? do_local_global(h) : do_global(h);
 }
@@ -843,8 +905,9 @@ int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t w
   h->stream = static_cast<cudaStream_t>(stream);
   h->t = 0;
   h->cursor = 0;
+  h->m_ok = h->off_M > 0;
   int rc;
-  if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_bytes, h->stream), "bind: memset"))) return rc;
+  if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_step_bytes, h->stream), "bind: memset"))) return rc;
   if (h->prec == HA_PREC_BF16) {
     if ((rc = h->cuda(ha::tc_configure(), "bind: kernel attributes"))) return rc;
     if ((rc = h->cuda(ha::head_configure(), "bind: kernel attributes"))) return rc;
@@ -1169,11 +1232,11 @@ extern "C" int hier_avg_step_static(hier_avg* h, float* params_dev, const void* 
   if (!h) return HA_EINVAL;
   if (!params_dev || !X_dev || !y_dev || N < 1)
     return h->fail(HA_EINVAL, "step_static: NULL buffer or N < 1");
-  if (h->ws_bytes > kStaticScratchBytes)
+  if (h->ws_step_bytes > kStaticScratchBytes)
     return h->fail(HA_ENOMEM,
                    "step_static: this configuration needs %lld bytes of scratch, the static "
                    "array holds %lld; use hier_avg_bind with a caller workspace",
-                   (long long)h->ws_bytes, (long long)kStaticScratchBytes);
+                   (long long)h->ws_step_bytes, (long long)kStaticScratchBytes);
   if (reinterpret_cast<uintptr_t>(params_dev) % 256)
     return h->fail(HA_EINVAL, "step_static: params must be 256-byte aligned");
   if (h->prec == HA_PREC_BF16 && reinterpret_cast<uintptr_t>(X_dev) % 16)
@@ -1198,8 +1261,9 @@ extern "C" int hier_avg_step_static(hier_avg* h, float* params_dev, const void* 
   h->stream = static_cast<cudaStream_t>(stream);
   // The array keeps whatever the previous call (of any handle) left in it; the
   // step needs its padding and its split-K counters to start at zero.
-  if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_bytes, h->stream), "step_static: clear")))
+  if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_step_bytes, h->stream), "step_static: clear")))
     return rc;
+  h->m_ok = false;   // the array holds a step's scratch only: rounds average in place
   if (h->prec == HA_PREC_BF16) {
     if ((rc = h->cuda(ha::tc_configure(), "step_static: kernel attributes"))) return rc;
     if ((rc = h->cuda(ha::head_configure(), "step_static: kernel attributes"))) return rc;

@@ -47,6 +47,9 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // every row of the group.  n = 1 is a no-op.
 cudaError_t launch_group_mean(float* w, int64_t P, int64_t n, int64_t D, int64_t ld,
                               cudaStream_t s);
+// The same means written once per group, to row g of out[P / n, ld] (w unchanged).
+cudaError_t launch_group_mean_to(const float* w, int64_t P, int64_t n, int64_t D, int64_t ld,
+                                 float* out, cudaStream_t s);
 // The local average (clusters of S) followed by the global average, in one pass.
 cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, int64_t ld,
                                      cudaStream_t s);
@@ -67,8 +70,14 @@ struct HeadArgs {
   int64_t ld, N;
   int64_t row0;               // first row of this step's batch in each learner's data (< N)
   float lr;
-  float* W;                   // learner 0's W_L [C][in] (fp32 master)
-  float* bias;                // learner 0's b_L
+  float* W;                   // learner 0's W_L [C][in] (fp32 master), written
+  float* bias;                // learner 0's b_L, written
+  // Parameters are read from row j / src_div of these (learner j; the same as W, bias,
+  // bias_prev with src_div = 1, or the cluster means right after a compact average).
+  const float* W_src;
+  const float* bias_src;
+  const float* bias_prev_src;
+  int src_div;
   const __nv_bfloat16* H;     // H_{L-1} [P][Bn][pitch_in], or X [P][N][in] when x_rows
   int x_rows;
   const int32_t* y;
@@ -80,7 +89,10 @@ struct HeadArgs {
 struct TcFwdArgs {
   int in, out, B, Bn;
   int64_t ld;                 // parameter row length (floats)
-  const float* bias;          // learner 0's b_l; learner j at + j * ld
+  const float* bias;          // b_l read for learner j at row j / b_div (+ row * ld)
+  int b_div;
+  int w_div;                  // learner j's W is row j / w_div of the W map it is given
+  float* bias_out;            // mode 2: b_L after its update, learner j at + j * ld
   int mode;                   // 0 hidden (ReLU -> H), 1 logits -> z_out, 2 fused softmax-CE
   __nv_bfloat16* h_out;       // mode 0: H_{l+1} [P][Bn][pitch_out]
   int pitch_out;              // mode 0: H pitch; mode 2: dZ_L pitch
@@ -103,8 +115,6 @@ struct TcFwdArgs {
   int x_direct, x_row0;
   int hc_row0;                // update+forward: rows of this step's batch in its map
   int w_stream;               // load W with the L2 evict-first policy
-  int share;                  // > 1: learners [g*share, (g+1)*share) hold identical W (right
-                              // after an average): all read learner g*share's copy
   // mode 2: labels and outputs of the fused cross-entropy
   const int32_t* y;
   int64_t N, row0;            // labels: rows row0 + b (mod N)
@@ -118,7 +128,10 @@ struct TcBwdArgs {
   int64_t ld;
   float lr;
   int has_dx;                 // compute dZ_{l-1} (every layer but the first)
-  float* bias_prev;           // learner 0's b_{l-1}
+  float* bias_prev;           // learner 0's b_{l-1}, written (row j)
+  const float* bias_prev_src; // b_{l-1} read for learner j at row j / src_div
+  int src_div;                // learner j's W (and b_{l-1}) read from row j / src_div of
+                              // the load map (and bias_prev_src)
   __nv_bfloat16* dz_prev;     // dZ_{l-1} [P][Bn][pitch_in]
   int pitch_in;
   int h_row0;                 // first batch row of H_{l-1} in its tensor map (X rows for l = 0)
@@ -140,26 +153,32 @@ int tc_bwd_smem_bytes();
 cudaError_t tc_configure();   // raises the dynamic shared-memory limits once
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s);
-cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
-                               const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s);
+// W is loaded through w_load (row j / a.src_div) and stored through w_store (row j).
+cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_store,
+                               const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
+                               int P, cudaStream_t s);
 // The first layer's backward (no dX): dW, update and store only, units claimed
 // dynamically (a.dyn zero on entry; reset by the kernel on exit).
-cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
-                             const CUtensorMap& dz, const TcBwdArgs& a, cudaStream_t s);
+cudaError_t launch_tc_update(const CUtensorMap& w_load, const CUtensorMap& w_store,
+                             const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
+                             cudaStream_t s);
 // The first layer's backward (dW, update, store) fused with the next step's first-layer
 // forward (H_1' = relu(X' W_1'^T + b_1), schedule and arithmetic of launch_tc_forward):
 // h_cur holds this step's batch rows (a.hc_row0 ..), x_next the next step's (a.x_row0 ..).
-cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_cur,
-                                     const CUtensorMap& x_next, const CUtensorMap& dz,
-                                     const TcFwdArgs& a, cudaStream_t s);
+// W is loaded through w_load (row j / a.w_div) and stored through w_store (row j).
+cudaError_t launch_tc_update_forward(const CUtensorMap& w_load, const CUtensorMap& w_store,
+                                     const CUtensorMap& h_cur, const CUtensorMap& x_next,
+                                     const CUtensorMap& dz, const TcFwdArgs& a, cudaStream_t s);
 // Mini-batch fetch for the bf16 path: rows (row0 + b) mod N of X -> H_0.
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
                                int pitch0, int64_t row0, int P, __nv_bfloat16* H0, cudaStream_t s);
 // Softmax cross-entropy gradient of the last layer (bf16 operands out), loss, and
 // the SGD update of the last bias.
+// b_L is read for learner j at row j / src_div of bias_src and written to row j of bias_L.
 cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t row0, int B,
-                             int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
-                             __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s);
+                             int Bn, int C, int pitch_c, float lr, const float* bias_src,
+                             int src_div, float* bias_L, int64_t ld, __nv_bfloat16* dZ,
+                             float* loss, int P, cudaStream_t s);
 
 bool head_supported(int C, int in, int B, int P);
 cudaError_t head_configure();   // raises the dynamic shared-memory limit once

@@ -321,22 +321,10 @@ __device__ __forceinline__ void xent_epilogue(const TcFwdArgs& a, int j, int t, 
   if (t < C) {
     float db = 0.f;
     for (int b = 0; b < B; ++b) db = __fadd_rn(db, gs[t * ZP + b]);
-    float* bp = const_cast<float*>(a.bias) + static_cast<int64_t>(j) * a.ld + t;
-    *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
+    const float bv = a.bias[static_cast<int64_t>(j / a.b_div) * a.ld + t];
+    a.bias_out[static_cast<int64_t>(j) * a.ld + t] = __fsub_rn(bv, __fmul_rn(a.lr, db));
   }
   gsync();   // the staging area is reused by the next tile
-}
-
-// First unit of CTA g when U units are split over G CTAs (G <= U).
-__device__ __forceinline__ int unit_begin(int g, int U, int G) {
-  return static_cast<int>(static_cast<int64_t>(g) * U / G);
-}
-// The CTA that owns unit u.
-__device__ __forceinline__ int cta_of(int u, int U, int G) {
-  int g = static_cast<int>(static_cast<int64_t>(u) * G / U);
-  while (g + 1 < G && unit_begin(g + 1, U, G) <= u) ++g;
-  while (g > 0 && unit_begin(g, U, G) > u) --g;
-  return g;
 }
 
 // kDyn: dynamic work items (compiled separately from cluster split-K, so that each
@@ -444,8 +432,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
           f = cl_item;
         }
         const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
-        // learners whose rows are identical (a.share > 1) read one copy: the group's first
-        const int jw = a.share > 1 ? (j / a.share) * a.share : j;
+        // learner j's weights: row j / w_div of the map (the cluster means right after a
+        // compact local average)
+        const int jw = j / a.w_div;
         for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
           const int s = i % nw;
           if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
@@ -595,7 +584,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
     for (int k = 0; ok && next_item(k, f); ++k) {
       const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
       const int ob = ot * 128 + r;
-      const float tbias = ob < a.out ? a.bias[static_cast<int64_t>(j) * a.ld + ob] : 0.f;
+      const float tbias = ob < a.out ? a.bias[static_cast<int64_t>(j / a.b_div) * a.ld + ob] : 0.f;
       for (int c = f.c_lo, p = 0; c < f.c_hi && ok; ++c, ++p, ++i) {
         const bool tlast = c == f.c_hi - 1;
         const int sw = i % nw, bb = i & 1;
@@ -811,8 +800,9 @@ __device__ __forceinline__ bool bwd_piece_end(const TcBwdArgs& a, const FwdItem&
 }
 
 __global__ void __launch_bounds__(kBwdThreads, 1)
-    k_tc_backward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
-                  const __grid_constant__ CUtensorMap tm_dz, const TcBwdArgs a) {
+    k_tc_backward(const __grid_constant__ CUtensorMap tm_wl, const __grid_constant__ CUtensorMap tm_ws,
+                  const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_dz,
+                  const TcBwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -895,7 +885,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     if (lane == 0) {
       // claim, announce, and load: each item's H tile (two 64-feature boxes) ahead of
       // its first W chunk, then its W chunks
-      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_wl);
       tma_prefetch_desc(&tm_h);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
       int i = 0, issued = 0;
@@ -916,7 +906,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           const int s = i % nw;
           if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
           mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
-          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], i0, c * 64, j, stream);
+          tma_load_3d_hint(wf(s), &tm_wl, &wfull[s], i0, c * 64, j / a.src_div, stream);
           issued = i + 1;
         }
       }
@@ -958,7 +948,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
           const int s = i % nw;
           if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) { ok = false; break; }
-          tma_store_3d_hint(&tm_w, wf(s), i0, c * 64, j, stream);
+          tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, j, stream);
           tma_store_commit();
           if (i > 0) {
             tma_store_wait_read_1();
@@ -1066,8 +1056,8 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             dz[static_cast<int64_t>(b) * a.pitch_in] = __float2bfloat16_rn(x);
           }
         }
-        float* bp = a.bias_prev + static_cast<int64_t>(j) * a.ld + fi;
-        *bp = __fsub_rn(*bp, __fmul_rn(a.lr, db));
+        const float bv = a.bias_prev_src[static_cast<int64_t>(j / a.src_div) * a.ld + fi];
+        a.bias_prev[static_cast<int64_t>(j) * a.ld + fi] = __fsub_rn(bv, __fmul_rn(a.lr, db));
       }
       return true;
     };
@@ -1171,8 +1161,9 @@ static_assert(upd_smem(64) <= kBwdSmemMax && upd_smem(48) <= kBwdSmemMax &&
               "update kernel shared-memory plan");
 
 __global__ void __launch_bounds__(kBwdThreads, 1)
-    k_tc_update(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
-                const __grid_constant__ CUtensorMap tm_dz, const TcBwdArgs a) {
+    k_tc_update(const __grid_constant__ CUtensorMap tm_wl, const __grid_constant__ CUtensorMap tm_ws,
+                const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_dz,
+                const TcBwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1255,7 +1246,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   if (warp == 4) {
     if (lane == 0) {
       // claim, announce, and load: W chunks and each item's H tile
-      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_wl);
       tma_prefetch_desc(&tm_h);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
       int i = 0, kt = 0, issued = 0;
@@ -1282,7 +1273,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           const int s = i % nw;
           if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
           mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
-          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], i0, c * 64, j, stream);
+          tma_load_3d_hint(wf(s), &tm_wl, &wfull[s], i0, c * 64, j / a.src_div, stream);
           issued = i + 1;
         }
       }
@@ -1326,7 +1317,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         for (int c = c_lo; c < c_hi; ++c, ++i) {
           const int s = i % nw;
           if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
-          tma_store_3d_hint(&tm_w, wf(s), i0, c * 64, j, stream);
+          tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, j, stream);
           tma_store_commit();
           if (i > 0) {
             tma_store_wait_read_1();
@@ -1488,9 +1479,9 @@ static_assert(uf_hring(64, 1) >= 3 && uf_hring(48, 1) >= 4 && uf_hring(32, 1) >=
 
 template <bool kDyn>
 __global__ void __launch_bounds__(kUfThreads, 1)
-    k_tc_update_forward(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_hc,
-                        const __grid_constant__ CUtensorMap tm_hn, const __grid_constant__ CUtensorMap tm_dz,
-                        const TcFwdArgs a) {
+    k_tc_update_forward(const __grid_constant__ CUtensorMap tm_wl, const __grid_constant__ CUtensorMap tm_ws,
+                        const __grid_constant__ CUtensorMap tm_hc, const __grid_constant__ CUtensorMap tm_hn,
+                        const __grid_constant__ CUtensorMap tm_dz, const TcFwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1584,7 +1575,7 @@ __global__ void __launch_bounds__(kUfThreads, 1)
   if (warp == 8) {
     if (lane == 0) {
       // claim (dynamic), announce, and stream the weight tiles
-      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_wl);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
       int i = 0, issued = 0;
       bool ok = true;
@@ -1600,13 +1591,13 @@ __global__ void __launch_bounds__(kUfThreads, 1)
           if (k > 0) break;
           f = cl_item;
         }
-        const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles;
+        const int j = f.tau / a.o_tiles, ot = f.tau - j * a.o_tiles, jw = j / a.w_div;
         for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
           const int s = i % nw;
           if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
           mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
-          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, ot * 128, j, stream);
-          tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, ot * 128, j, stream);
+          tma_load_3d_hint(wf(s), &tm_wl, &wfull[s], c * 64, ot * 128, jw, stream);
+          tma_load_3d_hint(wf(s) + kFwdWBox, &tm_wl, &wfull[s], c * 64 + 32, ot * 128, jw, stream);
           issued = i + 1;
         }
       }
@@ -1689,8 +1680,8 @@ __global__ void __launch_bounds__(kUfThreads, 1)
         for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
           const int s = i % nw;
           if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) { ok = false; break; }
-          tma_store_3d_hint(&tm_w, wf(s), c * 64, ot * 128, j, stream);
-          tma_store_3d_hint(&tm_w, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
+          tma_store_3d_hint(&tm_ws, wf(s), c * 64, ot * 128, j, stream);
+          tma_store_3d_hint(&tm_ws, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
           tma_store_commit();
           if (cq > 1) {
             tma_store_wait_read_all();
@@ -1816,14 +1807,15 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     // cluster build loads the bias of its one tile up front (cl_bias); the dynamic build,
     // short of registers, at the epilogue.
     const int cl_o = (cl_item.tau % a.o_tiles) * 128 + r;
-    const float cl_bias = !kDyn && cl_o < a.out
-                              ? a.bias[static_cast<int64_t>(cl_item.tau / a.o_tiles) * a.ld + cl_o]
-                              : 0.f;
+    const float cl_bias =
+        !kDyn && cl_o < a.out
+            ? a.bias[static_cast<int64_t>(cl_item.tau / a.o_tiles / a.b_div) * a.ld + cl_o]
+            : 0.f;
     auto epilogue = [&](int tau) {
       const int j = tau / a.o_tiles, ot = tau - j * a.o_tiles;
       const int o = ot * 128 + r;
       if (o < a.out) {
-        const float bias = kDyn ? a.bias[static_cast<int64_t>(j) * a.ld + o] : cl_bias;
+        const float bias = kDyn ? a.bias[static_cast<int64_t>(j / a.b_div) * a.ld + o] : cl_bias;
 #pragma unroll
         for (int m = 0; m < 2; ++m) {
           const int cb = (2 * m + gr) * 16;
@@ -1985,7 +1977,8 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
                                                            const int32_t* __restrict__ y,
                                                            int64_t N, int64_t row0, int B, int Bn,
                                                            int C, int pitch_c, float lr,
-                                                           float* bias_L, int64_t ld,
+                                                           const float* bias_src,
+                                                           int src_div, float* bias_L, int64_t ld,
                                                            __nv_bfloat16* dZ, float* loss) {
   __shared__ float row_max[64], row_sum[64], row_loss[64];
   __shared__ int row_y[64];
@@ -2018,6 +2011,8 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
   }
   const int c = blockIdx.y * kXentThreads + threadIdx.x;
   if (c >= C) return;
+  // (bias_src may be bias_L itself: read before the write below)
+  const float bv = bias_src[static_cast<int64_t>(j / src_div) * ld + c];
   const float fB = static_cast<float>(B);
   float db = 0.f;
   for (int b = 0; b < B; ++b) {
@@ -2026,8 +2021,7 @@ __global__ void __launch_bounds__(kXentThreads) k_xent_bf16(const float* __restr
     db = __fadd_rn(db, g);
     dZ[(static_cast<int64_t>(j) * Bn + b) * pitch_c + c] = __float2bfloat16_rn(g);
   }
-  float* bp = bias_L + static_cast<int64_t>(j) * ld + c;
-  *bp = __fsub_rn(*bp, __fmul_rn(lr, db));
+  bias_L[static_cast<int64_t>(j) * ld + c] = __fsub_rn(bv, __fmul_rn(lr, db));
 }
 
 }  // namespace
@@ -2064,30 +2058,34 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                     false, 1, w_fwd, h_in, a);
 }
 
-cudaError_t launch_tc_backward(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
-                               const CUtensorMap& dz, const TcBwdArgs& a, int P, cudaStream_t s) {
+cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_store,
+                               const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
+                               int P, cudaStream_t s) {
   (void)P;
   // dynamic work items, no CTA waits for another: an ordinary launch
   return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
-                    w_bwd, h_in, dz, a);
+                    w_load, w_store, h_in, dz, a);
 }
 
-cudaError_t launch_tc_update(const CUtensorMap& w_bwd, const CUtensorMap& h_in,
-                             const CUtensorMap& dz, const TcBwdArgs& a, cudaStream_t s) {
+cudaError_t launch_tc_update(const CUtensorMap& w_load, const CUtensorMap& w_store,
+                             const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
+                             cudaStream_t s) {
   // no CTA waits on another: an ordinary (programmatically serialised) launch
   return launch_pdl(k_tc_update, dim3(a.ctas), dim3(kBwdThreads), upd_smem(a.Bn), s, false, 1,
-                    w_bwd, h_in, dz, a);
+                    w_load, w_store, h_in, dz, a);
 }
 
-cudaError_t launch_tc_update_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_cur,
-                                     const CUtensorMap& x_next, const CUtensorMap& dz,
-                                     const TcFwdArgs& a, cudaStream_t s) {
+cudaError_t launch_tc_update_forward(const CUtensorMap& w_load, const CUtensorMap& w_store,
+                                     const CUtensorMap& h_cur, const CUtensorMap& x_next,
+                                     const CUtensorMap& dz, const TcFwdArgs& a, cudaStream_t s) {
   // an ordinary launch, as the forward
   if (a.cq > 1)
     return launch_pdl(k_tc_update_forward<false>, dim3(a.ctas), dim3(kUfThreads),
-                      uf_smem(a.Bn, uf_zbufs(a.Bn, false)), s, false, a.cq, w_fwd, h_cur, x_next, dz, a);
+                      uf_smem(a.Bn, uf_zbufs(a.Bn, false)), s, false, a.cq, w_load, w_store, h_cur,
+                      x_next, dz, a);
   return launch_pdl(k_tc_update_forward<true>, dim3(a.ctas), dim3(kUfThreads),
-                    uf_smem(a.Bn, uf_zbufs(a.Bn, true)), s, false, 1, w_fwd, h_cur, x_next, dz, a);
+                    uf_smem(a.Bn, uf_zbufs(a.Bn, true)), s, false, 1, w_load, w_store, h_cur, x_next,
+                    dz, a);
 }
 
 cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B, int Bn,
@@ -2097,11 +2095,12 @@ cudaError_t launch_gather_bf16(const __nv_bfloat16* X, int64_t N, int d0, int B,
 }
 
 cudaError_t launch_xent_bf16(const float* Z, const int32_t* y, int64_t N, int64_t row0, int B,
-                             int Bn, int C, int pitch_c, float lr, float* bias_L, int64_t ld,
-                             __nv_bfloat16* dZ, float* loss, int P, cudaStream_t s) {
+                             int Bn, int C, int pitch_c, float lr, const float* bias_src,
+                             int src_div, float* bias_L, int64_t ld, __nv_bfloat16* dZ,
+                             float* loss, int P, cudaStream_t s) {
   dim3 grid(P, (C + kXentThreads - 1) / kXentThreads);
   return launch_pdl(k_xent_bf16, grid, dim3(kXentThreads), 0, s, false, 1, Z, y, N, row0, B, Bn, C,
-                    pitch_c, lr, bias_L, ld, dZ, loss);
+                    pitch_c, lr, bias_src, src_div, bias_L, ld, dZ, loss);
 }
 
 }  // namespace ha

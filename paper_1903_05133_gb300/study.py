@@ -14,7 +14,7 @@ Every run processes the same number of samples.  After each global average all
 learners hold the global model, whose mean cross-entropy over every learner's whole
 data set is recorded (evaluated in plain fp32 PyTorch, outside the learner step).
 
-    python -m paper_1903_05133_gb300.study [--seeds 3] [--steps 2752] [--out study.md]
+    python -m paper_1903_05133_gb300.study [--seeds 6] [--steps 2752] [--out study.md]
 
 (2752 local steps = lcm of the global intervals 16, 32, 64 and 43: every run reads
 exactly the same samples.)
@@ -110,6 +110,44 @@ def study(seeds: Sequence[int], steps: int, device="cuda") -> Dict[str, Dict[str
     return out
 
 
+# Paired comparisons (a, b): per seed, loss(a) - loss(b) at the same samples; a
+# negative mean says run a trains faster.  The runs of one seed share data and
+# initialisation, so the per-seed difference removes what the seeds move together.
+PAIRS: Sequence[Tuple[str, str, str]] = (
+    ("Theorem 3.5, K1 (S = 4, 32 steps per global average)", "K1 = 2", "K1 = 16"),
+    ("Theorem 3.5, K1 (S = 4, 32 steps per global average)", "K1 = 4", "K1 = 8"),
+    ("Theorem 3.5, S (K1 = 4, 32 steps per global average)", "S = 16", "S = 1"),
+    ("Theorem 3.5, S (K1 = 4, 32 steps per global average)", "S = 4", "S = 2"),
+    ("Sec. 4.3: K-AVG with K vs Hier-AVG with 2K steps per global average, S = 4",
+     "Hier-AVG, 32 steps, K1 = 4", "K-AVG, K = 16"),
+    ("Sec. 4.3: K-AVG with K vs Hier-AVG with 2K steps per global average, S = 4",
+     "Hier-AVG, 64 steps, K1 = 4", "K-AVG, K = 32"),
+    ("non-integer beta (K1 = 20, 43 steps per global average, S = 4) vs K-AVG, K = 43",
+     "Hier-AVG, 43 steps, K1 = 20", "K-AVG, K = 43"),
+)
+
+
+def paired(res: Dict[str, Dict[str, List[list]]], pairs: Sequence[Tuple[str, str, str]],
+           marks: Sequence[int]) -> str:
+    """Per-seed paired differences loss(a) - loss(b): mean ± std over seeds, the
+    t statistic mean / (std / sqrt(n)), and how many seeds have a < b."""
+    lines = ["| a − b | " + " | ".join(f"{m} samples" for m in marks) + " |",
+             "|---|" + "---|" * len(marks)]
+    for section, a, b in pairs:
+        ca, cb = res[section][a], res[section][b]
+        cells = []
+        for m in marks:
+            d = [_interp(x, m) - _interp(y, m) for x, y in zip(ca, cb)]
+            n = len(d)
+            mu = sum(d) / n
+            sd = math.sqrt(sum((x - mu) ** 2 for x in d) / max(1, n - 1))
+            t = mu / (sd / math.sqrt(n)) if sd > 0 else float("inf") * (1 if mu >= 0 else -1)
+            wins = sum(1 for x in d if x < 0)
+            cells.append(f"{mu:+.5f} ± {sd:.5f} (t = {t:+.1f}, {wins}/{n} below)")
+        lines.append(f"| {a} − {b} | " + " | ".join(cells) + " |")
+    return "\n".join(lines) + "\n"
+
+
 def _interp(curve: List[Tuple[int, float]], samples: int) -> float:
     """The loss after `samples` samples per learner (linear between global averages)."""
     for (s0, l0), (s1, l1) in zip(curve, curve[1:]):
@@ -139,7 +177,7 @@ def report(res: Dict[str, Dict[str, List[list]]], marks: Sequence[int]) -> str:
 
 def main() -> None:
     ap = argparse.ArgumentParser()
-    ap.add_argument("--seeds", type=int, default=3)
+    ap.add_argument("--seeds", type=int, default=6)
     ap.add_argument("--steps", type=int, default=2752,
                     help="local steps per run, a multiple of every global interval")
     ap.add_argument("--out", default=None)
@@ -149,6 +187,9 @@ def main() -> None:
     B = base_workload(0).B
     marks = [args.steps * B // 4, args.steps * B // 2, args.steps * B]
     text = report(res, marks)
+    text += ("\n**Paired differences** (per seed, loss(a) − loss(b) at equal samples; "
+             "negative: a trains faster)\n\n")
+    text += paired(res, PAIRS, marks)
     text += f"\n({args.seeds} seeds, {args.steps} local steps per run, {time.time() - t0:.0f} s)\n"
     print(text)
     if args.out:

@@ -17,6 +17,20 @@ def test_interp_and_report():
     assert "run a" in text and "1.1000 ± 0.1414" in text and "0.6000 ± 0.1414" in text
 
 
+def test_paired_differences():
+    a = [[(0, 2.0), (100, 1.0)], [(0, 2.0), (100, 1.2)], [(0, 2.0), (100, 0.9)]]
+    b = [[(0, 2.0), (100, 1.1)], [(0, 2.0), (100, 1.25)], [(0, 2.0), (100, 1.0)]]
+    text = study.paired({"sec": {"a": a, "b": b}}, [("sec", "a", "b")], [100])
+    # differences -0.1, -0.05, -0.1: mean -0.08333, std 0.02887, t = -5.0, 3 of 3 below
+    assert "-0.08333 ± 0.02887 (t = -5.0, 3/3 below)" in text
+
+
+def test_pairs_name_existing_runs():
+    runs = {section: {r.label for r in rs} for section, rs in study.STUDY}
+    for section, a, b in study.PAIRS:
+        assert a in runs[section] and b in runs[section]
+
+
 def test_every_global_interval_divides_the_default_budget():
     for _section, runs in study.STUDY:
         for r in runs:
