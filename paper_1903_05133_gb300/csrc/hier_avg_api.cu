@@ -712,36 +712,103 @@ int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 // free in practice.  The local averages inside the round are compact (do_local_means)
 // when the workspace holds the means; the global average writes every learner row, so
 // the round ends with all P rows in place.
-// The round launches no cooperative kernel: every forward layer runs in cluster split-K
-// mode and only the first layer's backward (no dX) runs on the tensor cores.
-bool cooperative_free(const hier_avg* h) {
-  const int n_fwd = h->head ? h->L - 1 : h->L;
-  for (int l = 0; l < n_fwd; ++l)
-    if (h->fwd_cq[l] < 2) return false;
-  return (h->head ? h->L - 2 : h->L - 1) <= 0;
+// Rows [r0, r0 + n) of every learner's data from host memory.  Spans of at least
+// kRowCopySplit bytes per learner go as one contiguous copy per learner (a pitched 2-D
+// copy of 25 MB rows measured ~55 GB/s against ~200 GB/s for 1-D copies); shorter spans
+// as one pitched copy for all learners, which costs one call instead of P (the host's
+// calls are what limits a short round).
+constexpr int64_t kRowCopySplit = int64_t(1) << 20;
+
+int copy_rows(hier_avg* h, const void* X_host, const int32_t* y_host, int64_t r0, int64_t n,
+              cudaStream_t cs) {
+  const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
+  const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
+  uint8_t* X = static_cast<uint8_t*>(const_cast<void*>(h->X));
+  const uint8_t* Xh = static_cast<const uint8_t*>(X_host);
+  int32_t* y = const_cast<int32_t*>(h->y);
+  if (n * rowb < kRowCopySplit) {
+    if (int rc = h->cuda(cudaMemcpy2DAsync(X + r0 * rowb, h->N * rowb, Xh + r0 * rowb, h->N * rowb,
+                                           n * rowb, h->P, cudaMemcpyHostToDevice, cs),
+                         "round_host: X copy"))
+      return rc;
+    return h->cuda(cudaMemcpy2DAsync(y + r0, h->N * 4, y_host + r0, h->N * 4, n * 4, h->P,
+                                     cudaMemcpyHostToDevice, cs), "round_host: y copy");
+  }
+  for (int j = 0; j < h->P; ++j) {
+    const int64_t off = static_cast<int64_t>(j) * h->N + r0;
+    if (int rc = h->cuda(cudaMemcpyAsync(X + off * rowb, Xh + off * rowb, n * rowb,
+                                         cudaMemcpyHostToDevice, cs), "round_host: X copy"))
+      return rc;
+    if (int rc = h->cuda(cudaMemcpyAsync(y + off, y_host + off, n * 4, cudaMemcpyHostToDevice, cs),
+                         "round_host: y copy"))
+      return rc;
+  }
+  return HA_OK;
 }
 
-// ready (round_host): ready[k] is recorded once the rows of the round's step k (0-based)
-// are on the device.  Step k reads those rows and, in an update+forward kernel, step
-// k + 1's.  The handle's stream waits for ready[0] before step 0 (and for ready[1] just
-// before step 0's update+forward), then at steps k = 1, 3, 7, ... (k + 1 a power of two)
-// for the rows up to step 2k + 1, which cover every step until the next wait: few waits,
-// since each one ends the overlap of consecutive launches.
-int do_round(hier_avg* h, const std::vector<cudaEvent_t>* ready = nullptr) {
+// round_host's row feed: the rows of the round's steps are copied from host memory on
+// the library's copy stream in chunks of steps that double in length (step 0, step 1,
+// steps 2-3, 4-7, ...).  ensure(k) issues the chunks up to the one holding step k and
+// one more, so the copies stay a chunk ahead of the kernels while the host issues only
+// 2 P copies per chunk (O(P log G) per round) between kernel launches; event(k) is
+// recorded once step k's rows are on the device.
+struct RowFeed {
+  hier_avg* h;
+  const void* X_host;
+  const int32_t* y_host;
+  int G;
+  int issued_to = 0;            // steps [0, issued_to) have their copies issued
+  int chunks = 0;
+  std::vector<cudaEvent_t> ev;  // ev[k]: event of step k's chunk
+  int issue_next() {
+    const int k0 = issued_to;
+    if (k0 >= G) return HA_OK;
+    const int k1 = std::min(G, k0 <= 1 ? k0 + 1 : 2 * k0);
+    int64_t r0 = (h->cursor + static_cast<int64_t>(k0) * h->Bstep) % h->N;
+    const int64_t rows = static_cast<int64_t>(k1 - k0) * h->Bstep;
+    int64_t left = rows < h->N ? rows : h->N;
+    if (rows >= h->N) r0 = 0;
+    while (left > 0) {
+      const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
+      if (int rc = copy_rows(h, X_host, y_host, r0, n, h->copy_stream)) return rc;
+      left -= n;
+      r0 = 0;
+    }
+    cudaEvent_t e = h->copied[chunks++];
+    if (int rc = h->cuda(cudaEventRecord(e, h->copy_stream), "round_host: record")) return rc;
+    for (int k = k0; k < k1; ++k) ev[k] = e;
+    issued_to = k1;
+    return HA_OK;
+  }
+  int ensure(int k) {
+    while (issued_to <= k)
+      if (int rc = issue_next()) return rc;
+    return issue_next();   // one chunk ahead
+  }
+};
+
+// feed (round_host): step k reads the rows of step k and, in an update+forward kernel,
+// step k + 1's.  The handle's stream waits for step 0's and step 1's rows before step 0
+// (the latter just before step 0's update+forward), then at steps k = 1, 3, 7, ... (k + 1
+// a power of two) for the rows up to step 2k + 1, which cover every step until the next
+// wait: few waits, since each one ends the overlap of consecutive launches.
+int do_round(hier_avg* h, RowFeed* feed = nullptr) {
   int rc;
   const int G = round_steps(h);
   const bool compact = h->m_ok;
   bool h1_ready = false;
   for (int r = 1; r <= G; ++r) {
     const int k = r - 1;
-    if (ready && (k == 0 || (k & (k + 1)) == 0) &&
-        (rc = h->cuda(cudaStreamWaitEvent(h->stream, (*ready)[k == 0 ? 0 : std::min(2 * k + 1, G - 1)], 0),
-                      "round_host: wait for the rows")))
-      return rc;
+    if (feed && (k == 0 || (k & (k + 1)) == 0)) {
+      const int need = k == 0 ? 0 : std::min(2 * k + 1, G - 1);
+      if ((rc = feed->ensure(std::max(need, std::min(1, G - 1))))) return rc;
+      if ((rc = h->cuda(cudaStreamWaitEvent(h->stream, feed->ev[need], 0), "round_host: wait for the rows")))
+        return rc;
+    }
     const bool block_end = r % h->K1 == 0;              // a local average follows step r
     const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
     if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local && compact,
-                      ready && r == 1 && G > 1 ? (*ready)[1] : nullptr)))
+                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr)))
       return rc;
     if (r < G && block_end && (rc = compact ? do_local_means(h) : do_local(h))) return rc;
   }
@@ -945,8 +1012,6 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
   if (int rc = check_bound(h)) return rc;
   DeviceScope scope(h->device);
   if (!X_host || !y_host || !loss_host) return h->fail(HA_EINVAL, "round_host: NULL host buffer");
-  const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
-  const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
   const int G = round_steps(h);
   if (!h->copy_stream &&
       h->cuda(cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking), "round_host: stream"))
@@ -960,60 +1025,31 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
     h->copied.push_back(e);
   }
   int rc;
-  if (!(h->prec == HA_PREC_BF16 && !h->w_stream && cooperative_free(h))) {
-    // The round's rows, at most two contiguous ranges per learner (wrap-around), copied
-    // ahead of the round.  (Copied step by step instead, beside the kernels or ahead of
-    // them, the rounds with stream-K kernels and an evict-first weight stream measured
-    // much slower end to end: 3072-2048-2048-10 went from 2.85 to 2.20 or 1.54 M
-    // learner-samples/s.)
+  if (h->prec != HA_PREC_BF16) {
+    // fp32 path: the round's rows (at most two contiguous ranges per learner, at the
+    // wrap-around) copied ahead of the round
     const int64_t rows = static_cast<int64_t>(h->Bstep) * G;
     int64_t r0 = h->cursor % h->N, left = rows < h->N ? rows : h->N;
     if (rows >= h->N) r0 = 0;
     while (left > 0) {
       const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
-      if ((rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
-                                          h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
-                                          h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice, h->stream),
-                        "round_host: X copy")))
-        return rc;
-      if ((rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
-                                          n * 4, h->P, cudaMemcpyHostToDevice, h->stream),
-                        "round_host: y copy")))
-        return rc;
+      if ((rc = copy_rows(h, X_host, y_host, r0, n, h->stream))) return rc;
       left -= n;
       r0 = 0;
     }
     if ((rc = do_round(h))) return rc;
   } else {
-    // Rounds without cooperative kernels whose weights fit in L2: step k's rows,
-    // (row0 + b) mod N for b < B, are copied on a stream of the library's own (at most
-    // two contiguous ranges per learner), then copied[k] is recorded.  The copies start
-    // once the work already queued on the handle's stream is done, and overlap the
-    // kernels, which wait as do_round says.
-    const cudaStream_t cs = h->copy_stream;
+    // The rows are copied beside the kernels, chunk by chunk (RowFeed).  (Copies of
+    // every step issued ahead of the round, 2 P per step, kept the host busy for
+    // milliseconds before the first kernel launch: 3072-2048-2048-10 end to end 1.25x
+    // the device-resident round.)  The copies start once the work already queued on the
+    // handle's stream is done.
     if ((rc = h->cuda(cudaEventRecord(h->round_start, h->stream), "round_host: record")) ||
-        (rc = h->cuda(cudaStreamWaitEvent(cs, h->round_start, 0), "round_host: wait")))
+        (rc = h->cuda(cudaStreamWaitEvent(h->copy_stream, h->round_start, 0), "round_host: wait")))
       return rc;
-    for (int k = 0; k < G; ++k) {
-      int64_t r0 = (h->cursor + static_cast<int64_t>(k) * h->Bstep) % h->N;
-      int64_t left = h->Bstep < h->N ? h->Bstep : h->N;
-      while (left > 0) {
-        const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
-        if ((rc = h->cuda(cudaMemcpy2DAsync(static_cast<uint8_t*>(const_cast<void*>(h->X)) + r0 * rowb,
-                                            h->N * rowb, static_cast<const uint8_t*>(X_host) + r0 * rowb,
-                                            h->N * rowb, n * rowb, h->P, cudaMemcpyHostToDevice, cs),
-                          "round_host: X copy")))
-          return rc;
-        if ((rc = h->cuda(cudaMemcpy2DAsync(const_cast<int32_t*>(h->y) + r0, h->N * 4, y_host + r0, h->N * 4,
-                                            n * 4, h->P, cudaMemcpyHostToDevice, cs),
-                          "round_host: y copy")))
-          return rc;
-        left -= n;
-        r0 = 0;
-      }
-      if ((rc = h->cuda(cudaEventRecord(h->copied[k], cs), "round_host: record"))) return rc;
-    }
-    if ((rc = do_round(h, &h->copied))) return rc;
+    RowFeed feed{h, X_host, y_host, G};
+    feed.ev.assign(G, nullptr);
+    if ((rc = do_round(h, &feed))) return rc;
   }
   if ((rc = h->cuda(cudaMemcpyAsync(loss_host, h->loss(), h->P * 4, cudaMemcpyDeviceToHost, h->stream),
                     "round_host: loss copy")))

@@ -519,17 +519,25 @@ def test_full_size_step_sampled(w):
     assert stats["exempt_rows"] <= rows // 1000, stats.get("exempt")
 
 
-# SMALL_BF16: the rows are copied step by step beside the kernels (two layers, cluster
-# split-K, weights in L2); FUSE_THREE: copied ahead of the round (stream-K layers)
-@pytest.mark.parametrize("w", [SMALL_BF16, FUSE_THREE], ids=lambda w: w.name)
-def test_round_host_matches_device_round(w):
+# bf16 path: the rows are copied beside the kernels in chunks of steps that double in
+# length; SMALL_BF16's round reads more rows than each learner has (the chunks wrap
+# around N), FUSE_PIECES has 6 steps (chunks 0 | 1 | 2-3 | 4-5), a free global interval
+# of 7 steps ends on a short chunk.  fp32 path: the rows are copied ahead of the round.
+@pytest.mark.parametrize("w,G", [(SMALL_BF16, 0), (FUSE_THREE, 0), (FUSE_PIECES, 0),
+                                 (SMALL_BF16.replace(K1=3), 7), (SMALL_FP32, 0)],
+                         ids=lambda v: getattr(v, "name", str(v)))
+def test_round_host_matches_device_round(w, G):
     ha1, X, y = setup(w)
     ha2, _, _ = setup(w)
-    ha1.round()
-    loss = ha2.round_host(X.pin_memory(), y.pin_memory())
-    torch.cuda.synchronize()
-    assert torch.equal(ha1.params, ha2.params)
-    assert torch.allclose(loss, ha1.losses())
+    for h in (ha1, ha2):
+        h.set_global_steps(G)
+    Xh, yh = X.pin_memory(), y.pin_memory()
+    for _ in range(2):                  # the second round starts mid data set
+        ha1.round()
+        loss = ha2.round_host(Xh, yh)
+        torch.cuda.synchronize()
+        assert torch.equal(ha1.params, ha2.params)
+        assert torch.allclose(loss, ha1.losses())
 
 
 def test_resume_from_saved_step():
