@@ -276,12 +276,19 @@ def test_full_run_against_oracle(w):
     assert ha.get_step() == w.rounds * w.K1 * w.K2
 
 
-def test_literal_sequence_equals_round():
+# round() writes each intermediate local average as one mean row per cluster, read by
+# the next step, and fuses the last local average into the global one; the literal
+# sequence writes every row each time.  Cases: clusters of 2; clusters of 3 over a
+# ragged three-layer net (the generic, non-power-of-two averaging path, with K1 = 1: a
+# compact average after every step but the last); 5 clusters of 4 (a global tree over
+# a non-power-of-two count of clusters), head slices of 128 features.
+@pytest.mark.parametrize("w", [SMALL_BF16, RAGGED_BF16.replace(K2=3), HEAD_F128],
+                         ids=lambda w: w.name)
+def test_literal_sequence_equals_round(w):
     # step/local_average/global_average in Algorithm 1's order give the same bits
-    # as round(), which fuses the last local average into the global one.
-    w = SMALL_BF16
-    ha1, X, y = setup(w)
-    ha2, _, _ = setup(w)
+    # as round()
+    ha1, X, y = setup(w, perturb=(0.01, 0.01))
+    ha2, _, _ = setup(w, perturb=(0.01, 0.01))
     ha1.round()
     for b in range(w.K2):
         for k in range(w.K1):
