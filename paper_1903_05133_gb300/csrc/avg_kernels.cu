@@ -68,17 +68,19 @@ __global__ void __launch_bounds__(256) k_mean_pow2(float4* __restrict__ w, int64
   store_rows(p, ld_v, 1 << LOG, m);
 }
 
-// The same group means written once per group, to row blockIdx.y of out (compact
-// cluster means; the learner rows are only read).
+// The same group sums divided by div, written once per group, to row blockIdx.y of
+// out (row stride out_ld_v): compact cluster means, the rows of w only read.  div is
+// the group size, or, when the rows of w are themselves sums of the first tree levels
+// (group sums of Q learners), the cluster size.
 template <int LOG>
 __global__ void __launch_bounds__(256) k_mean_pow2_to(const float4* __restrict__ w, int64_t ld_v,
-                                                      int64_t cols_v, float4* __restrict__ out) {
+                                                      int64_t cols_v, float div,
+                                                      float4* __restrict__ out, int64_t out_ld_v) {
   grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   const float4* p = w + static_cast<int64_t>(blockIdx.y) * (int64_t(1) << LOG) * ld_v + c;
-  out[static_cast<int64_t>(blockIdx.y) * ld_v + c] =
-      vdiv(tree_pow2<LOG>(p, ld_v), static_cast<float>(1 << LOG));
+  out[static_cast<int64_t>(blockIdx.y) * out_ld_v + c] = vdiv(tree_pow2<LOG>(p, ld_v), div);
 }
 
 // Fused last local average + global average: G = 2^LOGG clusters of S = 2^LOGS.
@@ -152,12 +154,13 @@ __global__ void __launch_bounds__(256) k_mean_any(V* __restrict__ w, int64_t ld_
 
 template <class V>
 __global__ void __launch_bounds__(256) k_mean_any_to(const V* __restrict__ w, int64_t ld_v,
-                                                     int64_t cols_v, int n, V* __restrict__ out) {
+                                                     int64_t cols_v, int n, float div,
+                                                     V* __restrict__ out, int64_t out_ld_v) {
   grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   const V* p = w + static_cast<int64_t>(blockIdx.y) * n * ld_v + c;
-  out[static_cast<int64_t>(blockIdx.y) * ld_v + c] = vdiv(tree_any(p, ld_v, n), static_cast<float>(n));
+  out[static_cast<int64_t>(blockIdx.y) * out_ld_v + c] = vdiv(tree_any(p, ld_v, n), div);
 }
 
 template <class V>
@@ -211,34 +214,38 @@ void launch_mean_pow2(float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
   launch_pdl(k_mean_pow2<LOG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v);
 }
 
+// (The _to launches: rows of w with stride ld_v, rows of out with stride out_ld_v.)
 template <int LOG>
-void launch_mean_pow2_to(const float4* w, int64_t ld_v, int64_t cols_v, int64_t groups, float4* out,
-                         cudaStream_t s) {
+void launch_mean_pow2_to(const float4* w, int64_t ld_v, int64_t cols_v, int64_t groups, float div,
+                         float4* out, int64_t out_ld_v, cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
             static_cast<unsigned>(groups));
-  launch_pdl(k_mean_pow2_to<LOG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, out);
+  launch_pdl(k_mean_pow2_to<LOG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, div, out,
+             out_ld_v);
 }
 
 bool mean_pow2_to_dispatch(int log, const float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
-                           float4* out, cudaStream_t s) {
+                           float div, float4* out, int64_t out_ld_v, cudaStream_t s) {
   switch (log) {
-    case 1: launch_mean_pow2_to<1>(w, ld_v, cols_v, groups, out, s); return true;
-    case 2: launch_mean_pow2_to<2>(w, ld_v, cols_v, groups, out, s); return true;
-    case 3: launch_mean_pow2_to<3>(w, ld_v, cols_v, groups, out, s); return true;
-    case 4: launch_mean_pow2_to<4>(w, ld_v, cols_v, groups, out, s); return true;
-    case 5: launch_mean_pow2_to<5>(w, ld_v, cols_v, groups, out, s); return true;
-    case 6: launch_mean_pow2_to<6>(w, ld_v, cols_v, groups, out, s); return true;
-    case 7: launch_mean_pow2_to<7>(w, ld_v, cols_v, groups, out, s); return true;
+    case 0: launch_mean_pow2_to<0>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 1: launch_mean_pow2_to<1>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 2: launch_mean_pow2_to<2>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 3: launch_mean_pow2_to<3>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 4: launch_mean_pow2_to<4>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 5: launch_mean_pow2_to<5>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 6: launch_mean_pow2_to<6>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
+    case 7: launch_mean_pow2_to<7>(w, ld_v, cols_v, groups, div, out, out_ld_v, s); return true;
     default: return false;
   }
 }
 
 template <class V>
-void launch_mean_any_to(const V* w, int64_t ld_v, int64_t cols_v, int n, int64_t groups, V* out,
-                        cudaStream_t s) {
+void launch_mean_any_to(const V* w, int64_t ld_v, int64_t cols_v, int n, int64_t groups, float div,
+                        V* out, int64_t out_ld_v, cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
             static_cast<unsigned>(groups));
-  launch_pdl(k_mean_any_to<V>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, n, out);
+  launch_pdl(k_mean_any_to<V>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, n, div, out,
+             out_ld_v);
 }
 
 bool mean_pow2_dispatch(int log, float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
@@ -323,19 +330,26 @@ cudaError_t launch_group_mean(float* w, int64_t P, int64_t n, int64_t D, int64_t
 
 cudaError_t launch_group_mean_to(const float* w, int64_t P, int64_t n, int64_t D, int64_t ld,
                                  float* out, cudaStream_t s) {
+  return launch_group_sum_mean_to(w, P, n, D, ld, static_cast<float>(n), out, ld, s);
+}
+
+cudaError_t launch_group_sum_mean_to(const float* w, int64_t rows, int64_t n, int64_t D, int64_t ld,
+                                     float div, float* out, int64_t out_ld, cudaStream_t s) {
   if (D == 0) return cudaSuccess;
-  const int64_t groups = P / n;
+  const int64_t groups = rows / n;
   int64_t head = 0;
-  if (vec_ok(w, ld) && vec_ok(out, ld) && D >= 4) {
+  if (vec_ok(w, ld) && vec_ok(out, out_ld) && D >= 4) {
     head = D & ~int64_t(3);
     const float4* w4 = reinterpret_cast<const float4*>(w);
     float4* o4 = reinterpret_cast<float4*>(out);
     const int log = ilog2_exact(n);
-    if (!(log >= 1 && mean_pow2_to_dispatch(log, w4, ld / 4, head / 4, groups, o4, s)))
-      launch_mean_any_to<float4>(w4, ld / 4, head / 4, static_cast<int>(n), groups, o4, s);
+    if (!(log >= 0 && mean_pow2_to_dispatch(log, w4, ld / 4, head / 4, groups, div, o4, out_ld / 4, s)))
+      launch_mean_any_to<float4>(w4, ld / 4, head / 4, static_cast<int>(n), groups, div, o4,
+                                 out_ld / 4, s);
   }
   if (head < D)
-    launch_mean_any_to<float>(w + head, ld, D - head, static_cast<int>(n), groups, out + head, s);
+    launch_mean_any_to<float>(w + head, ld, D - head, static_cast<int>(n), groups, div, out + head,
+                              out_ld, s);
   return cudaGetLastError();
 }
 

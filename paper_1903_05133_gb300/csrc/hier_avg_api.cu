@@ -71,6 +71,11 @@ struct hier_avg {
   // S > 1): after the step part of the workspace, which is all a single step needs.
   int64_t off_M = 0, ws_step_bytes = 0;
   bool m_ok = false;                          // the bound workspace holds the means
+  // The step that closes a local block inside a round (compact averages only) updates
+  // W_1 for groups of upd_group learners of a cluster and stores their adjacent-pair
+  // tree sum, to the first learner row of each group through tm_gs (1: not used).
+  int upd_group = 1;
+  CUtensorMap tm_gs;
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
   int64_t off_dyn = 0;                        // update kernel's work-item counters
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
@@ -319,6 +324,13 @@ int build_maps(hier_avg* h) {
     if ((rc = make_map(h, &h->tm_wb[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
                        h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
       return rc;
+    if (h->m_ok && l == 0 && h->upd_group > 1) {
+      // group sums of W_1: row g*Q of the parameter matrix, g < P / Q
+      const uint64_t Q = h->upd_group;
+      if ((rc = make_map(h, &h->tm_gs, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P / Q, in * 4,
+                         Q * h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
+        return rc;
+    }
     if (h->m_ok) {
       float* Wm = h->means() + h->woff[l];
       const uint64_t G = P / h->S;
@@ -454,10 +466,15 @@ ha::HeadArgs head_args(hier_avg* h, ParamSrc src) {
 // per step, so after this step every learner row holds its parameters again.
 // next_rows (round_host): recorded once the next step's rows are on the device; the
 // update+forward kernel, which reads them, waits for it.
+// group_out: a compact local average follows this step; the first layer's update may
+// then store group sums of W_1 (h->upd_group learners each) instead of the learner
+// rows' W_1, and *grouped reports whether it did (the average must then read them).
 int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
-            bool from_means = false, cudaEvent_t next_rows = nullptr) {
+            bool from_means = false, cudaEvent_t next_rows = nullptr, bool group_out = false,
+            bool* grouped = nullptr) {
   const int L = h->L, P = h->P, B = h->Bstep;
   if (fused) *fused = false;
+  if (grouped) *grouped = false;
   cudaStream_t s = h->stream;
   int rc;
   const bool means = from_means && h->m_ok;
@@ -625,9 +642,13 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         }, "backward");
       } else {
         a.ctas = kTargetCtas;
-        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
-          return ha::launch_tc_update(wl, ws, hin, h->tm_dz[l + 1], a, s);
+        const int q = group_out && h->m_ok ? h->upd_group : 1;
+        // grouped: W_1 read per learner, its group sums written to row g*q, g < P / q
+        const double gb = q > 1 ? double(P) * h->dims[0] * h->dims[1] * 4.0 * (1.0 - 1.0 / q) : 0.0;
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - gb, flops_gemm(h, l), [&] {
+          return ha::launch_tc_update(wl, q > 1 ? h->tm_gs : ws, hin, h->tm_dz[l + 1], a, q, s);
         }, "backward");
+        if (grouped) *grouped = q > 1;
       }
       if (rc) return rc;
     }
@@ -689,6 +710,25 @@ int do_local_means(hier_avg* h) {
   return h->timed(HA_KERNEL_LOCAL_AVG, 4.0 * h->P * h->ld + 4.0 * (h->P / h->S) * h->ld,
                   double(h->P) * h->ld, [&] {
     return ha::launch_group_mean_to(h->params, h->P, h->S, h->ld, h->ld, h->means(), h->stream);
+  }, "local average");
+}
+
+// The compact local average after a grouped first-layer update: W_1 from the group
+// sums (rows g*Q, g < P / Q, which hold the first log2(Q) levels of every cluster's
+// adjacent-pair tree), the rest of the row from the learner rows.  The tree over a
+// cluster's S / Q group sums has the same levels above them as the tree over its S
+// rows (Q divides S, so every group is a complete, aligned sub-tree), so the means
+// are the bits of do_local_means.
+int do_local_means_grouped(hier_avg* h) {
+  const int64_t P = h->P, S = h->S, Q = h->upd_group, ld = h->ld;
+  const int64_t w1 = static_cast<int64_t>(h->dims[0]) * h->dims[1];   // W_1 at column 0
+  const double bytes = 4.0 * (P / Q) * w1 + 4.0 * P * (ld - w1) + 4.0 * (P / S) * ld;
+  return h->timed(HA_KERNEL_LOCAL_AVG, bytes, double(P) * ld, [&] {
+    ++h->launches;   // two launches
+    cudaError_t e = ha::launch_group_sum_mean_to(h->params, P / Q, S / Q, w1, Q * ld,
+                                                 static_cast<float>(S), h->means(), ld, h->stream);
+    if (e != cudaSuccess) return e;
+    return ha::launch_group_mean_to(h->params + w1, P, S, ld - w1, ld, h->means() + w1, h->stream);
   }, "local average");
 }
 
@@ -807,10 +847,14 @@ int do_round(hier_avg* h, RowFeed* feed = nullptr) {
     }
     const bool block_end = r % h->K1 == 0;              // a local average follows step r
     const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
+    bool grouped = false;
     if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local && compact,
-                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr)))
+                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr,
+                      compact && block_end && r < G, &grouped)))
       return rc;
-    if (r < G && block_end && (rc = compact ? do_local_means(h) : do_local(h))) return rc;
+    if (r < G && block_end &&
+        (rc = grouped ? do_local_means_grouped(h) : compact ? do_local_means(h) : do_local(h)))
+      return rc;
   }
   return G % h->K1 == 0 ? do_local_global(h) : do_global(h);
 }
@@ -973,6 +1017,9 @@ int hier_avg_bind(hier_avg* h, float* params_dev, void* workspace_dev, int64_t w
   h->t = 0;
   h->cursor = 0;
   h->m_ok = h->off_M > 0;
+  h->upd_group = 1;
+  if (h->m_ok && h->S % 2 == 0 && !(h->head && h->L == 1))
+    h->upd_group = h->S % 4 == 0 && ha::tc_update_max_group(h->Bn) >= 4 ? 4 : 2;
   int rc;
   if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_step_bytes, h->stream), "bind: memset"))) return rc;
   if (h->prec == HA_PREC_BF16) {
@@ -1300,6 +1347,7 @@ extern "C" int hier_avg_step_static(hier_avg* h, float* params_dev, const void* 
   if ((rc = h->cuda(cudaMemsetAsync(h->ws, 0, h->ws_step_bytes, h->stream), "step_static: clear")))
     return rc;
   h->m_ok = false;   // the array holds a step's scratch only: rounds average in place
+  h->upd_group = 1;
   if (h->prec == HA_PREC_BF16) {
     if ((rc = h->cuda(ha::tc_configure(), "step_static: kernel attributes"))) return rc;
     if ((rc = h->cuda(ha::head_configure(), "step_static: kernel attributes"))) return rc;

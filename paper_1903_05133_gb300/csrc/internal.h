@@ -50,6 +50,12 @@ cudaError_t launch_group_mean(float* w, int64_t P, int64_t n, int64_t D, int64_t
 // The same means written once per group, to row g of out[P / n, ld] (w unchanged).
 cudaError_t launch_group_mean_to(const float* w, int64_t P, int64_t n, int64_t D, int64_t ld,
                                  float* out, cudaStream_t s);
+// Rows of w (stride ld) in groups of n consecutive rows: the adjacent-pair tree sum of
+// each group divided by div, to row g of out (stride out_ld).  With div = n this is
+// launch_group_mean_to; with rows that are sums of the first tree levels (Q learners
+// each, n = S / Q, div = S) it finishes a local average from them.
+cudaError_t launch_group_sum_mean_to(const float* w, int64_t rows, int64_t n, int64_t D, int64_t ld,
+                                     float div, float* out, int64_t out_ld, cudaStream_t s);
 // The local average (clusters of S) followed by the global average, in one pass.
 cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, int64_t ld,
                                      cudaStream_t s);
@@ -140,8 +146,10 @@ struct TcBwdArgs {
   // claimed dynamically by `ctas` CTAs from dyn[0] (dyn[1] counts the CTAs done; both
   // zero on entry, reset on exit).  k_tc_backward: tiles [0, n_whole) whole, tiles
   // [n_whole, n_tiles) in np_tail pieces of piece_chunks chunks, dX partials and
-  // counters as the forward's.  k_tc_update: runs of up to 8 chunks.
+  // counters as the forward's.  k_tc_update: runs of up to `run` chunks (set by its
+  // launcher).
   int ctas, n_tiles, s_tiles;
+  int run;
   int n_whole, np_tail, piece_chunks;
   float* part;
   int* counters;
@@ -158,10 +166,14 @@ cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_s
                                const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
                                int P, cudaStream_t s);
 // The first layer's backward (no dX): dW, update and store only, units claimed
-// dynamically (a.dyn zero on entry; reset by the kernel on exit).
+// dynamically (a.dyn zero on entry; reset by the kernel on exit).  a.n_tiles = P *
+// s_tiles.  group = 1: every learner's W is stored through w_store (row j).  group = 2
+// or 4 (at most tc_update_max_group(Bn)): learners g*group .. g*group+group-1 are
+// updated together and only their adjacent-pair tree sum is stored, to row g of w_store.
 cudaError_t launch_tc_update(const CUtensorMap& w_load, const CUtensorMap& w_store,
                              const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
-                             cudaStream_t s);
+                             int group, cudaStream_t s);
+int tc_update_max_group(int Bn);
 // The first layer's backward (dW, update, store) fused with the next step's first-layer
 // forward (H_1' = relu(X' W_1'^T + b_1), schedule and arithmetic of launch_tc_forward):
 // h_cur holds this step's batch rows (a.hc_row0 ..), x_next the next step's (a.x_row0 ..).

@@ -1154,29 +1154,63 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
 // kRun chunks of one tile, claimed by warp 4 from a global counter and announced to
 // the other roles through a small queue in shared memory; the last CTA to finish
 // resets the counters.  Roles as in k_tc_backward, without the dX path.
+//
+// Q > 1 (the step that closes a local block, followed by a compact local average): a
+// work item covers the same tile and chunks of Q consecutive learners of a cluster
+// (learners q*Q .. q*Q+Q-1).  Each learner's updated chunk is formed as for Q = 1, and
+// the converter threads add the Q of them in the first log2(Q) levels of the
+// adjacent-pair tree of the local average ((w0 + w1) for Q = 2; (w0 + w1) + (w2 + w3)
+// for Q = 4), so that only this group sum is stored, to row q of the group-sum buffer
+// (store map) instead of Q learner rows.  The local average finishes the tree from
+// the group sums: the bits of the literal update and average.
 constexpr int kRun = 8;                 // chunks per work item
 __host__ __device__ constexpr int upd_smem(int Bn) { return bwd_smem(Bn) + 512; }
 static_assert(upd_smem(64) <= kBwdSmemMax && upd_smem(48) <= kBwdSmemMax &&
                   upd_smem(32) <= kBwdSmemMax && upd_smem(16) <= kBwdSmemMax,
               "update kernel shared-memory plan");
+// Group layout (Q > 1): W ring (4 slots) | 2 x Q H tiles | dZ ring | barriers and queue.
+__host__ __device__ constexpr int updg_h_off(int Q, int Bn) { return (void)Q, (void)Bn, 4 * kBwdWf32; }
+__host__ __device__ constexpr int updg_z_off(int Q, int Bn) { return updg_h_off(Q, Bn) + 2 * Q * 2 * Bn * 128; }
+__host__ __device__ constexpr int updg_zring(int Q, int Bn) {
+  return (kBwdSmemMax - 1024 - kBarBytes - updg_z_off(Q, Bn)) / (Bn * 128) < kBwdZRingMax
+             ? (kBwdSmemMax - 1024 - kBarBytes - updg_z_off(Q, Bn)) / (Bn * 128)
+             : kBwdZRingMax;
+}
+__host__ __device__ constexpr int updg_bar_off(int Q, int Bn) {
+  return updg_z_off(Q, Bn) + updg_zring(Q, Bn) * Bn * 128;
+}
+__host__ __device__ constexpr int updg_smem(int Q, int Bn) { return updg_bar_off(Q, Bn) + kBarBytes + 1024; }
+static_assert(updg_zring(4, 32) >= 4 && updg_smem(4, 32) <= kBwdSmemMax && updg_zring(4, 16) >= 4 &&
+                  updg_smem(4, 16) <= kBwdSmemMax && updg_zring(2, 64) >= 4 &&
+                  updg_smem(2, 64) <= kBwdSmemMax && updg_zring(2, 48) >= 4 &&
+                  updg_smem(2, 48) <= kBwdSmemMax,
+              "group update kernel shared-memory plan");
 
-__global__ void __launch_bounds__(kBwdThreads, 1)
+// Q > 1: eight converter warps (0-3 and 8-11), each thread half of a column.
+__host__ __device__ constexpr int upd_conv_warps(int Q) { return Q == 1 ? kBwdConv / 32 : 8; }
+__host__ __device__ constexpr int upd_threads(int Q) { return 128 + 32 * upd_conv_warps(Q); }
+
+template <int Q>
+__global__ void __launch_bounds__(upd_threads(Q), 1)
     k_tc_update(const __grid_constant__ CUtensorMap tm_wl, const __grid_constant__ CUtensorMap tm_ws,
                 const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_dz,
                 const TcBwdArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kChunks = a.run;                               // chunks per item and learner
   const int nc = (a.out + 63) / 64;
-  const int rpt = (nc + kRun - 1) / kRun;                  // work items per tile
-  const int n_items = a.n_tiles * rpt;
-  const int nw = bwd_wring(a.Bn), nz = bwd_zring(a.Bn);
+  const int rpt = (nc + kChunks - 1) / kChunks;            // work items per tile
+  const int n_items = a.n_tiles / Q * rpt;                 // tiles of learner groups
+  const int nw = Q == 1 ? bwd_wring(a.Bn) : 4;
+  const int nz = Q == 1 ? bwd_zring(a.Bn) : updg_zring(Q, a.Bn);
   const int tbytes = a.Bn * 128;
-  uint8_t* h_base = smem + bwd_h_off(a.Bn);
-  uint8_t* z_base = smem + bwd_z_off(a.Bn);
-  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + bwd_bar_off(a.Bn));
+  uint8_t* h_base = smem + (Q == 1 ? bwd_h_off(a.Bn) : updg_h_off(Q, a.Bn));
+  uint8_t* z_base = smem + (Q == 1 ? bwd_z_off(a.Bn) : updg_z_off(Q, a.Bn));
+  uint8_t* bar_base = smem + (Q == 1 ? bwd_bar_off(a.Bn) : updg_bar_off(Q, a.Bn));
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(bar_base);
   uint64_t* wempty = wfull + kBwdWRingMax;   // chunk stored back (TMA has read it)
-  uint64_t* upd = wempty + kBwdWRingMax;     // chunk updated in shared memory
+  uint64_t* upd = wempty + kBwdWRingMax;     // chunk updated (or read) in shared memory
   uint64_t* zfull = upd + kBwdWRingMax;
   uint64_t* zempty = zfull + kBwdZRingMax;   // dZ tile consumed by the MMA
   uint64_t* hfull = zempty + kBwdZRingMax;   // [2]
@@ -1185,19 +1219,21 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   uint64_t* dwfree = dwdone + 2;             // [2]
   uint64_t* done = dwfree + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
-  uint64_t* qfull = reinterpret_cast<uint64_t*>(smem + bwd_bar_off(a.Bn) + 512);
+  uint64_t* qfull = reinterpret_cast<uint64_t*>(bar_base + 512);
   uint64_t* qempty = qfull + kQueue;         // read by the 7 consuming warps
   int* items = reinterpret_cast<int*>(qempty + kQueue);
   auto wf = [&](int s) { return smem + s * kBwdWf32; };
-  auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
+  // member m's H tile (two 64-feature boxes) in buffer hbuf
+  auto hb = [&](int hbuf, int m) { return h_base + (hbuf * Q + m) * 2 * tbytes; };
   auto zb = [&](int s) { return z_base + s * tbytes; };
-  constexpr int kConsumers = 3 + kBwdConv / 32;             // dZ, MMA, store + converter warps
+  constexpr int kConv = upd_conv_warps(Q);
+  constexpr int kConsumers = 3 + kConv;                     // dZ, MMA, store + converter warps
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kBwdWRingMax; ++s) {
       mbar_init(&wfull[s], 1);
       mbar_init(&wempty[s], 1);
-      mbar_init(&upd[s], kBwdConv / 32);
+      mbar_init(&upd[s], kConv);
     }
     for (int s = 0; s < kBwdZRingMax; ++s) {
       mbar_init(&zfull[s], 1);
@@ -1207,7 +1243,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       mbar_init(&hfull[b], 1);
       mbar_init(&hempty[b], 1);
       mbar_init(&dwdone[b], 1);
-      mbar_init(&dwfree[b], kBwdConv / 32);
+      mbar_init(&dwfree[b], kConv);
     }
     for (int q = 0; q < kQueue; ++q) {
       mbar_init(&qfull[q], 1);
@@ -1236,16 +1272,18 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     if (lane == 0) mbar_arrive(&qempty[q]);
     return it;
   };
-  // Chunks [c_lo, c_hi) of tile `tile` for work item `it`.
+  // Group tile `tile` (group tile / s_tiles, input features 128 * (tile % s_tiles) ..)
+  // and its chunks [c_lo, c_hi) for work item `it`.
   auto decode = [&](int it, int& tile, int& c_lo, int& c_hi) {
     tile = it / rpt;
-    c_lo = (it - tile * rpt) * kRun;
-    c_hi = c_lo + kRun < nc ? c_lo + kRun : nc;
+    c_lo = (it - tile * rpt) * kChunks;
+    c_hi = c_lo + kChunks < nc ? c_lo + kChunks : nc;
   };
 
   if (warp == 4) {
     if (lane == 0) {
-      // claim, announce, and load: W chunks and each item's H tile
+      // claim, announce, and load: each item's H tiles, then per chunk the W chunks of
+      // the group's learners in order
       tma_prefetch_desc(&tm_wl);
       tma_prefetch_desc(&tm_h);
       const uint64_t stream = l2_stream_policy(a.w_stream != 0);
@@ -1262,19 +1300,23 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         next = atomicAdd(a.dyn, 1);           // the next claim, hidden behind these loads
         int tile, c_lo, c_hi;
         decode(it, tile, c_lo, c_hi);
-        const int j = tile / a.s_tiles, i0 = (tile - j * a.s_tiles) * 128;
+        const int g = tile / a.s_tiles, i0 = (tile - g * a.s_tiles) * 128, j0 = g * Q;
         const int hbuf = kt & 1;
         if (kt >= 2 && !mbar_wait(&hempty[hbuf], ((kt >> 1) - 1) & 1, a.err)) break;
-        mbar_arrive_expect_tx(&hfull[hbuf], 2 * tbytes);
-        tma_load_3d(hb(hbuf), &tm_h, &hfull[hbuf], i0, a.h_row0, j);
-        tma_load_3d(hb(hbuf) + tbytes, &tm_h, &hfull[hbuf], i0 + 64, a.h_row0, j);
+        mbar_arrive_expect_tx(&hfull[hbuf], Q * 2 * tbytes);
+        for (int m = 0; m < Q; ++m) {
+          tma_load_3d(hb(hbuf, m), &tm_h, &hfull[hbuf], i0, a.h_row0, j0 + m);
+          tma_load_3d(hb(hbuf, m) + tbytes, &tm_h, &hfull[hbuf], i0 + 64, a.h_row0, j0 + m);
+        }
         ++kt;
-        for (int c = c_lo; c < c_hi; ++c, ++i) {
-          const int s = i % nw;
-          if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
-          mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
-          tma_load_3d_hint(wf(s), &tm_wl, &wfull[s], i0, c * 64, j / a.src_div, stream);
-          issued = i + 1;
+        for (int c = c_lo; c < c_hi && ok; ++c) {
+          for (int m = 0; m < Q; ++m, ++i) {
+            const int s = i % nw;
+            if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+            mbar_arrive_expect_tx(&wfull[s], kBwdWf32);
+            tma_load_3d_hint(wf(s), &tm_wl, &wfull[s], i0, c * 64, (j0 + m) / a.src_div, stream);
+            issued = i + 1;
+          }
         }
       }
       for (int u = issued - nw > 0 ? issued - nw : 0; u < issued; ++u)
@@ -1290,13 +1332,16 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       if (lane == 0) {
         int tile, c_lo, c_hi;
         decode(it, tile, c_lo, c_hi);
-        const int j = tile / a.s_tiles;
-        for (int c = c_lo; c < c_hi; ++c, ++i) {
-          const int s = i % nz;
-          if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) break;
-          mbar_arrive_expect_tx(&zfull[s], tbytes);
-          tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j);
-          issued = i + 1;
+        const int j0 = tile / a.s_tiles * Q;
+        bool ok = true;
+        for (int c = c_lo; c < c_hi && ok; ++c) {
+          for (int m = 0; m < Q; ++m, ++i) {
+            const int s = i % nz;
+            if (i >= nz && !mbar_wait(&zempty[s], ((i / nz) - 1) & 1, a.err)) { ok = false; break; }
+            mbar_arrive_expect_tx(&zfull[s], tbytes);
+            tma_load_3d(zb(s), &tm_dz, &zfull[s], c * 64, 0, j0 + m);
+            issued = i + 1;
+          }
         }
       }
       __syncwarp();
@@ -1305,6 +1350,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       for (int u = issued - nz > 0 ? issued - nz : 0; u < issued; ++u)
         mbar_wait(&zfull[u % nz], (u / nz) & 1, a.err);
   } else if (warp == 7) {
+    // Q = 1: store each updated chunk, freeing its slot one store behind.  Q > 1: free
+    // the slots of the first Q - 1 learners as soon as they are read, store the group
+    // sum (row g of the store map) and free its slot once the store has read it.
     const uint64_t stream = l2_stream_policy(a.w_stream != 0);
     int i = 0;
     for (int k = 0;; ++k) {
@@ -1313,15 +1361,27 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       if (lane == 0) {
         int tile, c_lo, c_hi;
         decode(it, tile, c_lo, c_hi);
-        const int j = tile / a.s_tiles, i0 = (tile - j * a.s_tiles) * 128;
-        for (int c = c_lo; c < c_hi; ++c, ++i) {
-          const int s = i % nw;
-          if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) break;
-          tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, j, stream);
-          tma_store_commit();
-          if (i > 0) {
-            tma_store_wait_read_1();
-            mbar_arrive(&wempty[(i - 1) % nw]);
+        const int g = tile / a.s_tiles, i0 = (tile - g * a.s_tiles) * 128;
+        bool ok = true;
+        for (int c = c_lo; c < c_hi && ok; ++c) {
+          for (int m = 0; m < Q; ++m, ++i) {
+            const int s = i % nw;
+            if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) { ok = false; break; }
+            if constexpr (Q == 1) {
+              tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, g, stream);
+              tma_store_commit();
+              if (i > 0) {
+                tma_store_wait_read_1();
+                mbar_arrive(&wempty[(i - 1) % nw]);
+              }
+            } else if (m + 1 < Q) {
+              mbar_arrive(&wempty[s]);
+            } else {
+              tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, g, stream);
+              tma_store_commit();
+              tma_store_wait_read_all();
+              mbar_arrive(&wempty[s]);
+            }
           }
         }
       }
@@ -1329,7 +1389,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     }
     if (lane == 0) {
       tma_store_wait_read_all();   // (before the shared memory is released)
-      if (i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
+      if (Q == 1 && i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
     }
   } else if (warp == 5) {
     const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
@@ -1344,20 +1404,21 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         int tile, c_lo, c_hi;
         decode(it, tile, c_lo, c_hi);
         if (!mbar_wait(&hfull[kt & 1], (kt >> 1) & 1, a.err)) ok = false;
-        const uint32_t hs = smem_u32(hb(kt & 1));
-        for (int c = c_lo; c < c_hi && ok; ++c, ++i) {
-          const int sz = i % nz, b = i & 1;
-          if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) { ok = false; break; }
-          if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t zs = smem_u32(zb(sz));
-          for (int kk = 0; kk < kb; ++kk)
-            tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
-                        umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
-          tc_commit(&dwdone[b]);
-          tc_commit(&zempty[sz]);
+        for (int c = c_lo; c < c_hi && ok; ++c) {
+          for (int m = 0; m < Q; ++m, ++i) {
+            const int sz = i % nz, b = i & 1;
+            if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) { ok = false; break; }
+            if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t hs = smem_u32(hb(kt & 1, m)), zs = smem_u32(zb(sz));
+            for (int kk = 0; kk < kb; ++kk)
+              tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
+                          umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+            tc_commit(&dwdone[b]);
+            tc_commit(&zempty[sz]);
+          }
         }
-        tc_commit(&hempty[kt & 1]);          // the H tile is free once these MMAs are
+        tc_commit(&hempty[kt & 1]);          // the H tiles are free once these MMAs are
       }
       ok = __all_sync(0xffffffffu, ok);
     }
@@ -1365,7 +1426,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       tc_commit(done);
       mbar_wait(done, 0, a.err);
     }
-  } else {
+  } else if constexpr (Q == 1) {
     // ---- warps 0-3: thread t owns input feature i0 + t of the current chunk
     const int t = threadIdx.x;
     const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
@@ -1376,7 +1437,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       if (it < 0) break;
       int tile, c_lo, c_hi;
       decode(it, tile, c_lo, c_hi);
-      for (int c = c_lo; c < c_hi; ++c, ++i) {
+      for (int c = c_lo; c < c_hi && ok; ++c, ++i) {
         const int sw = i % nw, b = i & 1;
         if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
         float* w = reinterpret_cast<float*>(wf(sw));
@@ -1385,6 +1446,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         for (int o = 0; o < 64; ++o) wv[o] = w[o * 128 + t];
         if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
         tc_fence_after();
+        // the updated column: w - lr * dW, IEEE multiply then subtract
 #pragma unroll
         for (int qb = 0; qb < 4; ++qb) {
           float d[16];
@@ -1401,6 +1463,62 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&upd[sw]);
+      }
+    }
+  } else {
+    // ---- warps 0-3 and 8-11: thread (warp % 4, lane) owns input feature i0 + t of the
+    // chunk, warps 0-3 its outputs 0-31, warps 8-11 its outputs 32-63
+    const int t = 32 * (warp & 3) + lane, o0 = warp >= 8 ? 32 : 0;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+    int i = 0;
+    bool ok = true;
+    float s0[32], s1[32];                    // partial sums of the pair tree
+    for (int k = 0; ok; ++k) {
+      const int it = take(k);
+      if (it < 0) break;
+      int tile, c_lo, c_hi;
+      decode(it, tile, c_lo, c_hi);
+      for (int c = c_lo; c < c_hi && ok; ++c) {
+        for (int m = 0; m < Q; ++m, ++i) {
+          const int sw = i % nw, b = i & 1;
+          if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+          float* w = reinterpret_cast<float*>(wf(sw)) + o0 * 128;
+          if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
+          // learner m's updated column, w - lr * dW (IEEE multiply then subtract), goes
+          // into pair partial m / 2 of the tree (s0 or s1): the first of a pair starts
+          // it, the second is added to it
+          const bool second = (m & 1) != 0, upper = Q == 4 && m >= 2;
+#pragma unroll
+          for (int qb = 0; qb < 2; ++qb) {
+            float d[16];
+            tmem_ld16(tbase + kBwdTmemW + 64 * b + o0 + 16 * qb, d);
+            float v[16];
+#pragma unroll
+            for (int q = 0; q < 16; ++q) v[q] = w[(16 * qb + q) * 128 + t];
+            tmem_ld_wait();
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+              const int o = 16 * qb + q;
+              const float u = __fsub_rn(v[q], __fmul_rn(a.lr, d[q]));
+              if (upper)
+                s1[o] = second ? __fadd_rn(s1[o], u) : u;
+              else
+                s0[o] = second ? __fadd_rn(s0[o], u) : u;
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&dwfree[b]);
+          if (m + 1 == Q) {
+            // the group sum (w0 + w1) or ((w0 + w1) + (w2 + w3)) replaces the last slot
+#pragma unroll
+            for (int o = 0; o < 32; ++o) w[o * 128 + t] = Q == 4 ? __fadd_rn(s0[o], s1[o]) : s0[o];
+            fence_proxy_async_smem();
+          }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&upd[sw]);
+        }
       }
     }
   }
@@ -2040,7 +2158,11 @@ cudaError_t tc_configure() {
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_tc_update, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  e = cudaFuncSetAttribute(k_tc_update<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tc_update<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tc_update<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(k_tc_update_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               kFwdSmemMax);
@@ -2069,11 +2191,27 @@ cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_s
 
 cudaError_t launch_tc_update(const CUtensorMap& w_load, const CUtensorMap& w_store,
                              const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,
-                             cudaStream_t s) {
+                             int group, cudaStream_t s) {
+  // Items of kRun chunks per learner, unless a group of learners then leaves fewer than
+  // 4 items per CTA: then kRun / group chunks per learner (the same work per item).
+  TcBwdArgs b = a;
+  const int nc = (a.out + 63) / 64;
+  b.run = kRun;
+  if (group > 1 && static_cast<int64_t>(a.n_tiles / group) * ((nc + kRun - 1) / kRun) < 4 * a.ctas)
+    b.run = kRun / group > 0 ? kRun / group : 1;
   // no CTA waits on another: an ordinary (programmatically serialised) launch
-  return launch_pdl(k_tc_update, dim3(a.ctas), dim3(kBwdThreads), upd_smem(a.Bn), s, false, 1,
-                    w_load, w_store, h_in, dz, a);
+  if (group == 4 && a.Bn <= 32)
+    return launch_pdl(k_tc_update<4>, dim3(a.ctas), dim3(upd_threads(4)), updg_smem(4, a.Bn), s, false, 1,
+                      w_load, w_store, h_in, dz, b);
+  if (group == 2)
+    return launch_pdl(k_tc_update<2>, dim3(a.ctas), dim3(upd_threads(2)), updg_smem(2, a.Bn), s, false, 1,
+                      w_load, w_store, h_in, dz, b);
+  if (group != 1) return cudaErrorInvalidValue;
+  return launch_pdl(k_tc_update<1>, dim3(a.ctas), dim3(upd_threads(1)), upd_smem(a.Bn), s, false, 1,
+                    w_load, w_store, h_in, dz, b);
 }
+
+int tc_update_max_group(int Bn) { return Bn <= 32 ? 4 : 2; }
 
 cudaError_t launch_tc_update_forward(const CUtensorMap& w_load, const CUtensorMap& w_store,
                                      const CUtensorMap& h_cur, const CUtensorMap& x_next,

@@ -276,13 +276,36 @@ def test_full_run_against_oracle(w):
     assert ha.get_step() == w.rounds * w.K1 * w.K2
 
 
+# The step that closes a local block inside round() updates W_1 for groups of Q = 4
+# learners of a cluster (2 where S is not a multiple of 4 or the batch exceeds 32) and
+# stores only their sum in the first levels of the averaging tree; the local average
+# finishes the tree from the S / Q group sums.  Cases: Q = 4 with S = 8 (two group sums
+# per cluster); Q = 2 with S = 6 (three per cluster: the generic tree) and a ragged
+# 200-input layer; Q = 4 with S = 12 and K1 = 1 (every step both reads the cluster
+# means and writes group sums); Q = 2 because the batch is 64.
+GROUP_S8 = configs.Workload("mlp_bf16_group4_S8", P=16, S=8, K1=2, K2=3, rounds=1,
+                            dims=(256, 192, 10), precision="bf16", N=128, B=32, lr=0.05,
+                            sigma_mu=0.1, init="he")
+GROUP_S6 = configs.Workload("mlp_bf16_group2_S6", P=12, S=6, K1=2, K2=2, rounds=1,
+                            dims=(200, 136, 13), precision="bf16", N=144, B=48, lr=0.05,
+                            sigma_mu=0.1, init="he")
+GROUP_S12_K1 = configs.Workload("mlp_bf16_group4_S12_K1_1", P=24, S=12, K1=1, K2=3, rounds=1,
+                                dims=(128, 64, 10), precision="bf16", N=64, B=16, lr=0.05,
+                                sigma_mu=0.1, init="he")
+GROUP_B64 = configs.Workload("mlp_bf16_group2_B64", P=8, S=4, K1=2, K2=2, rounds=1,
+                             dims=(256, 128, 10), precision="bf16", N=256, B=64, lr=0.05,
+                             sigma_mu=0.1, init="he")
+
+
 # round() writes each intermediate local average as one mean row per cluster, read by
 # the next step, and fuses the last local average into the global one; the literal
-# sequence writes every row each time.  Cases: clusters of 2; clusters of 3 over a
-# ragged three-layer net (the generic, non-power-of-two averaging path, with K1 = 1: a
-# compact average after every step but the last); 5 clusters of 4 (a global tree over
-# a non-power-of-two count of clusters), head slices of 128 features.
-@pytest.mark.parametrize("w", [SMALL_BF16, RAGGED_BF16.replace(K2=3), HEAD_F128],
+# sequence writes every row each time.  Cases: clusters of 2 (group sums of 2: one per
+# cluster); clusters of 3 over a ragged three-layer net (the generic, non-power-of-two
+# averaging path, with K1 = 1: a compact average after every step but the last; no
+# groups); 5 clusters of 4 (a global tree over a non-power-of-two count of clusters),
+# head slices of 128 features; the group cases above.
+@pytest.mark.parametrize("w", [SMALL_BF16, RAGGED_BF16.replace(K2=3), HEAD_F128, GROUP_S8,
+                               GROUP_S6, GROUP_S12_K1, GROUP_B64],
                          ids=lambda w: w.name)
 def test_literal_sequence_equals_round(w):
     # step/local_average/global_average in Algorithm 1's order give the same bits
@@ -342,8 +365,9 @@ def test_fused_next_forward_equals_steps(w):
         ha2.local_average()
     ha2.global_average()
     # the literal sequence launches every kernel; round() saves the fused forwards and
-    # fuses the last local average into the global one
-    saved = n_fused + 1
+    # fuses the last local average into the global one, and takes each local average
+    # inside the round from group sums of W_1 in a launch of its own (S even)
+    saved = n_fused + 1 - (w.K2 - 1 if w.S % 2 == 0 else 0)
     assert ha2.launches() - n1 == n_round + saved
     ha1.check()
     ha2.check()
