@@ -145,14 +145,34 @@ struct FwdItem {
   int tau, c_lo, c_hi, piece, np;
 };
 
+// Tiles per learner and the row divisor of the weights a kernel reads (> 1: the
+// learners of a cluster read the same row of the cluster means).
+__device__ __forceinline__ int item_span(const TcFwdArgs& a) { return a.o_tiles; }
+__device__ __forceinline__ int item_span(const TcBwdArgs& a) { return a.s_tiles; }
+__device__ __forceinline__ int item_div(const TcFwdArgs& a) { return a.w_div; }
+__device__ __forceinline__ int item_div(const TcBwdArgs& a) { return a.src_div; }
+
 // Work item `it` of the dynamic schedule: items [0, n_whole) are the whole tiles
-// [0, n_whole) in tile order; then come the pieces of the tail tiles [n_whole,
-// n_tiles), tile by tile, the pieces of a tile in order.
+// [0, n_whole); then come the pieces of the tail tiles [n_whole, n_tiles), tile by
+// tile, the pieces of a tile in order.  Whole tiles go in tile order, except when the
+// learners of a cluster share their weights (item_div > 1): within each cluster whose
+// tiles are all whole, its learners' tiles with the same weight tile are claimed one
+// after the other, so that they stream the same weight rows at about the same time and
+// L2 serves all but the first.  (The split into whole and tail tiles is unchanged, so
+// every tile is summed the same way.)
 template <class Args>
 __device__ __forceinline__ FwdItem fwd_item(const Args& a, int nk, int it) {
   FwdItem f;
   if (it < a.n_whole) {
     f.tau = it;
+    const int S = item_div(a);
+    if (S > 1) {
+      const int span = item_span(a), blk = S * span, c = it / blk;
+      if ((c + 1) * blk <= a.n_whole) {
+        const int r = it - c * blk, o = r / S, m = r - o * S;
+        f.tau = c * blk + m * span + o;
+      }
+    }
     f.c_lo = 0;
     f.c_hi = nk;
     f.piece = 0;
@@ -414,9 +434,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 
   if (warp == 8) {
     if (lane == 0) {
-      // claim (dynamic), announce, and stream the weight tiles
+      // claim (dynamic), announce, and stream the weight tiles (kept in L2 as usual when
+      // the learners of a cluster read the same ones)
       tma_prefetch_desc(&tm_w);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0 && a.w_div == 1);
       int i = 0, issued = 0;
       bool ok = true;
       int next = dyn ? atomicAdd(a.dyn, 1) : 0;
@@ -887,7 +908,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       // its first W chunk, then its W chunks
       tma_prefetch_desc(&tm_wl);
       tma_prefetch_desc(&tm_h);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0 && a.src_div == 1);
       int i = 0, issued = 0;
       bool ok = true;
       int next = atomicAdd(a.dyn, 1);
@@ -1694,7 +1715,7 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     if (lane == 0) {
       // claim (dynamic), announce, and stream the weight tiles
       tma_prefetch_desc(&tm_wl);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      const uint64_t stream = l2_stream_policy(a.w_stream != 0 && a.w_div == 1);
       int i = 0, issued = 0;
       bool ok = true;
       int next = dyn ? atomicAdd(a.dyn, 1) : 0;
