@@ -81,6 +81,7 @@ struct hier_avg {
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
   std::vector<int> fwd_cq;                    // per layer: cluster split factor (1 = dynamic)
   std::vector<int> fwd_whole, fwd_np;         // per layer (dynamic): whole tiles, tail pieces
+  int fwd_group = 1;                          // learners per grouped forward after an average
   std::vector<int> bwd_ctas, bwd_tiles;       // per layer: CTAs, input slices of 128
   std::vector<int> bwd_whole, bwd_np;         // per layer: whole tiles, tail pieces
   bool fused_xent = false;                    // d_L <= 128: CE in the last forward epilogue
@@ -207,6 +208,7 @@ int plan_layout(hier_avg* h) {
     // per SM of a GB300 (152).  They depend on the shapes only, so the summation
     // order of split tiles is the same on every GPU.  Forward tile = 128 outputs x
     // 64-input chunks; backward tile = 128 inputs x 64-output chunks.
+    h->fwd_group = h->S > 1 ? ha::tc_forward_group_size(h->S, h->Bn) : 1;
     h->fwd_ctas.assign(L, 1);
     h->fwd_tiles.assign(L, 1);
     h->fwd_cq.assign(L, 1);
@@ -237,7 +239,12 @@ int plan_layout(hier_avg* h) {
         // and the update+forward sum every H_1 entry the same way.  Later layers keep
         // whole tiles: there a piece's partial round trip costs more than the balance
         // gains (measured).
-        const int64_t t_tail = l == 0 ? std::min<int64_t>(ftiles * P, kTargetCtas) : 0;
+        // (With groups of G learners forwarded together after a compact average, the
+        // tail is rounded down to whole groups, at least one: the grouped kernel splits
+        // the same tiles.  Rounding up measured slightly slower.)
+        const int64_t gt = h->fwd_group * ftiles;
+        const int64_t t_tail =
+            l == 0 ? std::min<int64_t>(ftiles * P, std::max<int64_t>(gt, kTargetCtas / gt * gt)) : 0;
         const int64_t np = (nk + kPieceChunks - 1) / kPieceChunks;
         h->fwd_whole[l] = static_cast<int>(ftiles * P - t_tail);
         h->fwd_np[l] = static_cast<int>(np);
@@ -409,6 +416,13 @@ double bytes_backward(const hier_avg* h, int l) {
   return P * (in * out * 8.0 + B * in * act + B * out * act + dx);
 }
 
+// Right after a compact local average the S learners of a cluster read one row of
+// means: the weights of layer l count once per cluster, not once per learner.
+double shared_w_bytes(const hier_avg* h, int l, bool means) {
+  if (!means) return 0.0;
+  return double(h->P) * h->dims[l] * h->dims[l + 1] * 4.0 * (1.0 - 1.0 / h->S);
+}
+
 // Algorithmic flops of the learner-step products (2 per multiply-add): one
 // [B x in] x [in x out] product per learner for the forward, dW and dX each.
 double flops_gemm(const hier_avg* h, int l) {
@@ -536,15 +550,29 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       }
       a.err = h->err_word();
       const CUtensorMap& hin = a.x_direct ? h->tm_x : h->tm_h[l];
-      rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l), flops_gemm(h, l), [&] {
-        return ha::launch_tc_forward(means ? h->tm_wf_m[l] : h->tm_wf[l], hin, a, P, s);
-      }, "forward");
+      // Right after a compact local average: groups of G learners of a cluster share the
+      // cluster mean's weights, forwarded as one product per weight tile.
+      const int G = h->fwd_group;
+      if (means && G > 1 && a.cq == 1 && a.mode != 2 && a.n_whole % (G * a.o_tiles) == 0) {
+        const int gw = a.n_whole / G;
+        a.ctas = static_cast<int>(std::min<int64_t>(kTargetCtas, gw + int64_t(a.n_tiles / G - gw) * a.np_tail));
+        rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l) - shared_w_bytes(h, l, true),
+                      flops_gemm(h, l), [&] {
+          return ha::launch_tc_forward_group(h->tm_wf_m[l], hin, a, G, s);
+        }, "forward");
+      } else {
+        rc = h->timed(HA_KERNEL_FORWARD, bytes_forward(h, l) - shared_w_bytes(h, l, means),
+                      flops_gemm(h, l), [&] {
+          return ha::launch_tc_forward(means ? h->tm_wf_m[l] : h->tm_wf[l], hin, a, P, s);
+        }, "forward");
+      }
       if (rc) return rc;
     }
     const int C = h->dims[L];
     if (h->head) {
       const ha::HeadArgs a = head_args(h, src);
-      const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0));
+      const double hb = double(P) * (8.0 * C * a.in + 2.0 * B * a.in * 2 + (L > 1 ? 4.0 * B * a.in : 0)) -
+                        shared_w_bytes(h, L - 1, means);
       const double hf = flops_gemm(h, L - 1) * (L > 1 ? 3 : 2);   // forward, dW (, dX)
       rc = h->timed(HA_KERNEL_HEAD, hb, hf, [&] { return ha::launch_head(a, P, s); }, "head");
       if (rc) return rc;
@@ -625,7 +653,8 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.err = h->err_word();
         if (next_rows && (rc = h->cuda(cudaStreamWaitEvent(s, next_rows, 0), "round_host: wait for the rows")))
           return rc;
-        rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h), 2 * flops_gemm(h, 0), [&] {
+        rc = h->timed(HA_KERNEL_UPDATE_FORWARD, bytes_update_forward(h) - shared_w_bytes(h, 0, means),
+                      2 * flops_gemm(h, 0), [&] {
           return ha::launch_tc_update_forward(means ? h->tm_wf_m[0] : h->tm_wf[0], h->tm_wf[0], hin,
                                               h->tm_x, h->tm_dz[1], f, s);
         }, "update+forward");
@@ -637,7 +666,8 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       // runs of 8 chunks, claimed dynamically (measured faster than the backward
       // kernel's items for short layers too: 3072-512-10 round 0.859 -> 0.850 ms).
       if (a.has_dx) {
-        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l), flops_gemm(h, l) * (l > 0 ? 2 : 1), [&] {
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - shared_w_bytes(h, l, means),
+                      flops_gemm(h, l) * 2, [&] {
           return ha::launch_tc_backward(wl, ws, hin, h->tm_dz[l + 1], a, P, s);
         }, "backward");
       } else {
@@ -645,7 +675,8 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         const int q = group_out && h->m_ok ? h->upd_group : 1;
         // grouped: W_1 read per learner, its group sums written to row g*q, g < P / q
         const double gb = q > 1 ? double(P) * h->dims[0] * h->dims[1] * 4.0 * (1.0 - 1.0 / q) : 0.0;
-        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - gb, flops_gemm(h, l), [&] {
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - gb - shared_w_bytes(h, l, means),
+                      flops_gemm(h, l), [&] {
           return ha::launch_tc_update(wl, q > 1 ? h->tm_gs : ws, hin, h->tm_dz[l + 1], a, q, s);
         }, "backward");
         if (grouped) *grouped = q > 1;

@@ -161,6 +161,15 @@ int tc_bwd_smem_bytes();
 cudaError_t tc_configure();   // raises the dynamic shared-memory limits once
 cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                               const TcFwdArgs& a, int P, cudaStream_t s);
+// The forward of groups of G learners that share their weights (the first step after
+// a compact local average, a.w_div = a.b_div = S, G | S): one product of each weight
+// tile with the G stacked batch tiles, bit-identical to launch_tc_forward.  Dynamic
+// schedule only (a.cq == 1), modes 0 and 1; a.n_whole must be a multiple of
+// G * a.o_tiles; a.ctas CTAs claim (n_whole + (n_tiles - n_whole) * np_tail) / G items.
+cudaError_t launch_tc_forward_group(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
+                                    const TcFwdArgs& a, int G, cudaStream_t s);
+// The largest G <= 128 / Bn dividing S (1: none above 1).
+int tc_forward_group_size(int S, int Bn);
 // W is loaded through w_load (row j / a.src_div) and stored through w_store (row j).
 cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_store,
                                const CUtensorMap& h_in, const CUtensorMap& dz, const TcBwdArgs& a,

@@ -64,11 +64,8 @@ namespace {
 // plus (fused cross-entropy only) a staging area for the epilogue.  A chunk takes
 // about 4-5 us from TMA issue to arrival under full load, so both rings are as deep
 // as shared memory allows.
-// Right after a local average (TcFwdArgs::share > 1) the members of a cluster hold
-// identical weights and all read the first member's copy.  (Ordering the items so
-// that the members' items for one weight tile are claimed together measured no
-// faster: the CTAs sharing a tile drift apart over its chunks by more than the time
-// the tile stays in L2.)
+// Right after a compact local average the learners of a cluster read their cluster's
+// mean (TcFwdArgs::w_div > 1); k_tc_forward_group then forwards groups of them at once.
 constexpr int kFwdConv = 256;
 constexpr int kFwdThreads = kFwdConv + 96;
 constexpr int kFwdWRingMax = 6, kFwdHRingMax = 8;
@@ -707,6 +704,390 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   if (dyn && threadIdx.x == 0) {
     // the last CTA out resets the claim counters for the next launch (every claim of
     // every CTA precedes that CTA's increment here)
+    __threadfence();
+    if (atomicAdd(a.dyn + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+      a.dyn[0] = 0;
+      a.dyn[1] = 0;
+    }
+  }
+}
+
+
+// ------------------------------------------------------------------ grouped forward
+// Right after a compact local average the learners of a cluster hold the same weights,
+// their cluster's mean.  The forward of G learners of a cluster is then one product of
+// each weight tile of the mean with their G stacked batch tiles (N = G * Bn <= 128
+// columns): a weight chunk is streamed and converted once for G learners instead of G
+// times.  Every output (learner, sample) is summed exactly as k_tc_forward sums it: the
+// same chunks, the same every-kSegChunks promotion from the item's first chunk, the
+// same pieces added in piece order, and the columns of one MMA do not mix, so the bits
+// are the per-learner forward's.  Work item = group tile (learners q*G .. q*G+G-1,
+// outputs 128*ot ..): whole group tiles first, then the pieces of the tail group tiles;
+// the plan's tail must consist of whole groups (n_whole a multiple of G * o_tiles).
+// Hidden layers (mode 0) and logits (mode 1).  Roles as in k_tc_forward.
+constexpr int kGfWRing = 5;
+constexpr uint32_t kGfTmemCols = 512;          // accumulators at 0 and 128, A tiles at 256
+constexpr uint32_t kGfTmemA = 256;
+__host__ __device__ constexpr int gf_h_off() { return kGfWRing * kFwdWf32; }
+__host__ __device__ constexpr int gf_hring(int N) {
+  return (kFwdSmemMax - 1024 - kBarBytes - gf_h_off()) / (N * 128) < kFwdHRingMax
+             ? (kFwdSmemMax - 1024 - kBarBytes - gf_h_off()) / (N * 128)
+             : kFwdHRingMax;
+}
+__host__ __device__ constexpr int gf_bar_off(int N) { return gf_h_off() + gf_hring(N) * N * 128; }
+__host__ __device__ constexpr int gf_smem(int N) { return gf_bar_off(N) + kBarBytes + 1024; }
+static_assert(gf_hring(128) >= 4 && gf_smem(128) <= kFwdSmemMax && gf_smem(96) <= kFwdSmemMax,
+              "grouped forward shared-memory plan");
+
+struct GfItem {
+  int q, ot, c_lo, c_hi, piece, np;
+};
+
+__device__ __forceinline__ GfItem gf_item(const TcFwdArgs& a, int G, int nk, int it) {
+  const int gw = a.n_whole / G;                 // whole group tiles
+  GfItem f;
+  int gt = it;
+  if (it < gw) {
+    f.c_lo = 0;
+    f.c_hi = nk;
+    f.piece = 0;
+    f.np = 1;
+  } else {
+    const int np = a.np_tail, i2 = it - gw, tt = i2 / np, p = i2 - tt * np;
+    gt = gw + tt;
+    f.c_lo = p * a.piece_chunks;
+    f.c_hi = f.c_lo + a.piece_chunks < nk ? f.c_lo + a.piece_chunks : nk;
+    f.piece = p;
+    f.np = np;
+  }
+  f.q = gt / a.o_tiles;
+  f.ot = gt - f.q * a.o_tiles;
+  return f;
+}
+
+__global__ void __launch_bounds__(kFwdThreads, 1)
+    k_tc_forward_group(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_h,
+                       const TcFwdArgs a, int G) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nk = (a.in + 63) / 64;
+  const int N = G * a.Bn;
+  const int gtiles = a.n_tiles / G, gw = a.n_whole / G;
+  const int n_items = gw + (gtiles - gw) * a.np_tail;
+  const int nw = kGfWRing, nh = gf_hring(N);
+  const int tbytes = a.Bn * 128, hbytes = N * 128;
+  const int h_row0 = a.x_direct ? a.x_row0 : 0;
+  uint8_t* h_base = smem + gf_h_off();
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + gf_bar_off(N));
+  uint64_t* wempty = wfull + kFwdWRingMax;
+  uint64_t* hfull = wempty + kFwdWRingMax;
+  uint64_t* hempty = hfull + kFwdHRingMax;
+  uint64_t* conv = hempty + kFwdHRingMax;  // [2] A tile written to TMEM
+  uint64_t* wfree = conv + 2;              // [2] A tile consumed by the MMA
+  uint64_t* accf = wfree + 2;              // [2] accumulator segment complete
+  uint64_t* accr = accf + 2;               // [2] accumulator segment drained
+  uint64_t* gbar = accr + 2;
+  uint64_t* done = gbar + 1;
+  ItemQueue queue{done + 1, done + 1 + kQueue, nullptr};
+  queue.items = reinterpret_cast<int*>(done + 1 + 2 * kQueue);
+  int* last_flag = queue.items + kQueue;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(last_flag + 1);
+  auto wf = [&](int s) { return smem + s * kFwdWf32; };
+  auto hb = [&](int s) { return h_base + s * hbytes; };
+  constexpr int kConsumers = 2 + kFwdConv / 32;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kFwdWRingMax; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], kFwdConv / 32);
+    }
+    for (int s = 0; s < kFwdHRingMax; ++s) {
+      mbar_init(&hfull[s], 1);
+      mbar_init(&hempty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&conv[b], kFwdConv / 32);
+      mbar_init(&wfree[b], 1);
+      mbar_init(&accf[b], 1);
+      mbar_init(&accr[b], kFwdConv);
+    }
+    for (int q = 0; q < kQueue; ++q) {
+      mbar_init(&queue.full[q], 1);
+      mbar_init(&queue.empty[q], kConsumers);
+    }
+    mbar_init(gbar, kFwdConv);
+    mbar_init(done, 1);
+    fence_barrier_init();
+  }
+  if (warp == 9) {
+    tmem_alloc(tmem_slot, kGfTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  grid_dep_wait();
+
+  auto next_item = [&](int k, GfItem& f) -> bool {
+    const int it = queue.take(k, lane, a.err);
+    if (it < 0) return false;
+    f = gf_item(a, G, nk, it);
+    return true;
+  };
+
+  if (warp == 8) {
+    if (lane == 0) {
+      // claim, announce, and stream the weight tiles of the cluster mean (normal L2
+      // policy: the cluster's other groups read them too)
+      tma_prefetch_desc(&tm_w);
+      const uint64_t pol = l2_stream_policy(false);
+      int i = 0, issued = 0;
+      bool ok = true;
+      int next = atomicAdd(a.dyn, 1);
+      for (int k = 0; ok; ++k) {
+        const int it = next < n_items ? next : -1;
+        if (!queue.put(k, it, a.err) || it < 0) break;
+        next = atomicAdd(a.dyn, 1);
+        const GfItem f = gf_item(a, G, nk, it);
+        const int jw = f.q * G / a.w_div;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nw;
+          if (i >= nw && !mbar_wait(&wempty[s], ((i / nw) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&wfull[s], kFwdWf32);
+          tma_load_3d_hint(wf(s), &tm_w, &wfull[s], c * 64, f.ot * 128, jw, pol);
+          tma_load_3d_hint(wf(s) + kFwdWBox, &tm_w, &wfull[s], c * 64 + 32, f.ot * 128, jw, pol);
+          issued = i + 1;
+        }
+      }
+      for (int u = issued - nw > 0 ? issued - nw : 0; u < issued; ++u)
+        mbar_wait(&wfull[u % nw], (u / nw) & 1, a.err);
+    }
+  } else if (warp == 10) {
+    // the G learners' batch tiles of each chunk, stacked: learner m's rows at m * Bn
+    if (lane == 0) tma_prefetch_desc(&tm_h);
+    int i = 0, issued = 0;
+    bool ok = true;
+    GfItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        const int j0 = f.q * G;
+        for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
+          const int s = i % nh;
+          if (i >= nh && !mbar_wait(&hempty[s], ((i / nh) - 1) & 1, a.err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&hfull[s], hbytes);
+          for (int m = 0; m < G; ++m)
+            tma_load_3d(hb(s) + m * tbytes, &tm_h, &hfull[s], c * 64, h_row0, j0 + m);
+          issued = i + 1;
+        }
+      }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0)
+      for (int u = issued - nh > 0 ? issued - nh : 0; u < issued; ++u)
+        mbar_wait(&hfull[u % nh], (u / nh) & 1, a.err);
+  } else if (warp == 9) {
+    const uint32_t idesc = umma_idesc_bf16(128, N);
+    int q = -1, i = 0;
+    bool ok = true;
+    GfItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      if (lane == 0) {
+        for (int c = f.c_lo, p = 0; c < f.c_hi; ++c, ++p, ++i) {
+          const bool tlast = c == f.c_hi - 1;
+          const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
+          const int sh = i % nh, b = i & 1;
+          if (first) ++q;
+          const int ab = q & 1;
+          if (first && q >= 2 && !mbar_wait(&accr[ab], ((q >> 1) - 1) & 1, a.err)) { ok = false; break; }
+          if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+          if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t at = tmem + kGfTmemA + 32 * b;
+          const uint64_t bd = umma_desc_sw128(smem_u32(hb(sh)));
+          const uint32_t d = tmem + 128 * ab;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            tc_mma_bf16_ta(d, at + 8 * kk, bd + 2 * kk, idesc, (!first || kk > 0) ? 1u : 0u);
+          tc_commit(&hempty[sh]);
+          tc_commit(&wfree[b]);
+          if (last) tc_commit(&accf[ab]);
+        }
+      }
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (lane == 0) {
+      tc_commit(done);
+      mbar_wait(done, 0, a.err);
+    }
+  } else {
+    // ---- warps 0-7: fp32 -> bf16 A tile, the accumulator drains and the epilogues.
+    // Thread t: accumulator row r (output 128 * ot + r), column blocks 2m + gr of 16
+    // (m = 0..3), column = learner (q * G + col / Bn), sample col % Bn.
+    const int t = threadIdx.x;
+    const int r = t & 127, gr = t >> 7;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+    GroupSync gsync{gbar, 0, a.err};
+    float acc[64];
+#pragma unroll
+    for (int q = 0; q < 64; ++q) acc[q] = 0.f;
+    int qc = -1, drained = 0;
+    auto drain = [&]() -> bool {
+      const int ab = drained & 1;
+      if (!wait_warp(&accf[ab], (drained >> 1) & 1, a.err)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const int cb = (2 * m + gr) * 16;
+        if (cb < N) {
+          float v[16];
+          tmem_ld16(tbase + 128 * ab + cb, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < 16; ++q) acc[16 * m + q] = __fadd_rn(acc[16 * m + q], v[q]);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&accr[ab]);
+      ++drained;
+      return true;
+    };
+    auto epilogue = [&](const GfItem& f, float bias) {
+      const int o = f.ot * 128 + r;
+      if (o >= a.out) return;
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const int cb = (2 * m + gr) * 16;
+        if (cb >= N) break;
+        const int ml = cb / a.Bn, b0 = cb - ml * a.Bn;
+        const int64_t j = static_cast<int64_t>(f.q) * G + ml;
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          if (b0 + q >= a.B) break;
+          if (a.mode == kFwdHidden)
+            a.h_out[(j * a.Bn + b0 + q) * a.pitch_out + o] =
+                __float2bfloat16_rn(fmaxf(__fadd_rn(acc[16 * m + q], bias), 0.f));
+          else
+            a.z_out[(j * a.B + b0 + q) * a.out + o] = __fadd_rn(acc[16 * m + q], bias);
+        }
+      }
+    };
+    // A tail piece ends: its partials go to the G learners' slots (slot of learner j's
+    // tile tau = j * o_tiles + ot, as k_tc_forward's), counted on the first learner's
+    // tile; the piece completing the group tile sums every learner's partials in piece
+    // order (true: it runs the epilogue).
+    auto group_piece_end = [&](const GfItem& f, bool& ok) -> bool {
+      const int64_t slot_stride = static_cast<int64_t>(128) * a.Bn;
+      auto slot = [&](int ml, int p) {
+        const int64_t tt = (static_cast<int64_t>(f.q) * G + ml) * a.o_tiles + f.ot - a.n_whole;
+        return a.part + ((tt * f.np + p) * 128 + r) * a.Bn;
+      };
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const int cb = (2 * m + gr) * 16;
+        if (cb < N) {
+          const int ml = cb / a.Bn, b0 = cb - ml * a.Bn;
+          float* dst = slot(ml, f.piece) + b0;
+#pragma unroll
+          for (int q = 0; q < 16; q += 4)
+            __stcg(reinterpret_cast<float4*>(dst + q),
+                   make_float4(acc[16 * m + q], acc[16 * m + q + 1], acc[16 * m + q + 2], acc[16 * m + q + 3]));
+        }
+      }
+      if (!gsync()) { ok = false; return false; }
+      if (t == 0) {
+        const int64_t tt0 = static_cast<int64_t>(f.q) * G * a.o_tiles + f.ot - a.n_whole;
+        fence_acq_rel_gpu();
+        const int before = atomicAdd(a.counters + tt0, 1);
+        const int lastp = before == f.np - 1;
+        if (lastp) {
+          fence_acq_rel_gpu();
+          a.counters[tt0] = 0;
+        }
+        *last_flag = lastp;
+      }
+      if (!gsync()) { ok = false; return false; }
+      if (!*reinterpret_cast<volatile int*>(last_flag)) return false;
+#pragma unroll
+      for (int m = 0; m < 4; ++m) {
+        const int cb = (2 * m + gr) * 16;
+        if (cb < N) {
+          const int ml = cb / a.Bn, b0 = cb - ml * a.Bn;
+          const float* src = slot(ml, 0) + b0;
+#pragma unroll
+          for (int q = 0; q < 16; q += 4) {
+            float4 s0 = __ldcg(reinterpret_cast<const float4*>(src + q));
+            for (int p = 1; p < f.np; ++p) {
+              const float4 v = __ldcg(reinterpret_cast<const float4*>(src + p * slot_stride + q));
+              s0.x = __fadd_rn(s0.x, v.x);
+              s0.y = __fadd_rn(s0.y, v.y);
+              s0.z = __fadd_rn(s0.z, v.z);
+              s0.w = __fadd_rn(s0.w, v.w);
+            }
+            acc[16 * m + q] = s0.x;
+            acc[16 * m + q + 1] = s0.y;
+            acc[16 * m + q + 2] = s0.z;
+            acc[16 * m + q + 3] = s0.w;
+          }
+        }
+      }
+      return true;
+    };
+    bool ok = true;
+    int i = 0;
+    GfItem f;
+    for (int k = 0; ok && next_item(k, f); ++k) {
+      const int ob = f.ot * 128 + r;
+      const float tbias = ob < a.out ? a.bias[static_cast<int64_t>(f.q * G / a.b_div) * a.ld + ob] : 0.f;
+      for (int c = f.c_lo, p = 0; c < f.c_hi && ok; ++c, ++p, ++i) {
+        const bool tlast = c == f.c_hi - 1;
+        const int sw = i % nw, bb = i & 1;
+        if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
+        if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        tc_fence_after();
+        {
+          const int row = 32 * (warp & 3) + lane, half = warp >> 2;
+          const uint8_t* src = wf(sw) + half * kFwdWBox + row * 128;
+          uint32_t pk[16];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 x = *reinterpret_cast<const float4*>(src + ((q ^ (row & 7)) << 4));
+            pk[2 * q] = pack_bf16x2(x.x, x.y);
+            pk[2 * q + 1] = pack_bf16x2(x.z, x.w);
+          }
+          tmem_st16(tbase + kGfTmemA + 32 * bb + 16 * half, pk);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&wempty[sw]);
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&conv[bb]);
+        if (p % kSegChunks == 0) ++qc;
+        if (tlast) {
+          while (ok && drained <= qc)
+            if (!drain()) ok = false;
+          if (!ok) break;
+          const bool fin = f.np == 1 || group_piece_end(f, ok);
+          if (ok && fin) epilogue(f, tbias);
+#pragma unroll
+          for (int q = 0; q < 64; ++q) acc[q] = 0.f;
+          ok = __all_sync(0xffffffffu, ok);
+        } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
+          if (!drain()) ok = false;
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kGfTmemCols);
+  }
+  if (threadIdx.x == 0) {
     __threadfence();
     if (atomicAdd(a.dyn + 1, 1) == static_cast<int>(gridDim.x) - 1) {
       a.dyn[0] = 0;
@@ -2174,6 +2555,8 @@ cudaError_t tc_configure() {
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_forward<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kFwdSmemMax);
   if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tc_forward_group, cudaFuncAttributeMaxDynamicSharedMemorySize, kFwdSmemMax);
+  if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_update_forward<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            kFwdSmemMax);
   if (e != cudaSuccess) return e;
@@ -2199,6 +2582,21 @@ cudaError_t launch_tc_forward(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
                       false, a.cq, w_fwd, h_in, a);
   return launch_pdl(k_tc_forward<true>, dim3(a.ctas), dim3(kFwdThreads), fwd_smem(a.mode, a.Bn), s,
                     false, 1, w_fwd, h_in, a);
+}
+
+int tc_forward_group_size(int S, int Bn) {
+  for (int G = 128 / Bn; G >= 2; --G)
+    if (S % G == 0) return G;
+  return 1;
+}
+
+cudaError_t launch_tc_forward_group(const CUtensorMap& w_fwd, const CUtensorMap& h_in,
+                                    const TcFwdArgs& a, int G, cudaStream_t s) {
+  if (G < 2 || G * a.Bn > 128 || a.n_tiles % G != 0 || a.n_whole % (G * a.o_tiles) != 0 ||
+      a.mode == kFwdXent)
+    return cudaErrorInvalidValue;
+  return launch_pdl(k_tc_forward_group, dim3(a.ctas), dim3(kFwdThreads), gf_smem(G * a.Bn), s, false,
+                    1, w_fwd, h_in, a, G);
 }
 
 cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_store,

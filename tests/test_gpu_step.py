@@ -295,6 +295,17 @@ GROUP_S12_K1 = configs.Workload("mlp_bf16_group4_S12_K1_1", P=24, S=12, K1=1, K2
 GROUP_B64 = configs.Workload("mlp_bf16_group2_B64", P=8, S=4, K1=2, K2=2, rounds=1,
                              dims=(256, 128, 10), precision="bf16", N=256, B=64, lr=0.05,
                              sigma_mu=0.1, init="he")
+# The first step after a compact local average forwards groups of G learners of a
+# cluster with one product per weight tile (N = G * Bn <= 128).  Cases: G = 2 with a
+# 48-sample batch (N = 96), a ragged 1200-wide layer, whole and tail group tiles, the
+# tail split into pieces; G = 8 with a 16-sample batch, a 300-class logits layer (mode
+# 1); and the 300-class net with K1 = 1, where every step but the first reads the means.
+GFWD_B48 = configs.Workload("mlp_bf16_gfwd2_B48", P=32, S=2, K1=2, K2=2, rounds=1,
+                            dims=(3136, 1200, 10), precision="bf16", N=192, B=48, lr=0.05,
+                            sigma_mu=0.1, init="he")
+GFWD_B16 = configs.Workload("mlp_bf16_gfwd8_B16", P=32, S=8, K1=2, K2=2, rounds=1,
+                            dims=(1024, 1152, 300), precision="bf16", N=64, B=16, lr=0.05,
+                            sigma_mu=0.1, init="he")
 
 
 # round() writes each intermediate local average as one mean row per cluster, read by
@@ -303,9 +314,10 @@ GROUP_B64 = configs.Workload("mlp_bf16_group2_B64", P=8, S=4, K1=2, K2=2, rounds
 # cluster); clusters of 3 over a ragged three-layer net (the generic, non-power-of-two
 # averaging path, with K1 = 1: a compact average after every step but the last; no
 # groups); 5 clusters of 4 (a global tree over a non-power-of-two count of clusters),
-# head slices of 128 features; the group cases above.
+# head slices of 128 features; the group update and group forward cases above.
 @pytest.mark.parametrize("w", [SMALL_BF16, RAGGED_BF16.replace(K2=3), HEAD_F128, GROUP_S8,
-                               GROUP_S6, GROUP_S12_K1, GROUP_B64],
+                               GROUP_S6, GROUP_S12_K1, GROUP_B64, GFWD_B48, GFWD_B16,
+                               MANY_CLASSES_BF16.replace(K2=3)],
                          ids=lambda w: w.name)
 def test_literal_sequence_equals_round(w):
     # step/local_average/global_average in Algorithm 1's order give the same bits
