@@ -22,6 +22,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -36,7 +37,17 @@ METRIC = "learner-samples/s per Hier-AVG round"
 UNIT = "learner-samples/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 512 << 20
-DOM_SAMPLE = 7   # time 1 in 7 launches of the dominant kernel (coprime with the layer counts)
+DOM_SAMPLE = 7   # time about 1 in 7 launches of the dominant kernel (see dom_sample)
+
+
+def dom_sample(per_round: int) -> int:
+    """The sampling interval: the smallest n >= DOM_SAMPLE coprime with the dominant
+    kernel's launches per round, so that the timed launches cycle through every position
+    in the round (the first step of a block reads the cluster means and runs faster)."""
+    n = DOM_SAMPLE
+    while math.gcd(n, max(1, per_round)) != 1:
+        n += 1
+    return n
 
 
 def parse():
@@ -387,8 +398,10 @@ def run_ours(args):
     time.sleep(0.05)
     # one launch in DOM_SAMPLE of the dominant kernel is timed (events separate it from
     # its neighbours; timing every launch cost ~9 % of the round at 3072-512-10)
+    n_prof_rounds = max(1, min(args.steps, 3))
+    sample = dom_sample(prof[dom].launches // n_prof_rounds)
     ha.profile([dom])
-    ha.profile_every(DOM_SAMPLE)
+    ha.profile_every(sample)
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     if ws > 1:
@@ -452,7 +465,7 @@ def run_ours(args):
                 "traffic": traffic,
                 "algorithmic_bytes_per_launch": dom_bytes / max(1, dom_n),
                 "avg_launch_us": 1e3 * dom_ms / max(1, dom_n),
-                "timing": f"CUDA events around every {DOM_SAMPLE}th launch of this kernel inside the timed rounds",
+                "timing": f"CUDA events around every {sample}th launch of this kernel inside the timed rounds",
                 "launches_timed": dom_n}
     if dom_flops > 0:
         roofline["tensor"] = gemm_report(dom_bytes, dom_flops, dom_ms, hbm, tc)

@@ -165,6 +165,13 @@ __device__ __forceinline__ uint64_t l2_keep_policy() {
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+// The weights' policy: evict-first when all learners' parameters exceed L2 (a stream
+// that must not push out the re-read activation tiles), except for the cluster means
+// that every learner of a cluster reads (`shared`: normal); evict-last when they fit,
+// so that a step's weights are still in L2 for the next kernel and the next step.
+__device__ __forceinline__ uint64_t l2_weight_policy(bool stream, bool shared = false) {
+  return stream ? l2_stream_policy(!shared) : l2_keep_policy();
+}
 __device__ __forceinline__ void tma_load_3d_hint(void* smem_dst, const void* tmap, uint64_t* bar,
                                                  int c0, int c1, int c2, uint64_t policy) {
   asm volatile(

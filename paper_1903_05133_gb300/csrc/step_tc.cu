@@ -434,7 +434,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       // claim (dynamic), announce, and stream the weight tiles (kept in L2 as usual when
       // the learners of a cluster read the same ones)
       tma_prefetch_desc(&tm_w);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0 && a.w_div == 1);
+      const uint64_t stream = l2_weight_policy(a.w_stream != 0, a.w_div > 1);
       int i = 0, issued = 0;
       bool ok = true;
       int next = dyn ? atomicAdd(a.dyn, 1) : 0;
@@ -842,7 +842,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       // claim, announce, and stream the weight tiles of the cluster mean (normal L2
       // policy: the cluster's other groups read them too)
       tma_prefetch_desc(&tm_w);
-      const uint64_t pol = l2_stream_policy(false);
+      const uint64_t pol = l2_weight_policy(a.w_stream != 0, true);
       int i = 0, issued = 0;
       bool ok = true;
       int next = atomicAdd(a.dyn, 1);
@@ -1289,7 +1289,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       // its first W chunk, then its W chunks
       tma_prefetch_desc(&tm_wl);
       tma_prefetch_desc(&tm_h);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0 && a.src_div == 1);
+      const uint64_t stream = l2_weight_policy(a.w_stream != 0, a.src_div > 1);
       int i = 0, issued = 0;
       bool ok = true;
       int next = atomicAdd(a.dyn, 1);
@@ -1340,7 +1340,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   } else if (warp == 7) {
     // Store each updated chunk; its slot is released once the TMA has read it (two
     // stores in flight).
-    const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+    const uint64_t stream = l2_weight_policy(a.w_stream != 0);
     int i = 0;
     bool ok = true;
     FwdItem f;
@@ -1688,7 +1688,7 @@ __global__ void __launch_bounds__(upd_threads(Q), 1)
       // the group's learners in order
       tma_prefetch_desc(&tm_wl);
       tma_prefetch_desc(&tm_h);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+      const uint64_t stream = l2_weight_policy(a.w_stream != 0);
       int i = 0, kt = 0, issued = 0;
       bool ok = true;
       int next = atomicAdd(a.dyn, 1);
@@ -1755,7 +1755,7 @@ __global__ void __launch_bounds__(upd_threads(Q), 1)
     // Q = 1: store each updated chunk, freeing its slot one store behind.  Q > 1: free
     // the slots of the first Q - 1 learners as soon as they are read, store the group
     // sum (row g of the store map) and free its slot once the store has read it.
-    const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+    const uint64_t stream = l2_weight_policy(a.w_stream != 0);
     int i = 0;
     for (int k = 0;; ++k) {
       const int it = take(k);
@@ -2088,15 +2088,14 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     f = fwd_item(a, nk, it);
     return true;
   };
-  // (the batch and dZ tiles are re-read for every output tile: kept in L2 ahead of
-  // the streamed W)
-  const uint64_t keep = a.w_stream ? l2_keep_policy() : l2_stream_policy(false);
+  // (the batch and dZ tiles are re-read for every output tile: kept in L2)
+  const uint64_t keep = l2_keep_policy();
 
   if (warp == 8) {
     if (lane == 0) {
       // claim (dynamic), announce, and stream the weight tiles
       tma_prefetch_desc(&tm_wl);
-      const uint64_t stream = l2_stream_policy(a.w_stream != 0 && a.w_div == 1);
+      const uint64_t stream = l2_weight_policy(a.w_stream != 0, a.w_div > 1);
       int i = 0, issued = 0;
       bool ok = true;
       int next = dyn ? atomicAdd(a.dyn, 1) : 0;
@@ -2190,7 +2189,7 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     // Store each updated W tile; its slot is released once the TMA has read it.  In
     // cluster mode (a short layer) each slot is released as soon as its own store has
     // been read; otherwise one store behind, two in flight.
-    const uint64_t stream = l2_stream_policy(a.w_stream != 0);
+    const uint64_t stream = l2_weight_policy(a.w_stream != 0);
     int i = 0, released = 0;
     bool ok = true;
     FwdItem f;

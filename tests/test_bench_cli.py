@@ -36,3 +36,17 @@ def test_reference_arm_prints_one_json_line():
     e2e = line["e2e"]
     assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
     assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
+
+
+def test_dominant_kernel_sample_cycles_through_the_round():
+    import math
+    sys.path.insert(0, ROOT)
+    import bench
+    # 28 update+forward launches per round at 3072-2048-2048-10 (K1 = 8): every 7th
+    # would always land on the first step of a block
+    assert bench.dom_sample(28) == 9
+    assert bench.dom_sample(24) == bench.DOM_SAMPLE
+    for per_round in range(1, 200):
+        n = bench.dom_sample(per_round)
+        assert n >= bench.DOM_SAMPLE and math.gcd(n, per_round) == 1
+        assert {(k * n) % per_round for k in range(per_round)} == set(range(per_round))
