@@ -562,6 +562,29 @@ def test_full_size_step_sampled(w):
     assert stats["exempt_rows"] <= rows // 1000, stats.get("exempt")
 
 
+# The full-size workloads in the launch configuration the bench times: a round (compact
+# averages, quad- or pair-sum block-end updates, grouped forwards of each block's first
+# step, fused update+forwards, tail pieces) gives the bits of the literal step / local /
+# global sequence, and every learner holds the same parameters after it.
+@pytest.mark.parametrize("w", [configs.MLP2048_P64, configs.MLP4096_P32], ids=lambda w: w.name)
+def test_full_size_round_equals_literal_sequence(w):
+    w = w.replace(N=2 * w.B * w.K1)
+    ha1, X, y = setup(w, data_device="cuda", perturb=(0.002, 0.05))
+    ha2, _, _ = setup(w, data_device="cuda", perturb=(0.002, 0.05))
+    ha1.round()
+    for b in range(w.K2):
+        for k in range(w.K1):
+            ha2.step()
+        ha2.local_average()
+    ha2.global_average()
+    ha1.check()
+    ha2.check()
+    assert torch.equal(ha1.params.view(torch.int32), ha2.params.view(torch.int32))
+    assert torch.equal(ha1.losses(), ha2.losses())
+    p = ha1.params.view(torch.int32)
+    assert torch.equal(p, p[:1].expand_as(p))
+
+
 # bf16 path: the rows are copied beside the kernels in chunks of steps that double in
 # length; SMALL_BF16's round reads more rows than each learner has (the chunks wrap
 # around N), FUSE_PIECES has 6 steps (chunks 0 | 1 | 2-3 | 4-5), a free global interval
