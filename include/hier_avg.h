@@ -163,11 +163,11 @@ int hier_avg_set_batch(hier_avg* h, int B);
 /* One round end to end from host memory: copies the rows this round reads from
  * X_host [P, N, d_0] / y_host [P, N] (pinned memory recommended) into the bound
  * device data set, runs hier_avg_round, and copies the per-learner loss of the
- * round's last step into loss_host [P].  The copies (one contiguous copy per learner
- * and chunk) run on a stream of the library's own in chunks of steps that double in
- * length, issued between the kernel launches, and overlap the kernels: a step waits
- * only for the chunk holding the rows it reads (bf16 path; the fp32 path copies the
- * round's rows first).  Synchronises. */
+ * round's last step into loss_host [P].  The copies (one pitched copy of X and one
+ * of y per chunk, for all learners) run on a stream of the library's own in chunks
+ * of steps that double in length, issued between the kernel launches, and overlap
+ * the kernels: a step waits only for the chunk holding the rows it reads (bf16 path;
+ * the fp32 path copies the round's rows first).  Synchronises. */
 int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host,
                         float* loss_host);
 

@@ -777,19 +777,10 @@ int do_global(hier_avg* h) {
 
 int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 
-// One global round (Algorithm 1, Sec. 3.1): G local steps, a local average after every
-// K1-th, the global average after the G-th (fused with the local average that closes
-// the round when K1 divides G).  G = K1 * K2 unless set: Sec. 3.1 leaves beta = G / K1
-// free in practice.  The local averages inside the round are compact (do_local_means)
-// when the workspace holds the means; the global average writes every learner row, so
-// the round ends with all P rows in place.
-// Rows [r0, r0 + n) of every learner's data from host memory.  Spans of at least
-// kRowCopySplit bytes per learner go as one contiguous copy per learner (a pitched 2-D
-// copy of 25 MB rows measured ~55 GB/s against ~200 GB/s for 1-D copies); shorter spans
-// as one pitched copy for all learners, which costs one call instead of P (the host's
-// calls are what limits a short round).
-constexpr int64_t kRowCopySplit = int64_t(1) << 20;
-
+// Rows [r0, r0 + n) of every learner's data from host memory: one pitched copy for all
+// learners (X, then y).  (Measured from a pinned [32][100 MB] buffer: 205-211 GB/s for
+// rows of 0.75 to 25 MB, the rate of one contiguous copy per learner, at ~3 us of host
+// time instead of ~32 us for the 32 calls.)
 int copy_rows(hier_avg* h, const void* X_host, const int32_t* y_host, int64_t r0, int64_t n,
               cudaStream_t cs) {
   const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
@@ -797,24 +788,12 @@ int copy_rows(hier_avg* h, const void* X_host, const int32_t* y_host, int64_t r0
   uint8_t* X = static_cast<uint8_t*>(const_cast<void*>(h->X));
   const uint8_t* Xh = static_cast<const uint8_t*>(X_host);
   int32_t* y = const_cast<int32_t*>(h->y);
-  if (n * rowb < kRowCopySplit) {
-    if (int rc = h->cuda(cudaMemcpy2DAsync(X + r0 * rowb, h->N * rowb, Xh + r0 * rowb, h->N * rowb,
-                                           n * rowb, h->P, cudaMemcpyHostToDevice, cs),
-                         "round_host: X copy"))
-      return rc;
-    return h->cuda(cudaMemcpy2DAsync(y + r0, h->N * 4, y_host + r0, h->N * 4, n * 4, h->P,
-                                     cudaMemcpyHostToDevice, cs), "round_host: y copy");
-  }
-  for (int j = 0; j < h->P; ++j) {
-    const int64_t off = static_cast<int64_t>(j) * h->N + r0;
-    if (int rc = h->cuda(cudaMemcpyAsync(X + off * rowb, Xh + off * rowb, n * rowb,
-                                         cudaMemcpyHostToDevice, cs), "round_host: X copy"))
-      return rc;
-    if (int rc = h->cuda(cudaMemcpyAsync(y + off, y_host + off, n * 4, cudaMemcpyHostToDevice, cs),
-                         "round_host: y copy"))
-      return rc;
-  }
-  return HA_OK;
+  if (int rc = h->cuda(cudaMemcpy2DAsync(X + r0 * rowb, h->N * rowb, Xh + r0 * rowb, h->N * rowb,
+                                         n * rowb, h->P, cudaMemcpyHostToDevice, cs),
+                       "round_host: X copy"))
+    return rc;
+  return h->cuda(cudaMemcpy2DAsync(y + r0, h->N * 4, y_host + r0, h->N * 4, n * 4, h->P,
+                                   cudaMemcpyHostToDevice, cs), "round_host: y copy");
 }
 
 // round_host's row feed: the rows of the round's steps are copied from host memory on
@@ -858,6 +837,12 @@ struct RowFeed {
   }
 };
 
+// One global round (Algorithm 1, Sec. 3.1): G local steps, a local average after every
+// K1-th, the global average after the G-th (fused with the local average that closes
+// the round when K1 divides G).  G = K1 * K2 unless set: Sec. 3.1 leaves beta = G / K1
+// free in practice.  The local averages inside the round are compact (do_local_means)
+// when the workspace holds the means; the global average writes every learner row, so
+// the round ends with all P rows in place.
 // feed (round_host): step k reads the rows of step k and, in an update+forward kernel,
 // step k + 1's.  The handle's stream waits for step 0's and step 1's rows before step 0
 // (the latter just before step 0's update+forward), then at steps k = 1, 3, 7, ... (k + 1
