@@ -255,7 +255,9 @@ def test_one_step_from_distinct_learners(w):
 
 @pytest.mark.parametrize("w", [configs.SOFTMAX_P4, SMALL_FP32, SMALL_BF16, SOFTMAX_BF16,
                                HEAD_C13, WIDE_SOFTMAX_BF16, RAGGED_BF16, MANY_CLASSES_BF16,
-                               HEAD_F128, FUSE_PIECES, BWD_PIECES], ids=lambda w: w.name)
+                               HEAD_F128, FUSE_PIECES, BWD_PIECES,
+                               SMALL_BF16.replace(name="tiny_mlp_bf16_kavg", S=1)],
+                         ids=lambda w: w.name)
 def test_full_run_against_oracle(w):
     ha, X, y = setup(w)
     o = make_oracle(w, ha, X, y, oracle_params(ha, ha.params))
@@ -308,6 +310,17 @@ GFWD_B16 = configs.Workload("mlp_bf16_gfwd8_B16", P=32, S=8, K1=2, K2=2, rounds=
                             sigma_mu=0.1, init="he")
 
 
+# S = 1 (K-AVG: the local average is the identity, every average in place); one cluster
+# of all 8 learners (S = P, quad sums and groups of 4); and 150 rows per learner with a
+# 32-row batch, so that batches straddle the end of the data set (the gather path, also
+# in the grouped forward, and steps whose successor's batch is not contiguous).
+KAVG_BF16 = SMALL_BF16.replace(name="tiny_mlp_bf16_kavg", S=1)
+GROUP_SP = configs.Workload("mlp_bf16_group4_S8_P8", P=8, S=8, K1=2, K2=2, rounds=1,
+                            dims=(256, 192, 10), precision="bf16", N=128, B=32, lr=0.05,
+                            sigma_mu=0.1, init="he")
+PIECES_WRAP = FUSE_PIECES.replace(name="mlp_bf16_pieces_wrap", N=150)
+
+
 # round() writes each intermediate local average as one mean row per cluster, read by
 # the next step, and fuses the last local average into the global one; the literal
 # sequence writes every row each time.  Cases: clusters of 2 (group sums of 2: one per
@@ -317,7 +330,8 @@ GFWD_B16 = configs.Workload("mlp_bf16_gfwd8_B16", P=32, S=8, K1=2, K2=2, rounds=
 # head slices of 128 features; the group update and group forward cases above.
 @pytest.mark.parametrize("w", [SMALL_BF16, RAGGED_BF16.replace(K2=3), HEAD_F128, GROUP_S8,
                                GROUP_S6, GROUP_S12_K1, GROUP_B64, GFWD_B48, GFWD_B16,
-                               MANY_CLASSES_BF16.replace(K2=3)],
+                               MANY_CLASSES_BF16.replace(K2=3), KAVG_BF16, GROUP_SP,
+                               PIECES_WRAP],
                          ids=lambda w: w.name)
 def test_literal_sequence_equals_round(w):
     # step/local_average/global_average in Algorithm 1's order give the same bits
