@@ -88,18 +88,23 @@ __global__ void __launch_bounds__(256) k_mean_pow2_to(const float4* __restrict__
 // (S copies of each cluster mean, in learner order), so the result is the literal
 // two-pass result: the S equal copies of a cluster form one complete sub-tree of
 // the global tree, whose value is the cluster mean added to itself LOGS times.
-template <int LOGS, int LOGG>
-__global__ void __launch_bounds__(256) k_local_global_pow2(float4* __restrict__ w,
-                                                           int64_t ld_v, int64_t cols_v) {
+// Each cluster's sum is the tree over its 2^(LOGS - LOGQ) rows of src (row stride
+// src_ld_v): the learner rows themselves (LOGQ = 0, src = w), or sums of Q = 2^LOGQ
+// learners each that hold the first LOGQ levels of the cluster's tree.  The result
+// is written to all P rows of w (src may be rows of w: a thread reads its column of
+// every source row before it writes).
+template <int LOGQ, int LOGS, int LOGG>
+__global__ void __launch_bounds__(256) k_local_global_pow2(const float4* src, int64_t src_ld_v,
+                                                           float4* w, int64_t ld_v, int64_t cols_v) {
   grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
-  constexpr int S = 1 << LOGS, G = 1 << LOGG;
-  float4* p = w + c;
+  constexpr int S = 1 << LOGS, G = 1 << LOGG, N = 1 << (LOGS - LOGQ);
+  const float4* q = src + c;
   float4 stack[LOGG + 1];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
-    float4 x = vdiv(tree_pow2<LOGS>(p + static_cast<int64_t>(g) * S * ld_v, ld_v),
+    float4 x = vdiv(tree_pow2<LOGS - LOGQ>(q + static_cast<int64_t>(g) * N * src_ld_v, src_ld_v),
                     static_cast<float>(S));
 #pragma unroll
     for (int l = 0; l < LOGS; ++l) x = vadd(x, x);
@@ -112,7 +117,7 @@ __global__ void __launch_bounds__(256) k_local_global_pow2(float4* __restrict__ 
     stack[l] = x;
   }
   const float4 m = vdiv(stack[LOGG], static_cast<float>(S * G));
-  store_rows(p, ld_v, S * G, m);
+  store_rows(w + c, ld_v, S * G, m);
 }
 
 // Generic path: any n (also non-powers of two) and scalar columns.  The binary
@@ -163,17 +168,20 @@ __global__ void __launch_bounds__(256) k_mean_any_to(const V* __restrict__ w, in
   out[static_cast<int64_t>(blockIdx.y) * out_ld_v + c] = vdiv(tree_any(p, ld_v, n), div);
 }
 
+// (src, src_ld_v, n: as in k_local_global_pow2, n = S / Q source rows per cluster.)
 template <class V>
-__global__ void __launch_bounds__(256) k_local_global_any(V* __restrict__ w, int64_t ld_v,
-                                                          int64_t cols_v, int S, int G) {
+__global__ void __launch_bounds__(256) k_local_global_any(const V* src, int64_t src_ld_v, int n,
+                                                          V* w, int64_t ld_v, int64_t cols_v, int S,
+                                                          int G) {
   grid_dep_wait();
   const int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (c >= cols_v) return;
   V* p = w + c;
+  const V* q = src + c;
   V stack[32];
   int64_t i = 0;   // index of the next pushed value of the global sequence
   for (int g = 0; g < G; ++g) {
-    const V m = vdiv(tree_any(p + static_cast<int64_t>(g) * S * ld_v, ld_v, S),
+    const V m = vdiv(tree_any(q + static_cast<int64_t>(g) * n * src_ld_v, src_ld_v, n),
                      static_cast<float>(S));
     for (int r = 0; r < S; ++r, ++i) {
       V x = m;
@@ -185,16 +193,16 @@ __global__ void __launch_bounds__(256) k_local_global_any(V* __restrict__ w, int
       stack[l] = x;
     }
   }
-  const int n = S * G;
+  const int total = S * G;
   V acc{};
   bool have = false;
   for (int l = 0; l < 32; ++l) {
-    if ((n >> l) & 1) {
+    if ((total >> l) & 1) {
       acc = have ? vadd(stack[l], acc) : stack[l];
       have = true;
     }
   }
-  store_rows(p, ld_v, n, vdiv(acc, static_cast<float>(n)));
+  store_rows(p, ld_v, total, vdiv(acc, static_cast<float>(total)));
 }
 
 constexpr int kThreads = 256;
@@ -262,31 +270,46 @@ bool mean_pow2_dispatch(int log, float4* w, int64_t ld_v, int64_t cols_v, int64_
   }
 }
 
-template <int LOGS, int LOGG>
-void launch_lg(float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
+template <int LOGQ, int LOGS, int LOGG>
+void launch_lg(const float4* src, int64_t src_ld_v, float4* w, int64_t ld_v, int64_t cols_v,
+               cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
-  launch_pdl(k_local_global_pow2<LOGS, LOGG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v);
+  launch_pdl(k_local_global_pow2<LOGQ, LOGS, LOGG>, grid, dim3(kThreads), 0, s, false, 1, src,
+             src_ld_v, w, ld_v, cols_v);
 }
 
-template <int LOGS>
-bool lg_dispatch_g(int logg, float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
-  if (logg == 0) { launch_lg<LOGS, 0>(w, ld_v, cols_v, s); return true; }
-  if constexpr (LOGS + 1 <= 7) if (logg == 1) { launch_lg<LOGS, 1>(w, ld_v, cols_v, s); return true; }
-  if constexpr (LOGS + 2 <= 7) if (logg == 2) { launch_lg<LOGS, 2>(w, ld_v, cols_v, s); return true; }
-  if constexpr (LOGS + 3 <= 7) if (logg == 3) { launch_lg<LOGS, 3>(w, ld_v, cols_v, s); return true; }
-  if constexpr (LOGS + 4 <= 7) if (logg == 4) { launch_lg<LOGS, 4>(w, ld_v, cols_v, s); return true; }
-  if constexpr (LOGS + 5 <= 7) if (logg == 5) { launch_lg<LOGS, 5>(w, ld_v, cols_v, s); return true; }
-  if constexpr (LOGS + 6 <= 7) if (logg == 6) { launch_lg<LOGS, 6>(w, ld_v, cols_v, s); return true; }
+template <int LOGQ, int LOGS>
+bool lg_dispatch_g(int logg, const float4* src, int64_t src_ld_v, float4* w, int64_t ld_v,
+                   int64_t cols_v, cudaStream_t s) {
+  if constexpr (LOGQ <= LOGS) {
+#define HA_LG(G_) \
+    if constexpr (LOGS + G_ <= 7) \
+      if (logg == G_) { launch_lg<LOGQ, LOGS, G_>(src, src_ld_v, w, ld_v, cols_v, s); return true; }
+    HA_LG(0) HA_LG(1) HA_LG(2) HA_LG(3) HA_LG(4) HA_LG(5) HA_LG(6)
+#undef HA_LG
+  }
   return false;
 }
 
-bool lg_dispatch(int logs, int logg, float4* w, int64_t ld_v, int64_t cols_v, cudaStream_t s) {
+template <int LOGQ>
+bool lg_dispatch_s(int logs, int logg, const float4* src, int64_t src_ld_v, float4* w,
+                   int64_t ld_v, int64_t cols_v, cudaStream_t s) {
   switch (logs) {
-    case 1: return lg_dispatch_g<1>(logg, w, ld_v, cols_v, s);
-    case 2: return lg_dispatch_g<2>(logg, w, ld_v, cols_v, s);
-    case 3: return lg_dispatch_g<3>(logg, w, ld_v, cols_v, s);
-    case 4: return lg_dispatch_g<4>(logg, w, ld_v, cols_v, s);
-    case 5: return lg_dispatch_g<5>(logg, w, ld_v, cols_v, s);
+    case 1: return lg_dispatch_g<LOGQ, 1>(logg, src, src_ld_v, w, ld_v, cols_v, s);
+    case 2: return lg_dispatch_g<LOGQ, 2>(logg, src, src_ld_v, w, ld_v, cols_v, s);
+    case 3: return lg_dispatch_g<LOGQ, 3>(logg, src, src_ld_v, w, ld_v, cols_v, s);
+    case 4: return lg_dispatch_g<LOGQ, 4>(logg, src, src_ld_v, w, ld_v, cols_v, s);
+    case 5: return lg_dispatch_g<LOGQ, 5>(logg, src, src_ld_v, w, ld_v, cols_v, s);
+    default: return false;
+  }
+}
+
+bool lg_dispatch(int logq, int logs, int logg, const float4* src, int64_t src_ld_v, float4* w,
+                 int64_t ld_v, int64_t cols_v, cudaStream_t s) {
+  switch (logq) {
+    case 0: return lg_dispatch_s<0>(logs, logg, src, src_ld_v, w, ld_v, cols_v, s);
+    case 1: return lg_dispatch_s<1>(logs, logg, src, src_ld_v, w, ld_v, cols_v, s);
+    case 2: return lg_dispatch_s<2>(logs, logg, src, src_ld_v, w, ld_v, cols_v, s);
     default: return false;
   }
 }
@@ -300,9 +323,11 @@ void launch_mean_any(V* w, int64_t ld_v, int64_t cols_v, int n, int64_t groups,
 }
 
 template <class V>
-void launch_lg_any(V* w, int64_t ld_v, int64_t cols_v, int S, int G, cudaStream_t s) {
+void launch_lg_any(const V* src, int64_t src_ld_v, int n, V* w, int64_t ld_v, int64_t cols_v, int S,
+                   int G, cudaStream_t s) {
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
-  launch_pdl(k_local_global_any<V>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v, S, G);
+  launch_pdl(k_local_global_any<V>, grid, dim3(kThreads), 0, s, false, 1, src, src_ld_v, n, w, ld_v,
+             cols_v, S, G);
 }
 
 }  // namespace
@@ -359,17 +384,28 @@ cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, 
   // S = 1: the local average is the identity, so the pair is one global mean.
   // (S = P is NOT shortcut: the literal second pass re-averages P equal copies.)
   if (S == 1) return launch_group_mean(w, P, P, D, ld, s);
-  const int64_t G = P / S;
+  return launch_local_global_from_groups(w, ld, 1, w, P, S, D, ld, s);
+}
+
+cudaError_t launch_local_global_from_groups(const float* src, int64_t src_ld, int64_t Q, float* w,
+                                            int64_t P, int64_t S, int64_t D, int64_t ld,
+                                            cudaStream_t s) {
+  if (D == 0) return cudaSuccess;
+  const int64_t G = P / S, n = S / Q;
   int64_t head = 0;
-  if (vec_ok(w, ld) && D >= 4) {
+  if (vec_ok(w, ld) && vec_ok(src, src_ld) && D >= 4) {
     head = D & ~int64_t(3);
     float4* w4 = reinterpret_cast<float4*>(w);
-    const int logs = ilog2_exact(S), logg = ilog2_exact(G);
-    if (!(logs >= 1 && logg >= 0 && lg_dispatch(logs, logg, w4, ld / 4, head / 4, s)))
-      launch_lg_any<float4>(w4, ld / 4, head / 4, static_cast<int>(S), static_cast<int>(G), s);
+    const float4* s4 = reinterpret_cast<const float4*>(src);
+    const int logq = ilog2_exact(Q), logs = ilog2_exact(S), logg = ilog2_exact(G);
+    if (!(logq >= 0 && logs >= 1 && logg >= 0 &&
+          lg_dispatch(logq, logs, logg, s4, src_ld / 4, w4, ld / 4, head / 4, s)))
+      launch_lg_any<float4>(s4, src_ld / 4, static_cast<int>(n), w4, ld / 4, head / 4,
+                            static_cast<int>(S), static_cast<int>(G), s);
   }
   if (head < D)
-    launch_lg_any<float>(w + head, ld, D - head, static_cast<int>(S), static_cast<int>(G), s);
+    launch_lg_any<float>(src + head, src_ld, static_cast<int>(n), w + head, ld, D - head,
+                         static_cast<int>(S), static_cast<int>(G), s);
   return cudaGetLastError();
 }
 

@@ -480,9 +480,10 @@ ha::HeadArgs head_args(hier_avg* h, ParamSrc src) {
 // per step, so after this step every learner row holds its parameters again.
 // next_rows (round_host): recorded once the next step's rows are on the device; the
 // update+forward kernel, which reads them, waits for it.
-// group_out: a compact local average follows this step; the first layer's update may
-// then store group sums of W_1 (h->upd_group learners each) instead of the learner
-// rows' W_1, and *grouped reports whether it did (the average must then read them).
+// group_out: a local average follows this step (compact, or fused with the global
+// average) and reads the round's means; the first layer's update may then store group
+// sums of W_1 (h->upd_group learners each) instead of the learner rows' W_1, and
+// *grouped reports whether it did (the average must then read them).
 int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
             bool from_means = false, cudaEvent_t next_rows = nullptr, bool group_out = false,
             bool* grouped = nullptr) {
@@ -769,6 +770,22 @@ int do_local_global(hier_avg* h) {
   }, "local+global average");
 }
 
+// The fused last local average and global average after a grouped first-layer update:
+// W_1 from the group sums (rows g*Q), the rest of the row from the learner rows; every
+// row receives the global mean (the bits of do_local_global, as in do_local_means_grouped).
+int do_local_global_grouped(hier_avg* h) {
+  const int64_t P = h->P, S = h->S, Q = h->upd_group, ld = h->ld;
+  const int64_t w1 = static_cast<int64_t>(h->dims[0]) * h->dims[1];
+  const double bytes = 4.0 * (P / Q) * w1 + 4.0 * P * (ld - w1) + 4.0 * P * ld;
+  return h->timed(HA_KERNEL_GLOBAL_AVG, bytes, double(P) * ld, [&] {
+    ++h->launches;   // two launches
+    cudaError_t e = ha::launch_local_global_from_groups(h->params, Q * ld, Q, h->params, P, S, w1, ld,
+                                                        h->stream);
+    if (e != cudaSuccess) return e;
+    return ha::launch_local_global_mean(h->params + w1, P, S, ld - w1, ld, h->stream);
+  }, "local+global average");
+}
+
 int do_global(hier_avg* h) {
   return h->timed(HA_KERNEL_GLOBAL_AVG, 8.0 * h->P * h->ld, double(h->P) * h->ld, [&] {
     return ha::launch_group_mean(h->params, h->P, h->P, h->ld, h->ld, h->stream);
@@ -865,14 +882,15 @@ int do_round(hier_avg* h, RowFeed* feed = nullptr) {
     const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
     bool grouped = false;
     if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local && compact,
-                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr,
-                      compact && block_end && r < G, &grouped)))
+                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr, compact && block_end,
+                      &grouped)))
       return rc;
     if (r < G && block_end &&
         (rc = grouped ? do_local_means_grouped(h) : compact ? do_local_means(h) : do_local(h)))
       return rc;
+    if (r == G && block_end) return grouped ? do_local_global_grouped(h) : do_local_global(h);
   }
-  return G % h->K1 == 0 ? do_local_global(h) : do_global(h);
+  return do_global(h);
 }
 
 // Failure-detection self-test: the library's two kinds of bounded device wait, each

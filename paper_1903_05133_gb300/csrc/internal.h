@@ -59,6 +59,12 @@ cudaError_t launch_group_sum_mean_to(const float* w, int64_t rows, int64_t n, in
 // The local average (clusters of S) followed by the global average, in one pass.
 cudaError_t launch_local_global_mean(float* w, int64_t P, int64_t S, int64_t D, int64_t ld,
                                      cudaStream_t s);
+// The same, with each cluster's sum taken from S / Q rows of src (stride src_ld) that
+// hold sums of Q learners in the first levels of its adjacent-pair tree (Q = 1, 2 or 4,
+// Q | S); the result goes to all P rows of w (src may point into w).
+cudaError_t launch_local_global_from_groups(const float* src, int64_t src_ld, int64_t Q, float* w,
+                                            int64_t P, int64_t S, int64_t D, int64_t ld,
+                                            cudaStream_t s);
 
 // ----------------------------------------------------------------- bf16 tensor-core step
 // Activation buffers of the bf16 path (all zero-initialised once; kernels only

@@ -391,9 +391,9 @@ def test_fused_next_forward_equals_steps(w):
         ha2.local_average()
     ha2.global_average()
     # the literal sequence launches every kernel; round() saves the fused forwards and
-    # fuses the last local average into the global one, and takes each local average
-    # inside the round from group sums of W_1 in a launch of its own (S even)
-    saved = n_fused + 1 - (w.K2 - 1 if w.S % 2 == 0 else 0)
+    # fuses the last local average into the global one, and takes each average from
+    # group sums of W_1 in a launch of its own (S even: K2 - 1 local, one local+global)
+    saved = n_fused + 1 - (w.K2 if w.S % 2 == 0 else 0)
     assert ha2.launches() - n1 == n_round + saved
     ha1.check()
     ha2.check()
