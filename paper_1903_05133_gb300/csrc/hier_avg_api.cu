@@ -81,6 +81,7 @@ struct hier_avg {
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
   std::vector<int> fwd_cq;                    // per layer: cluster split factor (1 = dynamic)
   std::vector<int> fwd_whole, fwd_np;         // per layer (dynamic): whole tiles, tail pieces
+  std::vector<int> fwd_pc;                    // per layer (dynamic): chunks per tail piece
   int fwd_group = 1;                          // learners per grouped forward after an average
   std::vector<int> bwd_ctas, bwd_tiles;       // per layer: CTAs, input slices of 128
   std::vector<int> bwd_whole, bwd_np;         // per layer: whole tiles, tail pieces
@@ -214,6 +215,7 @@ int plan_layout(hier_avg* h) {
     h->fwd_cq.assign(L, 1);
     h->fwd_whole.assign(L, 0);
     h->fwd_np.assign(L, 1);
+    h->fwd_pc.assign(L, static_cast<int>(kPieceChunks));
     h->bwd_ctas.assign(L, 1);
     h->bwd_tiles.assign(L, 1);
     h->bwd_whole.assign(L, 0);
@@ -245,7 +247,8 @@ int plan_layout(hier_avg* h) {
         const int64_t gt = h->fwd_group * ftiles;
         const int64_t t_tail =
             l == 0 ? std::min<int64_t>(ftiles * P, std::max<int64_t>(gt, kTargetCtas / gt * gt)) : 0;
-        const int64_t np = (nk + kPieceChunks - 1) / kPieceChunks;
+        const int64_t pc = h->fwd_pc[l];
+        const int64_t np = (nk + pc - 1) / pc;
         h->fwd_whole[l] = static_cast<int>(ftiles * P - t_tail);
         h->fwd_np[l] = static_cast<int>(np);
         const int64_t items = (ftiles * P - t_tail) + t_tail * np;
@@ -525,7 +528,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       a.n_tiles = h->fwd_tiles[l] * P;
       a.n_whole = h->fwd_whole[l];
       a.np_tail = h->fwd_np[l];
-      a.piece_chunks = static_cast<int>(kPieceChunks);
+      a.piece_chunks = h->fwd_pc[l];
       a.part = h->wsp<float>(h->off_part);
       a.counters = h->wsp<int>(h->off_cnt);
       a.dyn = h->wsp<int>(h->off_dyn);
@@ -642,7 +645,7 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         f.n_tiles = h->fwd_tiles[0] * P;
         f.n_whole = h->fwd_whole[0];
         f.np_tail = h->fwd_np[0];
-        f.piece_chunks = static_cast<int>(kPieceChunks);
+        f.piece_chunks = h->fwd_pc[0];
         f.part = h->wsp<float>(h->off_part);
         f.counters = h->wsp<int>(h->off_cnt);
         f.dyn = h->wsp<int>(h->off_dyn);
