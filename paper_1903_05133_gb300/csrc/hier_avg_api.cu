@@ -73,9 +73,12 @@ struct hier_avg {
   bool m_ok = false;                          // the bound workspace holds the means
   // The step that closes a local block inside a round (compact averages only) updates
   // W_1 for groups of upd_group learners of a cluster and stores their adjacent-pair
-  // tree sum, to the first learner row of each group through tm_gs (1: not used).
+  // tree sum, to the first learner row of each group through tm_gs[l] (1: not used);
+  // the later layers' updates do the same (their dX from a backward without update).
+  // grp[l]: the last step stored group sums of W_l.
   int upd_group = 1;
-  CUtensorMap tm_gs;
+  std::vector<CUtensorMap> tm_gs;
+  std::vector<char> grp;
   int64_t off_part = 0, off_cnt = 0;          // stream-K partials and tile counters
   int64_t off_dyn = 0;                        // update kernel's work-item counters
   std::vector<int> fwd_ctas, fwd_tiles;       // per layer: stream-K CTAs, output tiles
@@ -320,6 +323,7 @@ int build_maps(hier_avg* h) {
   h->tm_wf.resize(L);
   h->tm_wb.resize(L);
   h->tm_wf_m.resize(h->m_ok ? L : 0);
+  h->tm_gs.resize(L);
   h->tm_wb_m.resize(h->m_ok ? L : 0);
   h->tm_h.resize(L);
   h->tm_dz.resize(L + 1);
@@ -334,10 +338,10 @@ int build_maps(hier_avg* h) {
     if ((rc = make_map(h, &h->tm_wb[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P, in * 4,
                        h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
       return rc;
-    if (h->m_ok && l == 0 && h->upd_group > 1) {
-      // group sums of W_1: row g*Q of the parameter matrix, g < P / Q
+    if (h->m_ok && h->upd_group > 1) {
+      // group sums of W_l: row g*Q of the parameter matrix, g < P / Q
       const uint64_t Q = h->upd_group;
-      if ((rc = make_map(h, &h->tm_gs, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P / Q, in * 4,
+      if ((rc = make_map(h, &h->tm_gs[l], CU_TENSOR_MAP_DATA_TYPE_FLOAT32, W, in, out, P / Q, in * 4,
                          Q * h->ld * 4, 128, 64, CU_TENSOR_MAP_SWIZZLE_NONE)))
         return rc;
     }
@@ -484,15 +488,15 @@ ha::HeadArgs head_args(hier_avg* h, ParamSrc src) {
 // next_rows (round_host): recorded once the next step's rows are on the device; the
 // update+forward kernel, which reads them, waits for it.
 // group_out: a local average follows this step (compact, or fused with the global
-// average) and reads the round's means; the first layer's update may then store group
-// sums of W_1 (h->upd_group learners each) instead of the learner rows' W_1, and
-// *grouped reports whether it did (the average must then read them).
+// average) and reads the round's means; the weight updates of the tensor-core layers may
+// then store group sums of W_l (h->upd_group learners each) instead of the learner rows'
+// W_l, and h->grp[l] records which did (the average must then read them).
 int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fused = nullptr,
-            bool from_means = false, cudaEvent_t next_rows = nullptr, bool group_out = false,
-            bool* grouped = nullptr) {
+            bool from_means = false, cudaEvent_t next_rows = nullptr, bool group_out = false) {
   const int L = h->L, P = h->P, B = h->Bstep;
   if (fused) *fused = false;
-  if (grouped) *grouped = false;
+  h->grp.assign(L, 0);
+  const int q = group_out && h->m_ok ? h->upd_group : 1;
   cudaStream_t s = h->stream;
   int rc;
   const bool means = from_means && h->m_ok;
@@ -669,6 +673,24 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
       // The first layer's backward (no dX) runs the update-only kernel: independent
       // runs of 8 chunks, claimed dynamically (measured faster than the backward
       // kernel's items for short layers too: 3072-512-10 round 0.859 -> 0.850 ms).
+      // Grouped (q > 1): W_l read per learner, its group sums written to row g*q of the
+      // W_l region, g < P / q.  A layer with dX first runs the backward without update
+      // (dZ_{l-1}, b_{l-1}), which reads W_l once more: worth it for quads only (per
+      // weight and learner 4 more bytes read, 2 * (4 - 4 / q) fewer moved by the update
+      // and the average; pairs measured slower, 3072-2048-2048-10 36.02 -> 36.21 ms).
+      const double wbytes = double(P) * h->dims[l] * h->dims[l + 1] * 4.0;
+      const int ql = a.has_dx && q < 4 ? 1 : q;
+      const double gb = ql > 1 ? wbytes * (1.0 - 1.0 / ql) : 0.0;
+      if (a.has_dx && ql > 1) {
+        a.no_update = 1;
+        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - wbytes - shared_w_bytes(h, l, means),
+                      flops_gemm(h, l), [&] {
+          return ha::launch_tc_backward(wl, ws, hin, h->tm_dz[l + 1], a, P, s);
+        }, "backward");
+        if (rc) return rc;
+        a.no_update = 0;
+        a.has_dx = 0;
+      }
       if (a.has_dx) {
         rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - shared_w_bytes(h, l, means),
                       flops_gemm(h, l) * 2, [&] {
@@ -676,14 +698,12 @@ int do_step(hier_avg* h, bool h1_ready = false, bool fuse_next = false, bool* fu
         }, "backward");
       } else {
         a.ctas = kTargetCtas;
-        const int q = group_out && h->m_ok ? h->upd_group : 1;
-        // grouped: W_1 read per learner, its group sums written to row g*q, g < P / q
-        const double gb = q > 1 ? double(P) * h->dims[0] * h->dims[1] * 4.0 * (1.0 - 1.0 / q) : 0.0;
-        rc = h->timed(HA_KERNEL_BACKWARD, bytes_backward(h, l) - gb - shared_w_bytes(h, l, means),
-                      flops_gemm(h, l), [&] {
-          return ha::launch_tc_update(wl, q > 1 ? h->tm_gs : ws, hin, h->tm_dz[l + 1], a, q, s);
+        const double ub = double(P) * (h->dims[l] * h->dims[l + 1] * 8.0 + double(B) * h->dims[l] * 2 +
+                                       double(B) * h->dims[l + 1] * 2);
+        rc = h->timed(HA_KERNEL_BACKWARD, ub - gb - shared_w_bytes(h, l, means), flops_gemm(h, l), [&] {
+          return ha::launch_tc_update(wl, ql > 1 ? h->tm_gs[l] : ws, hin, h->tm_dz[l + 1], a, ql, s);
         }, "backward");
-        if (grouped) *grouped = q > 1;
+        h->grp[l] = ql > 1;
       }
       if (rc) return rc;
     }
@@ -748,22 +768,49 @@ int do_local_means(hier_avg* h) {
   }, "local average");
 }
 
-// The compact local average after a grouped first-layer update: W_1 from the group
-// sums (rows g*Q, g < P / Q, which hold the first log2(Q) levels of every cluster's
+// The parameter row in column ranges for an average after a grouped step: the W_l
+// regions whose group sums the step stored (h->grp[l]) and the ranges between them
+// (biases, padding, the other layers' weights), read from the learner rows.
+struct AvgRange {
+  int64_t c0, c1;
+  bool grouped;
+};
+std::vector<AvgRange> avg_ranges(const hier_avg* h) {
+  std::vector<AvgRange> r;
+  int64_t c = 0;
+  for (int l = 0; l < h->L; ++l) {
+    if (!h->grp[l]) continue;
+    const int64_t w0 = h->woff[l], w1 = w0 + static_cast<int64_t>(h->dims[l]) * h->dims[l + 1];
+    if (w0 > c) r.push_back({c, w0, false});
+    r.push_back({w0, w1, true});
+    c = w1;
+  }
+  if (c < h->ld) r.push_back({c, h->ld, false});
+  return r;
+}
+
+// The compact local average after a grouped step: each grouped W_l from its group sums
+// (rows g*Q, g < P / Q, which hold the first log2(Q) levels of every cluster's
 // adjacent-pair tree), the rest of the row from the learner rows.  The tree over a
 // cluster's S / Q group sums has the same levels above them as the tree over its S
 // rows (Q divides S, so every group is a complete, aligned sub-tree), so the means
 // are the bits of do_local_means.
 int do_local_means_grouped(hier_avg* h) {
   const int64_t P = h->P, S = h->S, Q = h->upd_group, ld = h->ld;
-  const int64_t w1 = static_cast<int64_t>(h->dims[0]) * h->dims[1];   // W_1 at column 0
-  const double bytes = 4.0 * (P / Q) * w1 + 4.0 * P * (ld - w1) + 4.0 * (P / S) * ld;
+  const std::vector<AvgRange> rs = avg_ranges(h);
+  double bytes = 4.0 * (P / S) * ld;
+  for (const AvgRange& r : rs) bytes += 4.0 * (r.grouped ? P / Q : P) * (r.c1 - r.c0);
   return h->timed(HA_KERNEL_LOCAL_AVG, bytes, double(P) * ld, [&] {
-    ++h->launches;   // two launches
-    cudaError_t e = ha::launch_group_sum_mean_to(h->params, P / Q, S / Q, w1, Q * ld,
-                                                 static_cast<float>(S), h->means(), ld, h->stream);
-    if (e != cudaSuccess) return e;
-    return ha::launch_group_mean_to(h->params + w1, P, S, ld - w1, ld, h->means() + w1, h->stream);
+    h->launches += static_cast<int64_t>(rs.size()) - 1;   // one launch per range
+    for (const AvgRange& r : rs) {
+      const cudaError_t e =
+          r.grouped ? ha::launch_group_sum_mean_to(h->params + r.c0, P / Q, S / Q, r.c1 - r.c0, Q * ld,
+                                                   static_cast<float>(S), h->means() + r.c0, ld, h->stream)
+                    : ha::launch_group_mean_to(h->params + r.c0, P, S, r.c1 - r.c0, ld,
+                                               h->means() + r.c0, h->stream);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
   }, "local average");
 }
 
@@ -773,19 +820,24 @@ int do_local_global(hier_avg* h) {
   }, "local+global average");
 }
 
-// The fused last local average and global average after a grouped first-layer update:
-// W_1 from the group sums (rows g*Q), the rest of the row from the learner rows; every
-// row receives the global mean (the bits of do_local_global, as in do_local_means_grouped).
+// The fused last local average and global average after a grouped step: grouped W_l
+// from their group sums, the rest of the row from the learner rows; every row receives
+// the global mean (the bits of do_local_global, as in do_local_means_grouped).
 int do_local_global_grouped(hier_avg* h) {
   const int64_t P = h->P, S = h->S, Q = h->upd_group, ld = h->ld;
-  const int64_t w1 = static_cast<int64_t>(h->dims[0]) * h->dims[1];
-  const double bytes = 4.0 * (P / Q) * w1 + 4.0 * P * (ld - w1) + 4.0 * P * ld;
+  const std::vector<AvgRange> rs = avg_ranges(h);
+  double bytes = 4.0 * P * ld;
+  for (const AvgRange& r : rs) bytes += 4.0 * (r.grouped ? P / Q : P) * (r.c1 - r.c0);
   return h->timed(HA_KERNEL_GLOBAL_AVG, bytes, double(P) * ld, [&] {
-    ++h->launches;   // two launches
-    cudaError_t e = ha::launch_local_global_from_groups(h->params, Q * ld, Q, h->params, P, S, w1, ld,
-                                                        h->stream);
-    if (e != cudaSuccess) return e;
-    return ha::launch_local_global_mean(h->params + w1, P, S, ld - w1, ld, h->stream);
+    h->launches += static_cast<int64_t>(rs.size()) - 1;   // one launch per range
+    for (const AvgRange& r : rs) {
+      const cudaError_t e =
+          r.grouped ? ha::launch_local_global_from_groups(h->params + r.c0, Q * ld, Q, h->params + r.c0, P,
+                                                          S, r.c1 - r.c0, ld, h->stream)
+                    : ha::launch_local_global_mean(h->params + r.c0, P, S, r.c1 - r.c0, ld, h->stream);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
   }, "local+global average");
 }
 
@@ -883,11 +935,11 @@ int do_round(hier_avg* h, RowFeed* feed = nullptr) {
     }
     const bool block_end = r % h->K1 == 0;              // a local average follows step r
     const bool after_local = r > 1 && (r - 1) % h->K1 == 0;
-    bool grouped = false;
     if ((rc = do_step(h, h1_ready, !block_end && r < G, &h1_ready, after_local && compact,
-                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr, compact && block_end,
-                      &grouped)))
+                      feed && r == 1 && G > 1 ? feed->ev[1] : nullptr, compact && block_end)))
       return rc;
+    bool grouped = false;
+    for (char g : h->grp) grouped = grouped || g;
     if (r < G && block_end &&
         (rc = grouped ? do_local_means_grouped(h) : compact ? do_local_means(h) : do_local(h)))
       return rc;

@@ -140,6 +140,8 @@ struct TcBwdArgs {
   int64_t ld;
   float lr;
   int has_dx;                 // compute dZ_{l-1} (every layer but the first)
+  int no_update;              // k_tc_backward: dZ_{l-1} and b_{l-1} only; W_l is neither
+                              // updated nor stored (a grouped update follows)
   float* bias_prev;           // learner 0's b_{l-1}, written (row j)
   const float* bias_prev_src; // b_{l-1} read for learner j at row j / src_div
   int src_div;                // learner j's W (and b_{l-1}) read from row j / src_div of

@@ -1201,6 +1201,9 @@ __device__ __forceinline__ bool bwd_piece_end(const TcBwdArgs& a, const FwdItem&
   return true;
 }
 
+// kNoUpd: dZ_{l-1} and b_{l-1} only (TcBwdArgs::no_update), compiled separately so that
+// the full backward carries none of its branches.
+template <bool kNoUpd>
 __global__ void __launch_bounds__(kBwdThreads, 1)
     k_tc_backward(const __grid_constant__ CUtensorMap tm_wl, const __grid_constant__ CUtensorMap tm_ws,
                   const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_dz,
@@ -1339,8 +1342,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         mbar_wait(&zfull[u % nz], (u / nz) & 1, a.err);
   } else if (warp == 7) {
     // Store each updated chunk; its slot is released once the TMA has read it (two
-    // stores in flight).
+    // stores in flight).  no_update: the slot is released as soon as it has been read.
     const uint64_t stream = l2_weight_policy(a.w_stream != 0);
+    const bool store = !kNoUpd;
     int i = 0;
     bool ok = true;
     FwdItem f;
@@ -1350,6 +1354,10 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         for (int c = f.c_lo; c < f.c_hi; ++c, ++i) {
           const int s = i % nw;
           if (!mbar_wait(&upd[s], (i / nw) & 1, a.err)) { ok = false; break; }
+          if (!store) {
+            mbar_arrive(&wempty[s]);
+            continue;
+          }
           tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, j, stream);
           tma_store_commit();
           if (i > 0) {
@@ -1360,7 +1368,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       }
       ok = __all_sync(0xffffffffu, ok);
     }
-    if (lane == 0) {
+    if (lane == 0 && store) {
       tma_store_wait_read_all();   // (before the shared memory is released)
       if (i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
     }
@@ -1380,13 +1388,15 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
           const int sz = i % nz, b = i & 1;
           if (!mbar_wait(&zfull[sz], (i / nz) & 1, a.err)) { ok = false; break; }
-          if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
-          tc_fence_after();
           const uint32_t zs = smem_u32(zb(sz));
-          for (int kk = 0; kk < kb; ++kk)
-            tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
-                        umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
-          tc_commit(&dwdone[b]);
+          if constexpr (!kNoUpd) {
+            if (i >= 2 && !mbar_wait(&dwfree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+            tc_fence_after();
+            for (int kk = 0; kk < kb; ++kk)
+              tc_mma_bf16(tmem + kBwdTmemW + 64 * b, umma_desc_sw128_mn(hs + kk * 2048, tbytes),
+                          umma_desc_sw128_mn(zs + kk * 2048, tbytes), idesc_dw, kk > 0 ? 1u : 0u);
+            tc_commit(&dwdone[b]);
+          }
           if (a.has_dx) {
             if (first) ++q;
             const int xb = q & 1;
@@ -1490,22 +1500,24 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&conv[b]);
         }
-        if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
-        tc_fence_after();
+        if constexpr (!kNoUpd) {
+          if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+          tc_fence_after();
 #pragma unroll
-        for (int qb = 0; qb < 4; ++qb) {
-          float d[16];
-          tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
-          tmem_ld_wait();
+          for (int qb = 0; qb < 4; ++qb) {
+            float d[16];
+            tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
+            tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
+            for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&dwfree[b]);
+#pragma unroll
+          for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
+          fence_proxy_async_smem();
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&dwfree[b]);
-#pragma unroll
-        for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
-        fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&upd[sw]);
         if (a.has_dx) {
@@ -2562,7 +2574,9 @@ cudaError_t tc_configure() {
   e = cudaFuncSetAttribute(k_tc_update_forward<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            kFwdSmemMax);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_tc_backward, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  e = cudaFuncSetAttribute(k_tc_backward<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tc_backward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tc_update<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kBwdSmemMax);
   if (e != cudaSuccess) return e;
@@ -2606,7 +2620,10 @@ cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_s
                                int P, cudaStream_t s) {
   (void)P;
   // dynamic work items, no CTA waits for another: an ordinary launch
-  return launch_pdl(k_tc_backward, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
+  if (a.no_update)
+    return launch_pdl(k_tc_backward<true>, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
+                      w_load, w_store, h_in, dz, a);
+  return launch_pdl(k_tc_backward<false>, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
                     w_load, w_store, h_in, dz, a);
 }
 

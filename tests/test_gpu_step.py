@@ -391,9 +391,16 @@ def test_fused_next_forward_equals_steps(w):
         ha2.local_average()
     ha2.global_average()
     # the literal sequence launches every kernel; round() saves the fused forwards and
-    # fuses the last local average into the global one, and takes each average from
-    # group sums of W_1 in a launch of its own (S even: K2 - 1 local, one local+global)
-    saved = n_fused + 1 - (w.K2 if w.S % 2 == 0 else 0)
+    # fuses the last local average into the global one.  With S even, each of the K2
+    # block ends stores group sums of W_1, and with quads (S a multiple of 4, B <= 32)
+    # of every later tensor-core layer's W too (a backward without update, then the
+    # grouped update); its average takes one launch per column range (each grouped W
+    # region and the range after it).
+    head = w.dims[-1] <= 16
+    quads = w.S % 4 == 0 and w.B <= 32
+    n_grouped = (len(w.dims) - 1 - (1 if head else 0)) if quads else 1
+    extra = (n_grouped - 1) + (2 * n_grouped - 1) if w.S % 2 == 0 else 0
+    saved = n_fused + 1 - w.K2 * extra
     assert ha2.launches() - n1 == n_round + saved
     ha1.check()
     ha2.check()
