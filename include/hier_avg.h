@@ -132,13 +132,19 @@ int hier_avg_global_average(hier_avg* h);
  * global average; the last local average is fused with the global one
  * (bit-identical to doing them in turn).  The other local averages write each
  * cluster's mean once, into the workspace, and the step that follows reads every
- * learner's parameters from its cluster's mean and writes the learner's row: the
- * values are those of the full write-back, and when the round returns every row of
- * params_dev holds its learner's parameters.  Within the round, a step whose successor
- * starts no local block and reads a contiguous batch also computes that successor's
- * first-layer output from the weights it has just updated (bf16 path, two or more
- * layers), so W_1 is read once per step; the results are those of calling
- * hier_avg_step in turn. */
+ * learner's parameters from its cluster's mean (forwarding groups of a cluster's
+ * learners with one product per weight tile) and writes the learner's row.  With S
+ * even (bf16 path), the step before each average stores, instead of every learner's
+ * updated weights, the sums of pairs or quads of a cluster's learners (the first
+ * levels of the averaging tree) in the first learner row of each pair or quad, and the
+ * average finishes the tree from them.  So within a round the rows of params_dev are
+ * scratch; the values every step and average computes are those of the literal
+ * sequence, and when the round returns every row holds its learner's parameters.
+ * Within the round, a step whose successor starts no local block and reads a
+ * contiguous batch also computes that successor's first-layer output from the weights
+ * it has just updated (bf16 path, two or more layers), so W_1 is read once per step;
+ * the results are those of calling hier_avg_step, hier_avg_local_average and
+ * hier_avg_global_average in turn, bit for bit. */
 int hier_avg_round(hier_avg* h);
 
 /* Global averaging interval in local steps: hier_avg_round then runs `steps` local
