@@ -120,6 +120,68 @@ __global__ void __launch_bounds__(256) k_local_global_pow2(const float4* src, in
   store_rows(w + c, ld_v, S * G, m);
 }
 
+// The same two kernels with each column's rows split between two threads (threadIdx.y),
+// for short rows (D small against the GPU): twice the threads, each walking half the
+// rows.  The tree over 2^LOG rows is the tree over each half joined by one addition
+// (first half + second half), so the result has the same bits.  blockDim = (128, 2).
+template <int LOG>
+__global__ void __launch_bounds__(256) k_mean_pow2_split(float4* w, int64_t ld_v, int64_t cols_v) {
+  __shared__ float4 part[128];
+  grid_dep_wait();
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * 128 + threadIdx.x;
+  const bool valid = c < cols_v;
+  constexpr int H = 1 << (LOG - 1);
+  float4* p = w + static_cast<int64_t>(blockIdx.y) * (int64_t(1) << LOG) * ld_v + c +
+              static_cast<int64_t>(threadIdx.y) * H * ld_v;
+  float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (valid) x = tree_pow2<LOG - 1>(p, ld_v);
+  if (threadIdx.y == 1) part[threadIdx.x] = x;
+  __syncthreads();
+  if (threadIdx.y == 0) part[threadIdx.x] = vdiv(vadd(x, part[threadIdx.x]), static_cast<float>(1 << LOG));
+  __syncthreads();
+  if (valid) store_rows(p, ld_v, H, part[threadIdx.x]);
+}
+
+// (threadIdx.y = which half of the G clusters; the first G / 2 clusters' S copies form a
+// complete sub-tree of the global tree.)
+template <int LOGQ, int LOGS, int LOGG>
+__global__ void __launch_bounds__(256) k_local_global_pow2_split(const float4* src, int64_t src_ld_v,
+                                                                 float4* w, int64_t ld_v,
+                                                                 int64_t cols_v) {
+  __shared__ float4 part[128];
+  grid_dep_wait();
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * 128 + threadIdx.x;
+  const bool valid = c < cols_v;
+  constexpr int S = 1 << LOGS, G2 = 1 << (LOGG - 1), N = 1 << (LOGS - LOGQ);
+  const int g0 = static_cast<int>(threadIdx.y) * G2;
+  float4 half = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (valid) {
+    const float4* q = src + c;
+    float4 stack[LOGG];
+#pragma unroll
+    for (int g = 0; g < G2; ++g) {
+      float4 x = vdiv(tree_pow2<LOGS - LOGQ>(q + static_cast<int64_t>(g0 + g) * N * src_ld_v, src_ld_v),
+                      static_cast<float>(S));
+#pragma unroll
+      for (int l = 0; l < LOGS; ++l) x = vadd(x, x);
+      int l = 0;
+#pragma unroll
+      for (; l < LOGG - 1; ++l) {
+        if (((g >> l) & 1) == 0) break;
+        x = vadd(stack[l], x);
+      }
+      stack[l] = x;
+    }
+    half = stack[LOGG - 1];
+  }
+  if (threadIdx.y == 1) part[threadIdx.x] = half;
+  __syncthreads();
+  if (threadIdx.y == 0)
+    part[threadIdx.x] = vdiv(vadd(half, part[threadIdx.x]), static_cast<float>(S * (2 * G2)));
+  __syncthreads();
+  if (valid) store_rows(w + c + static_cast<int64_t>(g0) * S * ld_v, ld_v, G2 * S, part[threadIdx.x]);
+}
+
 // Generic path: any n (also non-powers of two) and scalar columns.  The binary
 // counter lives in a small local array; after n pushes its pending partials are
 // the set bits of n, folded from the smallest upward.
@@ -214,9 +276,19 @@ int ilog2_exact(int64_t n) {
   return l;
 }
 
+// Fewer columns than about two waves of one-thread-per-column CTAs: split each column's
+// rows between two threads.
+constexpr int64_t kSplitCols = 2 * 152 * 8 * 256;
+bool split_rows(int64_t cols_v, int64_t groups) { return cols_v * groups <= kSplitCols; }
+
 template <int LOG>
 void launch_mean_pow2(float4* w, int64_t ld_v, int64_t cols_v, int64_t groups,
                       cudaStream_t s) {
+  if (split_rows(cols_v, groups)) {
+    dim3 grid(static_cast<unsigned>((cols_v + 127) / 128), static_cast<unsigned>(groups));
+    launch_pdl(k_mean_pow2_split<LOG>, grid, dim3(128, 2), 0, s, false, 1, w, ld_v, cols_v);
+    return;
+  }
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads),
             static_cast<unsigned>(groups));
   launch_pdl(k_mean_pow2<LOG>, grid, dim3(kThreads), 0, s, false, 1, w, ld_v, cols_v);
@@ -273,6 +345,14 @@ bool mean_pow2_dispatch(int log, float4* w, int64_t ld_v, int64_t cols_v, int64_
 template <int LOGQ, int LOGS, int LOGG>
 void launch_lg(const float4* src, int64_t src_ld_v, float4* w, int64_t ld_v, int64_t cols_v,
                cudaStream_t s) {
+  if constexpr (LOGG >= 1) {
+    if (split_rows(cols_v, 1)) {
+      dim3 grid(static_cast<unsigned>((cols_v + 127) / 128));
+      launch_pdl(k_local_global_pow2_split<LOGQ, LOGS, LOGG>, grid, dim3(128, 2), 0, s, false, 1, src,
+                 src_ld_v, w, ld_v, cols_v);
+      return;
+    }
+  }
   dim3 grid(static_cast<unsigned>((cols_v + kThreads - 1) / kThreads));
   launch_pdl(k_local_global_pow2<LOGQ, LOGS, LOGG>, grid, dim3(kThreads), 0, s, false, 1, src,
              src_ld_v, w, ld_v, cols_v);
