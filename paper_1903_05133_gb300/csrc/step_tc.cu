@@ -1112,21 +1112,29 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 // tiles (one per SM) split into pieces of TcBwdArgs::piece_chunks chunks; a piece
 // writes its dH^T partial to its slot, and the piece that completes a tile adds the
 // tile's partials in piece order and runs the epilogue (no CTA waits for another).
-// Warps 0-3: thread t owns input feature i0 + t (TMEM lane t): it converts its column
-// of the fp32 chunk to the bf16 A tile, applies the update in shared memory and runs
-// the tile epilogue.  Warp 4 claims the work items and loads W chunks and each item's
-// H tile, warp 5 issues the MMAs, warp 6 loads dZ tiles, warp 7 TMA-stores updated
-// chunks (bulk stores: per-thread row stores of the same bytes ran at half the speed)
-// and frees their slots once read.  Each waiting role has a warp of its own: a lane
-// blocked in an mbarrier wait holds up the other lanes of its warp.
+// Warps 0-3 and 8-11: the two threads (w % 4, lane) of warps w and w + 8 own input
+// feature i0 + 32 (w % 4) + lane (a TMEM lane), each half of the chunk's 64 outputs and
+// half of the dH^T columns: they convert their half column of the fp32 chunk to the bf16
+// A tile, apply the update in shared memory and promote dH^T; the tile epilogue gathers
+// the row in TMEM for one of them.  (With four converter warps, one thread per column,
+// the converters set the pace of the pipeline.)  Warp 4 claims the work items and loads
+// W chunks and each item's H tile, warp 5 issues the MMAs, warp 6 loads dZ tiles, warp 7
+// TMA-stores updated chunks (bulk stores: per-thread row stores of the same bytes ran at
+// half the speed) and frees their slots once read.  Each waiting role has a warp of its
+// own: a lane blocked in an mbarrier wait holds up the other lanes of its warp.
+// (k_tc_update keeps four converter warps, one thread per column, for Q = 1.)
 constexpr int kBwdConv = 128;
 constexpr int kBwdThreads = kBwdConv + 128;
+// k_tc_backward: eight converter warps (0-3 and 8-11), each thread half of a column.
+constexpr int kBxConv = 256;
+constexpr int kBxThreads = kBxConv + 128;
 constexpr int kBwdWf32 = 64 * 128 * 4;                 // 32 KB fp32 W chunk [64 o][128 i]
 constexpr int kBwdWRingMax = 5, kBwdZRingMax = 8;
 constexpr int kBwdSmemMax = 227 * 1024;
-// TMEM columns: dH^T accumulators at 0 and 64, dW^T at 128 and 192, W^T (A) at 256, 288.
+// TMEM columns: dH^T accumulators at 0 and 64, dW^T at 128 and 192, W^T (A) at 256, 288,
+// and (k_tc_backward) the tile's promoted dH^T gathered for its epilogue at 320.
 constexpr uint32_t kBwdTmemCols = 512;
-constexpr uint32_t kBwdTmemW = 128, kBwdTmemA = 256;
+constexpr uint32_t kBwdTmemW = 128, kBwdTmemA = 256, kBwdTmemS = 320;
 
 // Layout: W ring | 2 H tiles (2 x [Bn][64] bf16 each) | dZ ring ([Bn][64] bf16) | barriers.
 __host__ __device__ constexpr int bwd_wring(int Bn) { return (void)Bn, 5; }
@@ -1144,67 +1152,10 @@ static_assert(bwd_zring(64) >= 4 && bwd_zring(48) >= 6 && bwd_zring(32) >= 8 && 
                   bwd_smem(32) <= kBwdSmemMax && bwd_smem(16) <= kBwdSmemMax,
               "backward shared-memory plan");
 
-// The backward's counterpart of piece_end: thread t holds row t of the tile's dH^T
-// partial (all Bn columns) in accx.  Slot (tail tile tt, piece p) =
-// part[((tt * np + p) * 128 + t) * Bn].
-__device__ __forceinline__ bool bwd_piece_end(const TcBwdArgs& a, const FwdItem& f, int t,
-                                              float* accx, GroupSync& gsync, volatile int* flag,
-                                              bool& ok) {
-  const int tt = f.tau - a.n_whole;
-  const int64_t pstride = static_cast<int64_t>(128) * a.Bn;
-  float* mine = a.part + (static_cast<int64_t>(tt) * f.np + f.piece) * pstride +
-                static_cast<int64_t>(t) * a.Bn;
-#pragma unroll
-  for (int cb = 0; cb < 64; cb += 4)
-    if (cb < a.Bn)
-      __stcg(reinterpret_cast<float4*>(mine + cb),
-             make_float4(accx[cb], accx[cb + 1], accx[cb + 2], accx[cb + 3]));
-  if (!gsync()) { ok = false; return false; }   // every converter thread's partial is written
-  if (t == 0) {
-    fence_acq_rel_gpu();           // release: the CTA's partial before the count
-    const int before = atomicAdd(a.counters + tt, 1);
-    const int last = before == f.np - 1;
-    if (last) {
-      fence_acq_rel_gpu();         // acquire: every other piece's partial before the reads
-      a.counters[tt] = 0;          // ready for the next launch
-    }
-    *flag = last;
-  }
-  if (!gsync()) { ok = false; return false; }
-  if (!*flag) return false;
-  // accx = P_0 + P_1 + ... in piece order; two pieces' loads in flight at once
-  const float* src = a.part + static_cast<int64_t>(tt) * f.np * pstride + static_cast<int64_t>(t) * a.Bn;
-#pragma unroll
-  for (int cb = 0; cb < 64; cb += 4) {
-    if (cb >= a.Bn) continue;
-    float4 s0 = __ldcg(reinterpret_cast<const float4*>(src + cb));
-    for (int p = 1; p < f.np; p += 2) {
-      const float4 v1 = __ldcg(reinterpret_cast<const float4*>(src + p * pstride + cb));
-      float4 v2 = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (p + 1 < f.np) v2 = __ldcg(reinterpret_cast<const float4*>(src + (p + 1) * pstride + cb));
-      s0.x = __fadd_rn(s0.x, v1.x);
-      s0.y = __fadd_rn(s0.y, v1.y);
-      s0.z = __fadd_rn(s0.z, v1.z);
-      s0.w = __fadd_rn(s0.w, v1.w);
-      if (p + 1 < f.np) {
-        s0.x = __fadd_rn(s0.x, v2.x);
-        s0.y = __fadd_rn(s0.y, v2.y);
-        s0.z = __fadd_rn(s0.z, v2.z);
-        s0.w = __fadd_rn(s0.w, v2.w);
-      }
-    }
-    accx[cb] = s0.x;
-    accx[cb + 1] = s0.y;
-    accx[cb + 2] = s0.z;
-    accx[cb + 3] = s0.w;
-  }
-  return true;
-}
-
 // kNoUpd: dZ_{l-1} and b_{l-1} only (TcBwdArgs::no_update), compiled separately so that
 // the full backward carries none of its branches.
 template <bool kNoUpd>
-__global__ void __launch_bounds__(kBwdThreads, 1)
+__global__ void __launch_bounds__(kBxThreads, 1)
     k_tc_backward(const __grid_constant__ CUtensorMap tm_wl, const __grid_constant__ CUtensorMap tm_ws,
                   const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_dz,
                   const TcBwdArgs a) {
@@ -1239,13 +1190,13 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
   auto wf = [&](int s) { return smem + s * kBwdWf32; };
   auto hb = [&](int s) { return h_base + s * 2 * tbytes; };
   auto zb = [&](int s) { return z_base + s * tbytes; };
-  constexpr int kConsumers = 3 + kBwdConv / 32;             // MMA, dZ, store + converter warps
+  constexpr int kConsumers = 3 + kBxConv / 32;              // MMA, dZ, store + converter warps
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kBwdWRingMax; ++s) {
       mbar_init(&wfull[s], 1);
       mbar_init(&wempty[s], 1);
-      mbar_init(&upd[s], kBwdConv / 32);
+      mbar_init(&upd[s], kBxConv / 32);
     }
     for (int s = 0; s < kBwdZRingMax; ++s) {
       mbar_init(&zfull[s], 1);
@@ -1253,19 +1204,19 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&hfull[b], 1);
-      mbar_init(&hempty[b], kBwdConv / 32);
-      mbar_init(&conv[b], kBwdConv / 32);
+      mbar_init(&hempty[b], kBxConv / 32);
+      mbar_init(&conv[b], kBxConv / 32);
       mbar_init(&afree[b], 1);
       mbar_init(&dwdone[b], 1);
-      mbar_init(&dwfree[b], kBwdConv / 32);
+      mbar_init(&dwfree[b], kBxConv / 32);
       mbar_init(&xf[b], 1);
-      mbar_init(&xr[b], kBwdConv / 32);
+      mbar_init(&xr[b], kBxConv / 32);
     }
     for (int q = 0; q < kQueue; ++q) {
       mbar_init(&queue.full[q], 1);
       mbar_init(&queue.empty[q], kConsumers);
     }
-    mbar_init(gbar, kBwdConv);
+    mbar_init(gbar, kBxConv);
     mbar_init(done, 1);
     fence_barrier_init();
   }
@@ -1421,26 +1372,29 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       mbar_wait(done, 0, a.err);
     }
   } else {
-    // ---- warps 0-3
-    const int t = threadIdx.x;
-    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+    // ---- warps 0-3 and 8-11: thread (warp % 4, lane) owns input feature i0 + t of the
+    // tile (TMEM lane t); warps 0-3 outputs 0-31 of each chunk and the dH^T column blocks
+    // 0 and 2 (16 samples each), warps 8-11 outputs 32-63 and blocks 1 and 3
+    const int t = 32 * (warp & 3) + lane, hf = warp >= 8 ? 1 : 0, o0 = 32 * hf;
+    const uint32_t tbase = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
     GroupSync gsync{gbar, 0, a.err};
-    float accx[64];                                // dH^T[i0 + t][0 .. Bn), promoted
+    float accx[32];                                // dH^T[i0 + t][16 (2m + hf) + q], promoted
 #pragma unroll
-    for (int q = 0; q < 64; ++q) accx[q] = 0.f;
+    for (int q = 0; q < 32; ++q) accx[q] = 0.f;
     int qc = -1, drained = 0;
     auto drain = [&]() -> bool {
       const int xb = drained & 1;
       if (!wait_warp(&xf[xb], (drained >> 1) & 1, a.err)) return false;
       tc_fence_after();
 #pragma unroll
-      for (int cb = 0; cb < 64; cb += 16) {
+      for (int m = 0; m < 2; ++m) {
+        const int cb = 16 * (2 * m + hf);
         if (cb < a.Bn) {
           float v[16];
           tmem_ld16(tbase + 64 * xb + cb, v);
           tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < 16; ++q) accx[cb + q] = __fadd_rn(accx[cb + q], v[q]);
+          for (int q = 0; q < 16; ++q) accx[16 * m + q] = __fadd_rn(accx[16 * m + q], v[q]);
         }
       }
       tc_fence_before();
@@ -1449,29 +1403,114 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
       ++drained;
       return true;
     };
-    // dZ_{l-1}[b][i] = dH[b][i] * (H_{l-1}[b][i] > 0), b < B; b_{l-1}[i] -= lr sum_b.
-    // (The item's H tile landed long ago; the wait makes the TMA's writes visible here.)
-    auto epilogue = [&](int tau, int k) -> bool {
-      const int j = tau / a.s_tiles, fi = (tau - j * a.s_tiles) * 128 + t;
-      if (!wait_warp(&hfull[k & 1], (k >> 1) & 1, a.err)) return false;
-      if (fi < a.in) {
-        const uint8_t* hcol = hb(k & 1) + (t >> 6) * a.Bn * 128;
-        __nv_bfloat16* dz = a.dz_prev + static_cast<int64_t>(j) * a.Bn * a.pitch_in + fi;
-        float db = 0.f;
+    // A split tile's piece ends: this thread's blocks go to the piece's slot (slot (tail
+    // tile tt, piece p) = part[((tt * np + p) * 128 + t) * Bn]); the piece completing the
+    // tile replaces them with the sums of the tile's partials in piece order.
+    auto piece_end = [&](const FwdItem& f, bool& ok) -> bool {
+      const int tt = f.tau - a.n_whole;
+      const int64_t pstride = static_cast<int64_t>(128) * a.Bn;
+      float* mine = a.part + (static_cast<int64_t>(tt) * f.np + f.piece) * pstride +
+                    static_cast<int64_t>(t) * a.Bn;
 #pragma unroll
-        for (int b = 0; b < 64; ++b) {
-          if (b < a.B) {
-            const __nv_bfloat16 hv =
-                *reinterpret_cast<const __nv_bfloat16*>(hcol + sw128_offset(b, t & 63));
-            const float x = __bfloat162float(hv) > 0.f ? accx[b] : 0.f;
-            db = __fadd_rn(db, x);
-            dz[static_cast<int64_t>(b) * a.pitch_in] = __float2bfloat16_rn(x);
-          }
+      for (int m = 0; m < 2; ++m) {
+        const int cb = 16 * (2 * m + hf);
+        if (cb < a.Bn) {
+#pragma unroll
+          for (int q = 0; q < 16; q += 4)
+            __stcg(reinterpret_cast<float4*>(mine + cb + q),
+                   make_float4(accx[16 * m + q], accx[16 * m + q + 1], accx[16 * m + q + 2],
+                               accx[16 * m + q + 3]));
         }
-        const float bv = a.bias_prev_src[static_cast<int64_t>(j / a.src_div) * a.ld + fi];
-        a.bias_prev[static_cast<int64_t>(j) * a.ld + fi] = __fsub_rn(bv, __fmul_rn(a.lr, db));
+      }
+      if (!gsync()) { ok = false; return false; }
+      if (threadIdx.x == 0) {
+        fence_acq_rel_gpu();
+        const int before = atomicAdd(a.counters + tt, 1);
+        const int last = before == f.np - 1;
+        if (last) {
+          fence_acq_rel_gpu();
+          a.counters[tt] = 0;
+        }
+        *last_flag = last;
+      }
+      if (!gsync()) { ok = false; return false; }
+      if (!*reinterpret_cast<volatile int*>(last_flag)) return false;
+      const float* src = a.part + static_cast<int64_t>(tt) * f.np * pstride + static_cast<int64_t>(t) * a.Bn;
+#pragma unroll
+      for (int m = 0; m < 2; ++m) {
+        const int cb = 16 * (2 * m + hf);
+        if (cb >= a.Bn) continue;
+#pragma unroll
+        for (int q = 0; q < 16; q += 4) {
+          float4 s0 = __ldcg(reinterpret_cast<const float4*>(src + cb + q));
+          for (int p = 1; p < f.np; ++p) {
+            const float4 v = __ldcg(reinterpret_cast<const float4*>(src + p * pstride + cb + q));
+            s0.x = __fadd_rn(s0.x, v.x);
+            s0.y = __fadd_rn(s0.y, v.y);
+            s0.z = __fadd_rn(s0.z, v.z);
+            s0.w = __fadd_rn(s0.w, v.w);
+          }
+          accx[16 * m + q] = s0.x;
+          accx[16 * m + q + 1] = s0.y;
+          accx[16 * m + q + 2] = s0.z;
+          accx[16 * m + q + 3] = s0.w;
+        }
       }
       return true;
+    };
+    // dZ_{l-1}[b][i] = dH[b][i] * (H_{l-1}[b][i] > 0), b < B; b_{l-1}[i] -= lr sum_b.  The
+    // row's blocks are gathered in TMEM, so that one thread adds the bias gradient in
+    // sample order.  (The item's H tile landed long ago; the wait makes the TMA's writes
+    // visible here.)
+    auto epilogue = [&](int tau, int k) -> bool {
+#pragma unroll
+      for (int m = 0; m < 2; ++m) {
+        const int cb = 16 * (2 * m + hf);
+        if (cb < a.Bn) {
+          uint32_t r[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q) r[q] = __float_as_uint(accx[16 * m + q]);
+          tmem_st16(tbase + kBwdTmemS + cb, r);
+        }
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      if (!gsync()) return false;
+      tc_fence_after();
+      if (!wait_warp(&hfull[k & 1], (k >> 1) & 1, a.err)) return false;
+      const int j = tau / a.s_tiles, fi = (tau - j * a.s_tiles) * 128 + t;
+      if (hf == 0) {
+        float db = 0.f;
+        const uint8_t* hcol = hb(k & 1) + (t >> 6) * a.Bn * 128;
+        __nv_bfloat16* dz = a.dz_prev + static_cast<int64_t>(j) * a.Bn * a.pitch_in + fi;
+#pragma unroll
+        for (int cb = 0; cb < 64; cb += 16) {
+          if (cb < a.Bn) {
+            float v[16];
+            tmem_ld16(tbase + kBwdTmemS + cb, v);
+            tmem_ld_wait();
+            if (fi < a.in) {
+#pragma unroll
+              for (int q = 0; q < 16; ++q) {
+                const int b = cb + q;
+                if (b < a.B) {
+                  const __nv_bfloat16 hv =
+                      *reinterpret_cast<const __nv_bfloat16*>(hcol + sw128_offset(b, t & 63));
+                  const float x = __bfloat162float(hv) > 0.f ? v[q] : 0.f;
+                  db = __fadd_rn(db, x);
+                  dz[static_cast<int64_t>(b) * a.pitch_in] = __float2bfloat16_rn(x);
+                }
+              }
+            }
+          }
+        }
+        if (fi < a.in) {
+          const float bv = a.bias_prev_src[static_cast<int64_t>(j / a.src_div) * a.ld + fi];
+          a.bias_prev[static_cast<int64_t>(j) * a.ld + fi] = __fsub_rn(bv, __fmul_rn(a.lr, db));
+        }
+      }
+      tc_fence_before();
+      return gsync();   // the gathered blocks are read before the next tile writes them
     };
     bool ok = true;
     int i = 0;
@@ -1481,20 +1520,17 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
         const bool tlast = c == f.c_hi - 1;
         const int sw = i % nw, b = i & 1;
         if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
-        float* w = reinterpret_cast<float*>(wf(sw));
-        float wv[64];
+        float* w = reinterpret_cast<float*>(wf(sw)) + o0 * 128;
+        float wv[32];
 #pragma unroll
-        for (int o = 0; o < 64; ++o) wv[o] = w[o * 128 + t];
+        for (int o = 0; o < 32; ++o) wv[o] = w[o * 128 + t];
         if (a.has_dx) {
           if (i >= 2 && !wait_warp(&afree[b], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
           tc_fence_after();
+          uint32_t pk[16];
 #pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            uint32_t pk[16];
-#pragma unroll
-            for (int q = 0; q < 16; ++q) pk[q] = pack_bf16x2(wv[32 * hh + 2 * q], wv[32 * hh + 2 * q + 1]);
-            tmem_st16(tbase + kBwdTmemA + 32 * b + 16 * hh, pk);
-          }
+          for (int q = 0; q < 16; ++q) pk[q] = pack_bf16x2(wv[2 * q], wv[2 * q + 1]);
+          tmem_st16(tbase + kBwdTmemA + 32 * b + 16 * hf, pk);
           tmem_st_wait();
           tc_fence_before();
           __syncwarp();
@@ -1504,9 +1540,9 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           if (!wait_warp(&dwdone[b], (i >> 1) & 1, a.err)) { ok = false; break; }
           tc_fence_after();
 #pragma unroll
-          for (int qb = 0; qb < 4; ++qb) {
+          for (int qb = 0; qb < 2; ++qb) {
             float d[16];
-            tmem_ld16(tbase + kBwdTmemW + 64 * b + 16 * qb, d);
+            tmem_ld16(tbase + kBwdTmemW + 64 * b + o0 + 16 * qb, d);
             tmem_ld_wait();
 #pragma unroll
             for (int q = 0; q < 16; ++q) wv[16 * qb + q] = __fsub_rn(wv[16 * qb + q], __fmul_rn(a.lr, d[q]));
@@ -1515,7 +1551,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&dwfree[b]);
 #pragma unroll
-          for (int o = 0; o < 64; ++o) w[o * 128 + t] = wv[o];
+          for (int o = 0; o < 32; ++o) w[o * 128 + t] = wv[o];
           fence_proxy_async_smem();
         }
         __syncwarp();
@@ -1526,11 +1562,11 @@ __global__ void __launch_bounds__(kBwdThreads, 1)
             while (ok && drained <= qc)
               if (!drain()) ok = false;
             if (ok) {
-              const bool fin = f.np == 1 || bwd_piece_end(a, f, t, accx, gsync, last_flag, ok);
+              const bool fin = f.np == 1 || piece_end(f, ok);
               if (ok && fin && !epilogue(f.tau, k)) ok = false;
               ok = __all_sync(0xffffffffu, ok);
 #pragma unroll
-              for (int q = 0; q < 64; ++q) accx[q] = 0.f;
+              for (int q = 0; q < 32; ++q) accx[q] = 0.f;
             }
           } else if (p % kSegChunks == kSegChunks - 1 && qc >= 1 && drained < qc) {
             if (!drain()) ok = false;
@@ -2655,9 +2691,9 @@ cudaError_t launch_tc_backward(const CUtensorMap& w_load, const CUtensorMap& w_s
   (void)P;
   // dynamic work items, no CTA waits for another: an ordinary launch
   if (a.no_update)
-    return launch_pdl(k_tc_backward<true>, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
+    return launch_pdl(k_tc_backward<true>, dim3(a.ctas), dim3(kBxThreads), bwd_smem(a.Bn), s, false, 1,
                       w_load, w_store, h_in, dz, a);
-  return launch_pdl(k_tc_backward<false>, dim3(a.ctas), dim3(kBwdThreads), bwd_smem(a.Bn), s, false, 1,
+  return launch_pdl(k_tc_backward<false>, dim3(a.ctas), dim3(kBxThreads), bwd_smem(a.Bn), s, false, 1,
                     w_load, w_store, h_in, dz, a);
 }
 
