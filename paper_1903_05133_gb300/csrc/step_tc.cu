@@ -771,6 +771,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
 constexpr int kGfWRing = 5;
 constexpr uint32_t kGfTmemCols = 512;          // accumulators at 0 and 128, A tiles at 256
 constexpr uint32_t kGfTmemA = 256;
+// A tiles in flight (32 TMEM columns each): the converters run up to kGfABufs chunks
+// ahead of the MMA, which covers their pause at every accumulator drain.
+constexpr int kGfABufs = 4;
+static_assert(kGfTmemA + 32 * kGfABufs <= kGfTmemCols && (kGfABufs & (kGfABufs - 1)) == 0,
+              "grouped forward TMEM plan");
 __host__ __device__ constexpr int gf_h_off() { return kGfWRing * kFwdWf32; }
 __host__ __device__ constexpr int gf_hring(int N) {
   return (kFwdSmemMax - 1024 - kBarBytes - gf_h_off()) / (N * 128) < kFwdHRingMax
@@ -830,9 +835,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
   uint64_t* wempty = wfull + kFwdWRingMax;
   uint64_t* hfull = wempty + kFwdWRingMax;
   uint64_t* hempty = hfull + kFwdHRingMax;
-  uint64_t* conv = hempty + kFwdHRingMax;  // [2] A tile written to TMEM
-  uint64_t* wfree = conv + 2;              // [2] A tile consumed by the MMA
-  uint64_t* accf = wfree + 2;              // [2] accumulator segment complete
+  uint64_t* conv = hempty + kFwdHRingMax;  // [kGfABufs] A tile written to TMEM
+  uint64_t* wfree = conv + kGfABufs;       // [kGfABufs] A tile consumed by the MMA
+  uint64_t* accf = wfree + kGfABufs;       // [2] accumulator segment complete
   uint64_t* accr = accf + 2;               // [2] accumulator segment drained
   uint64_t* gbar = accr + 2;
   uint64_t* done = gbar + 1;
@@ -853,9 +858,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       mbar_init(&hfull[s], 1);
       mbar_init(&hempty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kGfABufs; ++b) {
       mbar_init(&conv[b], kFwdConv / 32);
       mbar_init(&wfree[b], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
       mbar_init(&accf[b], 1);
       mbar_init(&accr[b], kFwdConv);
     }
@@ -944,11 +951,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
         for (int c = f.c_lo, p = 0; c < f.c_hi; ++c, ++p, ++i) {
           const bool tlast = c == f.c_hi - 1;
           const bool first = p % kSegChunks == 0, last = tlast || p % kSegChunks == kSegChunks - 1;
-          const int sh = i % nh, b = i & 1;
+          const int sh = i % nh, b = i & (kGfABufs - 1);
           if (first) ++q;
           const int ab = q & 1;
           if (first && q >= 2 && !mbar_wait(&accr[ab], ((q >> 1) - 1) & 1, a.err)) { ok = false; break; }
-          if (!mbar_wait(&conv[b], (i >> 1) & 1, a.err)) { ok = false; break; }
+          if (!mbar_wait(&conv[b], (i / kGfABufs) & 1, a.err)) { ok = false; break; }
           if (!mbar_wait(&hfull[sh], (i / nh) & 1, a.err)) { ok = false; break; }
           tc_fence_after();
           const uint32_t at = tmem + kGfTmemA + 32 * b;
@@ -1089,9 +1096,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1)
       const float tbias = ob < a.out ? a.bias[static_cast<int64_t>(f.q * G / a.b_div) * a.ld + ob] : 0.f;
       for (int c = f.c_lo, p = 0; c < f.c_hi && ok; ++c, ++p, ++i) {
         const bool tlast = c == f.c_hi - 1;
-        const int sw = i % nw, bb = i & 1;
+        const int sw = i % nw, bb = i & (kGfABufs - 1);
         if (!wait_warp(&wfull[sw], (i / nw) & 1, a.err)) { ok = false; break; }
-        if (i >= 2 && !wait_warp(&wfree[bb], ((i >> 1) - 1) & 1, a.err)) { ok = false; break; }
+        if (i >= kGfABufs && !wait_warp(&wfree[bb], ((i / kGfABufs) - 1) & 1, a.err)) { ok = false; break; }
         tc_fence_after();
         {
           const int row = 32 * (warp & 3) + lane, half = warp >> 2;
