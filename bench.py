@@ -505,17 +505,27 @@ def run_ours(args):
         if ws > 1:
             dist.barrier()
         torch.cuda.synchronize()
+        # events on the handle's stream around every call: the device time of each
+        # round from host memory, next to the host clock over all of them
+        e_a = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        e_b = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         t0 = time.perf_counter()
-        for _ in range(args.steps):
+        for k in range(args.steps):
+            e_a[k].record()
             ha.round_host(Xh, yh, loss)
+            e_b[k].record()
         torch.cuda.synchronize()
         Te = job_seconds(time.perf_counter() - t0, ws, dev)
+        dev_ms = sorted(a.elapsed_time(b) for a, b in zip(e_a, e_b))
         rows = w.B * w.K1 * w.K2
         es = 2 if w.precision == "bf16" else 4
         line["e2e"] = {"value": replica_throughput(ws, per_round, args.steps, Te), "unit": UNIT,
-                       "h2d_bytes_per_step": w.P * rows * (w.dims[0] * es + 4),
+                       "h2d_bytes_per_step": w.P * rows * w.dims[0] * es + w.P * w.N * 4,
                        "d2h_bytes_per_step": w.P * 4,
-                       "api": "hier_avg_round_host (pinned host X, y; loss read back)"}
+                       "api": "hier_avg_round_host (pinned host X, y; loss read back)",
+                       "ms_per_step": 1000 * Te / args.steps,
+                       "device_ms_per_step_median": statistics.median(dev_ms),
+                       "device_ms_per_step_max": dev_ms[-1]}
         del Xh, yh
 
     if rank == 0 and not args.no_sweep_point:

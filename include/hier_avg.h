@@ -166,14 +166,16 @@ int hier_avg_set_lr(hier_avg* h, float lr);
  * HA_EINVAL outside that range; HA_ECUDA if clearing device buffers fails. */
 int hier_avg_set_batch(hier_avg* h, int B);
 
-/* One round end to end from host memory: copies the rows this round reads from
- * X_host [P, N, d_0] / y_host [P, N] (pinned memory recommended) into the bound
- * device data set, runs hier_avg_round, and copies the per-learner loss of the
- * round's last step into loss_host [P].  The copies (one pitched copy of X and one
- * of y per chunk, for all learners) run on a stream of the library's own in chunks
- * of steps that double in length, issued between the kernel launches, and overlap
- * the kernels: a step waits only for the chunk holding the rows it reads (bf16 path;
- * the fp32 path copies the round's rows first).  Synchronises. */
+/* One round end to end from host memory: copies the rows of X_host [P, N, d_0] that
+ * this round reads, and all of y_host [P, N] (P * N * 4 bytes, one copy), into the
+ * bound device data set (pinned host memory recommended), runs hier_avg_round, and
+ * copies the per-learner loss of the round's last step into loss_host [P].  The rows
+ * of X go in chunks of steps that double in length, on a stream of the library's own,
+ * issued between the kernel launches, and overlap the kernels: a step waits only for
+ * the chunk holding the rows it reads (bf16 path; the fp32 path copies the round's
+ * rows first).  A chunk whose rows span at least 512 KB per learner is one copy per
+ * learner when a learner's parameter row holds at least 4 Mi values, otherwise a
+ * single pitched copy for all learners.  Synchronises. */
 int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host,
                         float* loss_host);
 

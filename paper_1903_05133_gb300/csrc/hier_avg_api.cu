@@ -852,23 +852,42 @@ int do_global(hier_avg* h) {
 
 int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 
-// Rows [r0, r0 + n) of every learner's data from host memory: one pitched copy for all
-// learners (X, then y).  (Measured from a pinned [32][100 MB] buffer: 205-211 GB/s for
-// rows of 0.75 to 25 MB, the rate of one contiguous copy per learner, at ~3 us of host
-// time instead of ~32 us for the 32 calls.)
-int copy_rows(hier_avg* h, const void* X_host, const int32_t* y_host, int64_t r0, int64_t n,
-              cudaStream_t cs) {
+// Rows [r0, r0 + n) of every learner's X from host memory.  Spans of at least
+// kRowCopySplit bytes per learner go as one contiguous copy per learner when a learner's
+// parameter row holds at least kRowCopyMinLd values, so that the P calls (~2.5 us of
+// host time each) hide behind the kernels of a step; otherwise the span goes as one
+// pitched copy for all learners, one call.  (Pitched copies of [32][0.75-12.6 MB] spans
+// ran at 190-209 GB/s in one process and at 18 GB/s later in the same process, after
+// a few rounds, while per-learner copies of the same spans kept 168-184 GB/s: with
+// pitched copies only, some hosts lost 3.5-30 % of the 12288-4096-4096-1000 round end to
+// end.  At 3072-512-10 a step takes ~50 us, and 16 more calls per chunk cost more than
+// the pitched copies lose.)
+constexpr int64_t kRowCopySplit = int64_t(512) << 10;
+constexpr int64_t kRowCopyMinLd = int64_t(4) << 20;
+
+int copy_rows(hier_avg* h, const void* X_host, int64_t r0, int64_t n, cudaStream_t cs) {
   const int64_t es = h->prec == HA_PREC_BF16 ? 2 : 4;
   const int64_t rowb = static_cast<int64_t>(h->dims[0]) * es;
   uint8_t* X = static_cast<uint8_t*>(const_cast<void*>(h->X));
   const uint8_t* Xh = static_cast<const uint8_t*>(X_host);
-  int32_t* y = const_cast<int32_t*>(h->y);
-  if (int rc = h->cuda(cudaMemcpy2DAsync(X + r0 * rowb, h->N * rowb, Xh + r0 * rowb, h->N * rowb,
-                                         n * rowb, h->P, cudaMemcpyHostToDevice, cs),
-                       "round_host: X copy"))
-    return rc;
-  return h->cuda(cudaMemcpy2DAsync(y + r0, h->N * 4, y_host + r0, h->N * 4, n * 4, h->P,
-                                   cudaMemcpyHostToDevice, cs), "round_host: y copy");
+  if (n * rowb < kRowCopySplit || h->ld < kRowCopyMinLd)
+    return h->cuda(cudaMemcpy2DAsync(X + r0 * rowb, h->N * rowb, Xh + r0 * rowb, h->N * rowb, n * rowb,
+                                     h->P, cudaMemcpyHostToDevice, cs), "round_host: X copy");
+  for (int j = 0; j < h->P; ++j) {
+    const int64_t off = (static_cast<int64_t>(j) * h->N + r0) * rowb;
+    if (int rc = h->cuda(cudaMemcpyAsync(X + off, Xh + off, n * rowb, cudaMemcpyHostToDevice, cs),
+                         "round_host: X copy"))
+      return rc;
+  }
+  return HA_OK;
+}
+
+// Every learner's labels, y_host [P, N] whole, in one contiguous copy (P * N * 4 bytes:
+// 0.5 MB for 32 learners of 4096 samples), ahead of the round's rows of X.
+int copy_labels(hier_avg* h, const int32_t* y_host, cudaStream_t cs) {
+  return h->cuda(cudaMemcpyAsync(const_cast<int32_t*>(h->y), y_host,
+                                 static_cast<size_t>(h->P) * h->N * 4, cudaMemcpyHostToDevice, cs),
+                 "round_host: y copy");
 }
 
 // round_host's row feed: the rows of the round's steps are copied from host memory on
@@ -880,7 +899,6 @@ int copy_rows(hier_avg* h, const void* X_host, const int32_t* y_host, int64_t r0
 struct RowFeed {
   hier_avg* h;
   const void* X_host;
-  const int32_t* y_host;
   int G;
   int issued_to = 0;            // steps [0, issued_to) have their copies issued
   int chunks = 0;
@@ -895,7 +913,7 @@ struct RowFeed {
     if (rows >= h->N) r0 = 0;
     while (left > 0) {
       const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
-      if (int rc = copy_rows(h, X_host, y_host, r0, n, h->copy_stream)) return rc;
+      if (int rc = copy_rows(h, X_host, r0, n, h->copy_stream)) return rc;
       left -= n;
       r0 = 0;
     }
@@ -1170,9 +1188,10 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
     const int64_t rows = static_cast<int64_t>(h->Bstep) * G;
     int64_t r0 = h->cursor % h->N, left = rows < h->N ? rows : h->N;
     if (rows >= h->N) r0 = 0;
+    if ((rc = copy_labels(h, y_host, h->stream))) return rc;
     while (left > 0) {
       const int64_t n = (r0 + left <= h->N) ? left : h->N - r0;
-      if ((rc = copy_rows(h, X_host, y_host, r0, n, h->stream))) return rc;
+      if ((rc = copy_rows(h, X_host, r0, n, h->stream))) return rc;
       left -= n;
       r0 = 0;
     }
@@ -1184,9 +1203,10 @@ int hier_avg_round_host(hier_avg* h, const void* X_host, const int32_t* y_host, 
     // the device-resident round.)  The copies start once the work already queued on the
     // handle's stream is done.
     if ((rc = h->cuda(cudaEventRecord(h->round_start, h->stream), "round_host: record")) ||
-        (rc = h->cuda(cudaStreamWaitEvent(h->copy_stream, h->round_start, 0), "round_host: wait")))
+        (rc = h->cuda(cudaStreamWaitEvent(h->copy_stream, h->round_start, 0), "round_host: wait")) ||
+        (rc = copy_labels(h, y_host, h->copy_stream)))
       return rc;
-    RowFeed feed{h, X_host, y_host, G};
+    RowFeed feed{h, X_host, G};
     feed.ev.assign(G, nullptr);
     if ((rc = do_round(h, &feed))) return rc;
   }

@@ -606,12 +606,20 @@ def test_full_size_round_equals_literal_sequence(w):
     assert torch.equal(p, p[:1].expand_as(p))
 
 
+# A parameter row of 4.2M values and 512 KB of rows per learner and step: spans of at
+# least 64 rows go learner by learner; the chunk of steps 2-3 wraps around N = 160 and
+# leaves a 32-row span, which goes as one pitched copy.
+HOST_ROWS = configs.Workload("mlp_bf16_host_rows", P=4, S=2, K1=2, K2=2, rounds=1,
+                             dims=(4096, 1024, 10), precision="bf16", N=160, B=64, lr=0.05,
+                             sigma_mu=0.1, init="he")
+
+
 # bf16 path: the rows are copied beside the kernels in chunks of steps that double in
 # length; SMALL_BF16's round reads more rows than each learner has (the chunks wrap
 # around N), FUSE_PIECES has 6 steps (chunks 0 | 1 | 2-3 | 4-5), a free global interval
 # of 7 steps ends on a short chunk.  fp32 path: the rows are copied ahead of the round.
 @pytest.mark.parametrize("w,G", [(SMALL_BF16, 0), (FUSE_THREE, 0), (FUSE_PIECES, 0),
-                                 (SMALL_BF16.replace(K1=3), 7), (SMALL_FP32, 0)],
+                                 (SMALL_BF16.replace(K1=3), 7), (SMALL_FP32, 0), (HOST_ROWS, 0)],
                          ids=lambda v: getattr(v, "name", str(v)))
 def test_round_host_matches_device_round(w, G):
     ha1, X, y = setup(w)
