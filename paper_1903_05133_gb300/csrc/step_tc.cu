@@ -1347,10 +1347,11 @@ __global__ void __launch_bounds__(kBxThreads, 1)
         mbar_wait(&zfull[u % nz], (u / nz) & 1, a.err);
   } else if (warp == 7) {
     // Store each updated chunk; its slot is released once the TMA has read it (two
-    // stores in flight).  no_update: the slot is released as soon as it has been read.
+    // stores in flight; when the chunks come from the cluster means, as soon as its own
+    // store has been read).  no_update: the slot is released as soon as it has been read.
     const uint64_t stream = l2_weight_policy(a.w_stream != 0);
-    const bool store = !kNoUpd;
-    int i = 0;
+    const bool store = !kNoUpd, eager = a.src_div > 1;
+    int i = 0, released = 0;
     bool ok = true;
     FwdItem f;
     for (int k = 0; ok && next_item(k, f); ++k) {
@@ -1365,9 +1366,14 @@ __global__ void __launch_bounds__(kBxThreads, 1)
           }
           tma_store_3d_hint(&tm_ws, wf(s), i0, c * 64, j, stream);
           tma_store_commit();
-          if (i > 0) {
+          if (eager) {
+            tma_store_wait_read_all();
+            mbar_arrive(&wempty[s]);
+            released = i + 1;
+          } else if (i > 0) {
             tma_store_wait_read_1();
             mbar_arrive(&wempty[(i - 1) % nw]);
+            released = i;
           }
         }
       }
@@ -1375,7 +1381,7 @@ __global__ void __launch_bounds__(kBxThreads, 1)
     }
     if (lane == 0 && store) {
       tma_store_wait_read_all();   // (before the shared memory is released)
-      if (i > 0) mbar_arrive(&wempty[(i - 1) % nw]);
+      if (i > released) mbar_arrive(&wempty[(i - 1) % nw]);
     }
   } else if (warp == 5) {
     const uint32_t idesc_dw = umma_idesc_bf16(128, 64) | (1u << 15) | (1u << 16);
@@ -2292,9 +2298,12 @@ __global__ void __launch_bounds__(kUfThreads, 1)
     }
   } else if (warp == 11) {
     // Store each updated W tile; its slot is released once the TMA has read it.  In
-    // cluster mode (a short layer) each slot is released as soon as its own store has
-    // been read; otherwise one store behind, two in flight.
+    // cluster mode (a short layer), and when the tiles come from the cluster means (the
+    // first step of a block, which the SMs' chunk rate bounds, not DRAM), each slot is
+    // released as soon as its own store has been read; otherwise one store behind, two
+    // in flight.
     const uint64_t stream = l2_weight_policy(a.w_stream != 0);
+    const bool eager = cq > 1 || a.w_div > 1;
     int i = 0, released = 0;
     bool ok = true;
     FwdItem f;
@@ -2307,7 +2316,7 @@ __global__ void __launch_bounds__(kUfThreads, 1)
           tma_store_3d_hint(&tm_ws, wf(s), c * 64, ot * 128, j, stream);
           tma_store_3d_hint(&tm_ws, wf(s) + kFwdWBox, c * 64 + 32, ot * 128, j, stream);
           tma_store_commit();
-          if (cq > 1) {
+          if (eager) {
             tma_store_wait_read_all();
             mbar_arrive(&wempty[s]);
             released = i + 1;
