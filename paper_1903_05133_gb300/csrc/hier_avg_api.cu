@@ -855,13 +855,12 @@ int round_steps(const hier_avg* h) { return h->G > 0 ? h->G : h->K1 * h->K2; }
 // Rows [r0, r0 + n) of every learner's X from host memory.  Spans of at least
 // kRowCopySplit bytes per learner go as one contiguous copy per learner when a learner's
 // parameter row holds at least kRowCopyMinLd values, so that the P calls (~2.5 us of
-// host time each) hide behind the kernels of a step; otherwise the span goes as one
-// pitched copy for all learners, one call.  (Pitched copies of [32][0.75-12.6 MB] spans
-// ran at 190-209 GB/s in one process and at 18 GB/s later in the same process, after
-// a few rounds, while per-learner copies of the same spans kept 168-184 GB/s: with
-// pitched copies only, some hosts lost 3.5-30 % of the 12288-4096-4096-1000 round end to
-// end.  At 3072-512-10 a step takes ~50 us, and 16 more calls per chunk cost more than
-// the pitched copies lose.)
+// host time each on a fast host) hide behind the kernels of a step; otherwise the span
+// goes as one pitched copy for all learners, one call.  (Pitched copies of
+// [32][0.75-12.6 MB] spans ran at 190-209 GB/s in one process and at 18 GB/s later in the
+// same process, after a few rounds, while per-learner copies of the same spans kept
+// 168-184 GB/s.  At 3072-512-10 a step takes ~50 us, and the host's calls are what
+// limits its round.)
 constexpr int64_t kRowCopySplit = int64_t(512) << 10;
 constexpr int64_t kRowCopyMinLd = int64_t(4) << 20;
 
