@@ -8,7 +8,7 @@ learner-samples per second (P * B * K1 * K2 per round).
 
   python bench.py [--gpus N --steps K --warmup W] [--workload mlp4096|mlp2048|mlp512|softmax]
   python bench.py --impl reference ...   # the CPU oracle on a bounded sample
-  python bench.py --sweep                # averaging-only sweep (P = 128), GB/s table
+  python bench.py --sweep [--sweep-D D ...]   # averaging-only sweep (P = 128), GB/s table
 
 The default workload is the largest one that fits one GPU: 32 learners of the
 ImageNet-shaped MLP 12288 -> 4096 -> 4096 -> 1000 (about 71M parameters each).
@@ -58,6 +58,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mlp4096")
     ap.add_argument("--sweep", action="store_true")
+    ap.add_argument("--sweep-D", type=int, nargs="+", default=None,
+                    help="parameter counts of the sweep (default: 1M, 11.2M, 32M, 64M)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-sweep-point", action="store_true",
@@ -558,7 +560,7 @@ def run_sweep(args):
     pk, src = peaks()
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     torch.manual_seed(0)
-    for D in sw.D:
+    for D in args.sweep_D or sw.D:
         w = torch.randn(sw.P, D, device="cuda")
         by = 8.0 * sw.P * D
         for op, S in [("global", sw.P)] + [(o, s) for s in sw.S for o in ("local", "local_global")]:
