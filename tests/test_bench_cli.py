@@ -1,9 +1,12 @@
-"""bench.py's command line on the CPU: the reference arm (the oracle timed on the host
-cores) prints one JSON line with the keys the driver reads."""
+"""bench.py on the CPU: the reference arm (the oracle timed on the host cores) prints one
+JSON line with the keys the driver reads; the sampling, extrapolation and roofline
+arithmetic behind the GPU arm's line."""
 import json
 import os
 import subprocess
 import sys
+
+import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
@@ -50,3 +53,37 @@ def test_dominant_kernel_sample_cycles_through_the_round():
         n = bench.dom_sample(per_round)
         assert n >= bench.DOM_SAMPLE and math.gcd(n, per_round) == 1
         assert {(k * n) % per_round for k in range(per_round)} == set(range(per_round))
+
+
+def test_round_extrapolation_of_the_oracle_sample():
+    # A round of the 32-learner ImageNet-shaped workload: P * K1 * K2 = 1024 learner
+    # steps, K2 * P / S = 32 cluster averages and a global average over P rows, which
+    # the sample counts as (P - 1) / (S - 1) cluster averages (a tree over P values
+    # takes P - 1 additions, one over S takes S - 1).
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_1903_05133_gb300 import configs
+    w = configs.MLP4096_P32
+    smp = bench.OracleSample.__new__(bench.OracleSample)
+    smp.w, smp.steps, smp.avg_split = w, 1, 8
+    t_step, t_avg = 0.5, 0.01
+    want = 1024 * t_step + (32 + 31 / 7) * t_avg * 8
+    assert smp.round_seconds(t_step, t_avg) == pytest.approx(want)
+    smp.steps = 4                                    # four steps timed: a quarter each
+    assert smp.round_seconds(4 * t_step, t_avg) == pytest.approx(want)
+
+
+def test_gemm_report_against_the_hbm_bound_ceiling():
+    sys.path.insert(0, ROOT)
+    import bench
+    # 18 flop per byte against a 6790 GB/s copy rate and 1724 TFLOP/s: the HBM roofline
+    # allows 18 * 6.79 = 122.2 TFLOP/s, 0.0709 of the tensor rate
+    by, fl, ms = 1e12, 18e12, 10_000.0               # 1 TB and 18 PFLOP in 10 s
+    r = bench.gemm_report(by, fl, ms, 6790.0, 1724.0)
+    assert r["TFLOPs"] == pytest.approx(1.8, abs=1e-2)
+    assert r["flop_per_byte"] == pytest.approx(18.0)
+    assert r["hbm_bound_tensor_frac_ceiling"] == pytest.approx(18 * 6.79 / 1724, abs=1e-4)
+    assert r["frac_of_hbm_bound_ceiling"] == pytest.approx(1.8 / (18 * 6.79), abs=1e-4)
+    # a compute-bound intensity is capped by the tensor rate itself
+    r = bench.gemm_report(1e9, 1e15, 1000.0, 6790.0, 1724.0)
+    assert r["hbm_bound_tensor_frac_ceiling"] == pytest.approx(1.0)
